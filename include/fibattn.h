@@ -1,0 +1,128 @@
+/*
+ * fibattn.h -- C ABI of the GB300 (sm_103a) library for depth-staggered
+ * scaled-Fibonacci sparse attention (arXiv 2606.28560).
+ *
+ * The operation (Section 2, "Attended set"): query i attends to the dense
+ * causal window at distances 0..W plus K rungs at continuous distances
+ * d_k = alpha * f_k.  A rung is read by linear interpolation between the
+ * floor and floor-plus-one positions; RoPE is applied to q and k at their true
+ * positions before the gather; the attended scores go through a softmax and
+ * weight the (equally interpolated) values.  alpha = 0.5 + sigmoid(theta) is
+ * one scalar per layer (Section 2, "The per-layer scalar").
+ *
+ * Conventions shared by every call:
+ *   - Tensor layouts are row-major and contiguous: q, out, dout, dq are
+ *     [B][H][T][D]; k, v, dk, dv are [B][Hkv][T][D]; lse is [B][H][T] fp32.
+ *     Element type is given by `dtype` (fp32 or bf16); lse is always fp32.
+ *   - Tensor, workspace and output-scalar pointers are DEVICE pointers owned by
+ *     the caller and aligned to 16 bytes.  `offsets` is a HOST array of K floats
+ *     (the base sequence f_k, e.g. 1,2,3,5,...,987) read during the call only.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
+ *     Device work is asynchronous on that stream; a call returns after launch.
+ *   - Return value is a fibattn_status.  Argument errors are reported before
+ *     any launch.  Faults raised asynchronously by the device surface at the
+ *     caller's next synchronisation.  fibattn_last_error() gives a thread-local
+ *     message for the last non-OK status.  No C++ exception crosses the ABI.
+ *   - Limits: D == 64; 0 <= W <= 1024; 0 <= K <= 32; 1 <= T <= 2^20;
+ *     0.5 <= alpha <= 1.5; every d_k = fl32(alpha * f_k) must be finite and
+ *     >= 0; H % Hkv == 0.
+ *   - Readings of the paper taken where it is silent: scale = 1/sqrt(D); the
+ *     floor is taken of the distance, the far row i-floor(d)-1 has weight
+ *     d-floor(d); a rung with d_k > i is masked; with dedup a rung with
+ *     d_k <= W is dropped (the attended set is a set union); RoPE pairs
+ *     dimension m with m+D/2 at frequency rope_base^(-2m/D).
+ */
+#ifndef FIBATTN_H
+#define FIBATTN_H
+
+#include <stddef.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    FIBATTN_OK = 0,
+    FIBATTN_ERR_INVALID_ARG = 1,   /* bad shape, pointer, alignment, alpha, ...   */
+    FIBATTN_ERR_UNSUPPORTED = 2,   /* valid but not built (e.g. D != 64)           */
+    FIBATTN_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed         */
+    FIBATTN_ERR_INTERNAL = 4       /* an internal consistency check failed         */
+} fibattn_status;
+
+typedef enum { FIBATTN_F32 = 0, FIBATTN_BF16 = 1 } fibattn_dtype;
+
+/* Options.  Zero-initialised fields take the defaults in brackets. */
+typedef struct {
+    float rope_base;   /* RoPE frequency base [1e4] (Section 3, "Model and training") */
+    float scale;       /* score scale; <= 0 means 1/sqrt(D)                            */
+    int   Hkv;         /* key/value heads (GQA); 0 means Hkv = H                       */
+    int   no_dedup;    /* 0: drop rungs with d_k <= W [default]; 1: keep them          */
+} fibattn_opts;
+
+/* ---------------------------------------------------------------------------
+ * Forward: out[b,h,i,:] and lse[b,h,i] (log of the softmax normaliser, in the
+ * scaled-score domain) for every query (Section 2, "Attended set").
+ * workspace: device scratch of at least fibattn_fwd_workspace_bytes(...)
+ * bytes; contents on entry are ignored and on exit are unspecified.
+ * out may not alias q, k, v or workspace.
+ * ------------------------------------------------------------------------- */
+size_t fibattn_fwd_workspace_bytes(int B, int H, int T, int D, int W, int K,
+                                   int dtype, const fibattn_opts* opts);
+
+int fibattn_fwd(const void* q, const void* k, const void* v,
+                void* out, float* lse,
+                int B, int H, int T, int D, int W,
+                float alpha, const float* offsets, int K,
+                int dtype, const fibattn_opts* opts,
+                void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Backward (the chain rule of the forward definition; the paper trains every
+ * model through this path, Section 2 "Implementation note").
+ * Inputs: q, k, v, dout as above and lse from fibattn_fwd of the same inputs.
+ * Outputs (overwritten, not accumulated): dq [B,H,T,D], dk and dv [B,Hkv,T,D]
+ * in `dtype`, gradients with respect to the pre-RoPE q and k; dtheta (device,
+ * 1 float) = dL/dtheta with alpha = 0.5 + sigmoid(theta); dd (device, K floats,
+ * may be NULL) = dL/dd_k for each rung distance.  dL/dalpha = sum_k f_k dd_k.
+ * At an integer d_k the distance derivative is one-sided, from above.
+ * ------------------------------------------------------------------------- */
+size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K,
+                                   int dtype, const fibattn_opts* opts);
+
+int fibattn_bwd(const void* q, const void* k, const void* v,
+                const float* lse, const void* dout,
+                void* dq, void* dk, void* dv, float* dtheta, float* dd,
+                int B, int H, int T, int D, int W,
+                float alpha, const float* offsets, int K,
+                int dtype, const fibattn_opts* opts,
+                void* workspace, size_t workspace_bytes, void* stream);
+
+/* Thread-local message for the last non-OK status returned on this thread. */
+const char* fibattn_last_error(void);
+
+/* ---------------------------------------------------------------------------
+ * Host-side parameter prep (no GPU needed).
+ * ------------------------------------------------------------------------- */
+
+/* Rung prep (Section 2): d[k] = fl32(alpha * f[k]); s0[k] = floor(d[k]);
+ * w[k] = d[k] - s0[k]; active[k] = 1 unless dedup drops it (d[k] <= W).
+ * Any output pointer may be NULL.  Host pointers. */
+int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup,
+                        float* d, int* s0, float* w, int* active);
+
+/* Base sequences (Section 2): kind 0 = Fibonacci 1,2,3,5,... ; kind 1 =
+ * powers of two 1,2,4,... .  Writes K floats to host array f. */
+int fibattn_base(int kind, int K, float* f);
+
+/* Per-layer alpha schedules (Section 2, "The per-layer scalar"):
+ * kind 0 fixed (alpha = 1); 1 learned (alpha_l = 0.5 + sigmoid(theta[l]));
+ * 2 linear stagger (alpha_l = 0.5 + l/(L-1)); 3 coprime reassignment of the
+ * linear multiset, layer l takes linear index (stride*l mod L).
+ * theta is read only for kind 1.  Host arrays. */
+int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, float* alpha);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* FIBATTN_H */
