@@ -1,0 +1,460 @@
+"""Benchmark: depth-staggered scaled-Fibonacci sparse attention on GB300.
+
+Default workload (one "step" = the whole hot path over one batch): 16 layers
+of forward + backward, B=16, H=8, T=1024, D=64, W=8, Fibonacci base K=15,
+learned schedule alpha_l = 0.5 + sigmoid(theta_l) with theta_l ~ N(0, 0.5),
+bf16 I/O with fp32 accumulation, distinct per-layer buffers (1.07 GB of
+inputs per step, larger than L2).  Metric: query-heads per second (B*H*T per
+layer per fwd+bwd), with the achieved HBM bandwidth of the dominant kernel
+against the measured GB300 copy bandwidth.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gb300|reference]
+
+Under torchrun each rank runs its own copy of the workload on its own GPU
+(weak scaling, replicas only: the path has no exchange step); rank 0 prints
+one JSON line.  ``--impl reference`` times the fp64 CPU oracle on a bounded
+sample of the same workload (the paper ships no code to run).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+METRIC = "queries/s and achieved HBM GB/s (% of GB300 roofline), fwd+bwd, T=1024"
+UNIT = "query-heads/s"
+B, H, T, D, W, L, K = 16, 8, 1024, 64, 8, 16, 15
+SEED = 3                      # learned-alpha backward workload
+ESIZE = 2                     # bf16
+ROW_BYTES = D * ESIZE
+
+
+def workload_config():
+    return {"workload": "fwd+bwd, 16 layers, learned alpha (theta_l ~ N(0,0.5)), Fibonacci K=15",
+            "B": B, "H": H, "Hkv": H, "T": T, "D": D, "W": W, "layers": L, "K": K, "seed": SEED,
+            "io": "bf16, fp32 accumulate",
+            "l2": "inputs larger than L2: distinct per-layer buffers, 1.07 GB of inputs per step"}
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            p = json.load(fh)
+        return float(p["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+# ------------------------------------------------------------------ clocks --
+
+class ClockSampler:
+    """nvidia-smi clock/throttle sampling during the timed region."""
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+        self.t0 = self.t1 = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append((time.time(), line.strip()))
+
+    def mark(self, which):
+        setattr(self, which, time.time())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for ts, line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            rows.append((ts, parts))
+        inside = [r for ts, r in rows if self.t0 and self.t1 and self.t0 - 0.15 <= ts <= self.t1 + 0.15] or \
+            [r for _, r in rows]
+        if not inside:
+            return None
+
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+
+        sm = [num(r[1]) for r in inside if num(r[1]) is not None]
+        mx = [num(r[2]) for r in inside if num(r[2]) is not None]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in inside for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(inside)}
+
+
+# ------------------------------------------------------------ GPU workload --
+
+class Workload:
+    def __init__(self, device, seed_base=SEED, layers=L):
+        import paper_2606_28560_gb300 as fa
+        from paper_2606_28560_gb300 import inputs
+        self.fa = fa
+        self.dev = device
+        self.L = layers
+        theta = inputs.theta_learned(L, seed=SEED)
+        self.alphas = [float(a) for a in fa.alpha_schedule("learned", L, theta=theta)]
+        self.f = fa.base("fib", K)
+        shp = (B, H, T, D)
+        bf = torch.bfloat16
+        self.q, self.k, self.v, self.g = [], [], [], []
+        for l in range(layers):
+            s = inputs.layer_seed(seed_base, l)
+            ts = [torch.empty(shp, dtype=bf, device=device) for _ in range(4)]
+            for j, t in enumerate(ts):
+                inputs.device_normal_(t, s * 10 + j)
+            self.q.append(ts[0]); self.k.append(ts[1]); self.v.append(ts[2]); self.g.append(ts[3])
+        self.out = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
+        self.lse = [torch.empty((B, H, T), dtype=torch.float32, device=device) for _ in range(layers)]
+        self.dq = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
+        self.dk = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
+        self.dv = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
+        self.dth = torch.zeros((layers, 4), dtype=torch.float32, device=device)
+        self.dd = torch.zeros((layers, 32), dtype=torch.float32, device=device)
+        self.ws_f = torch.empty(fa.fwd_workspace_bytes(B, H, T, W, K, bf), dtype=torch.uint8, device=device)
+        self.ws_b = torch.empty(fa.bwd_workspace_bytes(B, H, T, W, K, bf), dtype=torch.uint8, device=device)
+        self.launches_per_step = layers * (2 + 5)
+
+    def step(self):
+        fa = self.fa
+        for l in range(self.L):
+            fa.fwd(self.q[l], self.k[l], self.v[l], self.alphas[l], self.f, W, out=self.out[l], lse=self.lse[l],
+                   workspace=self.ws_f)
+        for l in reversed(range(self.L)):
+            fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], self.alphas[l], self.f, W,
+                   dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], dtheta=self.dth[l], dd=self.dd[l],
+                   workspace=self.ws_b)
+
+    def fwd_only(self, W_):
+        fa = self.fa
+        for l in range(self.L):
+            fa.fwd(self.q[l], self.k[l], self.v[l], self.alphas[l], self.f, W_, out=self.out[l], lse=self.lse[l],
+                   workspace=self.ws_f)
+
+
+def algorithmic_bytes():
+    """Bytes each kernel must move once per launch (bf16 rows of 128 B,
+    fp32 lse and fp32 P / dS slots).  S = W + 1 + K slots per query."""
+    n = B * H * T
+    S = W + 1 + K
+    rows = n * ROW_BYTES
+    return {
+        "fwd": 4 * rows + 4 * n,                           # Q, K~, V read; O written; lse
+        "rope_k": 2 * rows, "rope_q": 2 * rows,            # read, write rotated
+        "bwd_query": 5 * rows + 4 * n + 2 * 4 * n * S,     # Q~ K~ V dO read, dQ written, lse, P/dS written
+        "bwd_key": 4 * rows + 2 * 4 * n * S,               # Q~ dO read, dK dV written, P/dS read
+        "bwd_finalize": 0,
+    }
+
+
+def run_gpu(args, rank, world, device):
+    import paper_2606_28560_gb300 as fa
+    from paper_2606_28560_gb300.binding import profile_enable, profile_summary
+
+    dist = world > 1
+    wl = Workload(device)
+    stream = torch.cuda.current_stream(device)
+    for _ in range(args.warmup):
+        wl.step()
+    torch.cuda.synchronize(device)
+
+    def barrier():
+        if dist:
+            torch.distributed.barrier()
+
+    clocks = ClockSampler(int(os.environ.get("LOCAL_RANK", "0")) if dist else device.index or 0)
+    if rank == 0:
+        clocks.start()
+        time.sleep(0.3)
+    profile_enable(True)
+    barrier()
+    torch.cuda.synchronize(device)
+    clocks.mark("t0")
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        wl.step()
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    clocks.mark("t1")
+    barrier()
+    ms = e0.elapsed_time(e1)
+    prof = profile_summary()
+    profile_enable(False)
+    clk = clocks.stop() if rank == 0 else None
+
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    if dist:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    ms_max = float(t.item())
+    queries = world * args.steps * L * B * H * T
+    value = queries / (ms_max / 1e3)
+
+    # roofline of the dominant kernel (largest share of device time)
+    hbm, peak_kind = peaks()
+    algo = algorithmic_bytes()
+    tot = sum(v[0] for v in prof.values()) or 1.0
+    dom = max(prof.items(), key=lambda kv: kv[1][0])[0] if prof else "fwd"
+    dms, dcnt = prof.get(dom, (0.0, 1))
+    avg_s = dms / max(dcnt, 1) / 1e3
+    achieved = algo.get(dom, 0) / avg_s / 1e9 if avg_s > 0 else 0.0
+    kernels = {k: {"ms_total": round(v[0], 4), "launches": v[1], "share": round(v[0] / tot, 4),
+                   "us_per_launch": round(v[0] / max(v[1], 1) * 1e3, 2),
+                   "algo_GBps": round(algo.get(k, 0) / (v[0] / max(v[1], 1) / 1e3) / 1e9, 1) if v[0] > 0 else None}
+               for k, v in prof.items()}
+
+    # forward-only at the same shape (W sweep): per-layer fwd kernel time
+    fwd_sweep = {}
+    for W_ in (6, 8, 10, 12):
+        wl.fwd_only(W_)
+        torch.cuda.synchronize(device)
+        profile_enable(True)
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        reps = max(3, args.steps // 4)
+        for _ in range(reps):
+            wl.fwd_only(W_)
+        a1.record(stream)
+        torch.cuda.synchronize(device)
+        p = profile_summary()
+        profile_enable(False)
+        fms, fcnt = p.get("fwd", (0.0, 1))
+        us = fms / max(fcnt, 1) * 1e3
+        layer_us = a0.elapsed_time(a1) / (reps * L) * 1e3
+        fwd_sweep[f"W{W_}"] = {"fwd_kernel_us": round(us, 2), "layer_us_incl_rope": round(layer_us, 2),
+                               "compulsory_GBps": round(4 * B * H * T * ROW_BYTES / (layer_us * 1e-6) / 1e9, 1),
+                               "frac_of_hbm": round(4 * B * H * T * ROW_BYTES / (layer_us * 1e-6) / 1e9 / hbm, 4)}
+
+    e2e = run_e2e(args, wl, device, dist)
+    return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
+                algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=wl.launches_per_step * args.steps)
+
+
+def run_e2e(args, wl, device, dist):
+    """Same step through the public API with host buffers: every step copies
+    its inputs (q, k, v, dout of all layers) from pinned host memory and reads
+    the results (out, dq, dk, dv, dtheta of all layers) back to pinned host
+    memory, inside the timed region."""
+    n_in = 4 * L
+    host_in = [torch.empty((B, H, T, D), dtype=torch.bfloat16, pin_memory=True) for _ in range(n_in)]
+    for i, h in enumerate(host_in):
+        src = (wl.q, wl.k, wl.v, wl.g)[i % 4][i // 4]
+        h.copy_(src)
+    host_out = [torch.empty((B, H, T, D), dtype=torch.bfloat16, pin_memory=True) for _ in range(4 * L)]
+    host_th = torch.empty((L, 4), dtype=torch.float32, pin_memory=True)
+    stream = torch.cuda.current_stream(device)
+    steps = max(2, min(args.steps, 10))
+
+    def one():
+        for i, h in enumerate(host_in):
+            dst = (wl.q, wl.k, wl.v, wl.g)[i % 4][i // 4]
+            dst.copy_(h, non_blocking=True)
+        wl.step()
+        for l in range(L):
+            host_out[4 * l].copy_(wl.out[l], non_blocking=True)
+            host_out[4 * l + 1].copy_(wl.dq[l], non_blocking=True)
+            host_out[4 * l + 2].copy_(wl.dk[l], non_blocking=True)
+            host_out[4 * l + 3].copy_(wl.dv[l], non_blocking=True)
+        host_th.copy_(wl.dth, non_blocking=True)
+
+    one()
+    torch.cuda.synchronize(device)
+    if dist:
+        torch.distributed.barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    torch.cuda.synchronize(device)
+    ms = e0.elapsed_time(e1)
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    if dist:
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    world = torch.distributed.get_world_size() if dist else 1
+    value = world * steps * L * B * H * T / (float(t.item()) / 1e3)
+    bi = n_in * B * H * T * ROW_BYTES
+    bo = 4 * L * B * H * T * ROW_BYTES + L * 4 * 4
+    return {"value": value, "unit": UNIT, "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo}
+
+
+# ------------------------------------------------------------- CPU oracle --
+
+def oracle_sample(seconds_target=10.0, nthreads=None):
+    """Time the fp64 oracle (as it stands) on a bounded sample of the
+    workload: fwd + bwd of whole layers (B=16, H=8, T=1024 each), layer after
+    layer, until about ``seconds_target`` of wall time has been spent."""
+    import oracle as O
+    from paper_2606_28560_gb300 import inputs
+    nthreads = nthreads or (os.cpu_count() or 1)
+    theta = inputs.theta_learned(L, seed=SEED)
+    alphas = O.alpha_schedule("learned", L, theta=theta)
+    f = O.fib_base(K)
+    done_q, spent, layers = 0, 0.0, 0
+    while spent < seconds_target and layers < L:
+        s = inputs.layer_seed(SEED, layers)
+        q, k, v = inputs.qkv(B, H, T, seed=s, dtype=torch.bfloat16)
+        g = inputs.dout(B, H, T, seed=s, dtype=torch.bfloat16)
+        q, k, v, g = (x.double().numpy() for x in (q, k, v, g))
+        d = O.offsets_fp32(float(np.float32(alphas[layers])), f)
+        t0 = time.perf_counter()
+        O.forward(q, k, v, W, d, nthreads=nthreads)
+        O.backward(q, k, v, g, W, d, nthreads=nthreads)
+        spent += time.perf_counter() - t0
+        done_q += B * H * T
+        layers += 1
+    return {"value": done_q / spent, "unit": UNIT, "cores": nthreads, "kind": "oracle",
+            "sample": f"{layers} full layer(s) fwd+bwd (B=16 H=8 T=1024 each, {done_q} query-heads), "
+                      f"fp64 C oracle, {spent:.1f} s wall on {nthreads} threads"}
+
+
+def run_reference(args, rank, world):
+    """Reference arm: the fp64 CPU oracle, timed as it stands on the host
+    cores; each step is a bounded sample (one layer fwd+bwd or part of one)."""
+    if rank != 0:
+        return
+    nthreads = os.cpu_count() or 1
+    per_step = []
+    budget = max(1.0, 60.0 / max(args.steps + args.warmup, 1))
+    for i in range(args.warmup + args.steps):
+        r = oracle_sample(seconds_target=budget, nthreads=nthreads)
+        if i >= args.warmup:
+            per_step.append(r["value"])
+    value = statistics.median(per_step)
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic N(0,1), seeded",
+            "config": workload_config(),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": nthreads, "kind": "oracle",
+                             "sample": r["sample"] + " (per step)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------- ncu cases --
+
+def ncu_case(which: str):
+    """A small fixed case for ncu captures of one kernel: B=32 H=8 T=1024 W=8,
+    two layers of distinct buffers (Q, K, V, O of one layer = 134 MB, larger
+    than L2), one forward (and backward) per layer after one warm-up pass."""
+    import __graft_entry__
+    __graft_entry__.build()
+    import paper_2606_28560_gb300 as fa
+    from paper_2606_28560_gb300 import inputs
+    dev = torch.device("cuda", 0)
+    Bc, layers = 32, 2
+    f = fa.base("fib", K)
+    bufs = []
+    for l in range(layers):
+        ts = [torch.empty((Bc, H, T, D), dtype=torch.bfloat16, device=dev) for _ in range(4)]
+        for j, t in enumerate(ts):
+            inputs.device_normal_(t, 1000 + 10 * l + j)
+        bufs.append(ts)
+    for rep in range(2):
+        for l, (q, k, v, g) in enumerate(bufs):
+            out, lse = fa.fwd(q, k, v, 0.8 + 0.1 * l, f, W)
+            if which == "bwd":
+                fa.bwd(q, k, v, lse, g, 0.8 + 0.1 * l, f, W)
+    torch.cuda.synchronize(dev)
+    print(f"ncu case {which} done")
+
+
+# -------------------------------------------------------------------- main --
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--ncu-case", choices=["fwd", "bwd"], default=None,
+                    help="run a small fixed case for an ncu capture and exit")
+    args = ap.parse_args()
+    if args.ncu_case:
+        ncu_case(args.ncu_case)
+        return
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+
+    import __graft_entry__
+    __graft_entry__.build()
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    if world > 1:
+        torch.distributed.init_process_group("nccl", device_id=device)
+    if args.warmup < 3:
+        args.warmup = 3
+    r = run_gpu(args, rank, world, device)
+    if rank == 0:
+        cpu = None
+        if not args.no_cpu_baseline and world == 1:
+            cpu = oracle_sample(seconds_target=10.0)
+        line = {
+            "metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": r["ms"] / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic N(0,1), seeded",
+            "config": workload_config(),
+            "roofline": {"bound": "hbm", "kernel": r["dom"], "achieved": round(r["achieved"], 1),
+                         "peak": r["hbm"], "unit": "GB/s", "frac": round(r["achieved"] / r["hbm"], 4),
+                         "traffic": None, "peak_source": r["peak_kind"],
+                         "algorithmic_bytes_per_launch": r["algo"].get(r["dom"])},
+            "kernels": r["kernels"],
+            "forward_only_B16H8T1024": r["fwd_sweep"],
+            "cpu_baseline": cpu,
+            "e2e": r["e2e"],
+            "gpu_launches": r["launches"],
+            "clocks": r["clk"],
+        }
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

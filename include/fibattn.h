@@ -121,6 +121,17 @@ int fibattn_base(int kind, int K, float* f);
  * theta is read only for kind 1.  Host arrays. */
 int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, float* alpha);
 
+/* ---------------------------------------------------------------------------
+ * Opt-in kernel timing (no counterpart in the paper; used to attribute time
+ * to kernels).  fibattn_profile_enable(1) clears the record and brackets every
+ * later launch with CUDA events on the launch stream; (0) stops and clears.
+ * fibattn_profile_summary(-1, ...) returns the number of distinct kernels
+ * recorded; with index i >= 0 it synchronises on those events and writes the
+ * kernel name, its summed device time in ms and its launch count.
+ * ------------------------------------------------------------------------- */
+int fibattn_profile_enable(int on);
+int fibattn_profile_summary(int index, char* name, int name_len, double* total_ms, int* launches);
+
 #ifdef __cplusplus
 }
 #endif

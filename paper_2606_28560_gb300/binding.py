@@ -1,0 +1,225 @@
+"""Thin ctypes binding of the C ABI in ``include/fibattn.h``.
+
+Argument marshalling only: tensors are passed as raw device pointers with the
+caller's current CUDA stream; every step of the computation runs in the CUDA
+library.  The binding raises ``RuntimeError`` when the library is missing or
+a call returns a non-OK status -- there is no fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import numpy as np
+import torch
+
+from . import build as _build
+
+FIBATTN_F32 = 0
+FIBATTN_BF16 = 1
+_STATUS = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "CUDA", 4: "INTERNAL"}
+
+_lock = threading.Lock()
+_lib = None
+
+
+class FibattnError(RuntimeError):
+    def __init__(self, status: int, message: str):
+        super().__init__(f"fibattn {_STATUS.get(status, status)}: {message}")
+        self.status = status
+
+
+class Opts(ctypes.Structure):
+    _fields_ = [("rope_base", ctypes.c_float), ("scale", ctypes.c_float),
+                ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int)]
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def lib():
+    """Load the CUDA library (it must have been built: ``__graft_entry__.build()``)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = _build.LIB
+            if not os.path.exists(path):
+                raise RuntimeError(f"CUDA library not built ({path} missing); run __graft_entry__.build()")
+            L = ctypes.CDLL(path)
+            vp, sz, ci, cf = ctypes.c_void_p, ctypes.c_size_t, ctypes.c_int, ctypes.c_float
+            fp = ctypes.POINTER(ctypes.c_float)
+            ip = ctypes.POINTER(ctypes.c_int)
+            op = ctypes.POINTER(Opts)
+            L.fibattn_fwd_workspace_bytes.argtypes = [ci] * 7 + [op]
+            L.fibattn_fwd_workspace_bytes.restype = sz
+            L.fibattn_fwd.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, fp, ci, ci, op, vp, sz, vp]
+            L.fibattn_fwd.restype = ci
+            L.fibattn_bwd_workspace_bytes.argtypes = [ci] * 7 + [op]
+            L.fibattn_bwd_workspace_bytes.restype = sz
+            L.fibattn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, fp, ci, ci, op,
+                                      vp, sz, vp]
+            L.fibattn_bwd.restype = ci
+            L.fibattn_last_error.argtypes = []
+            L.fibattn_last_error.restype = ctypes.c_char_p
+            L.fibattn_rung_params.argtypes = [cf, fp, ci, ci, ci, fp, ip, fp, ip]
+            L.fibattn_rung_params.restype = ci
+            L.fibattn_base.argtypes = [ci, ci, fp]
+            L.fibattn_base.restype = ci
+            L.fibattn_alpha_schedule.argtypes = [ci, ci, fp, ci, fp]
+            L.fibattn_alpha_schedule.restype = ci
+            _lib = L
+    return _lib
+
+
+def _check(rc: int):
+    if rc != 0:
+        raise FibattnError(rc, lib().fibattn_last_error().decode(errors="replace"))
+
+
+def _fptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+
+
+def _iptr(a: np.ndarray):
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
+
+
+def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True) -> Opts:
+    return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1)
+
+
+def _dtype_code(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return FIBATTN_F32
+    if t.dtype == torch.bfloat16:
+        return FIBATTN_BF16
+    raise TypeError(f"unsupported dtype {t.dtype}: fp32 or bf16")
+
+
+def _stream_ptr(stream) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream)
+
+
+def _offsets(offsets) -> np.ndarray:
+    return np.ascontiguousarray(np.asarray(offsets, dtype=np.float32))
+
+
+# ------------------------------------------------------------- host prep ----
+
+def base(kind: str, K: int) -> np.ndarray:
+    f = np.zeros(K, dtype=np.float32)
+    _check(lib().fibattn_base({"fib": 0, "pow2": 1}[kind], K, _fptr(f)))
+    return f
+
+
+def alpha_schedule(kind: str, L: int = 16, theta=None, stride: int = 7) -> np.ndarray:
+    code = {"fixed": 0, "learned": 1, "linear": 2, "coprime": 3}[kind]
+    out = np.zeros(L, dtype=np.float32)
+    th = np.ascontiguousarray(np.asarray(theta, dtype=np.float32)) if theta is not None else None
+    _check(lib().fibattn_alpha_schedule(code, L, _fptr(th) if th is not None else None, stride, _fptr(out)))
+    return out
+
+
+def rung_params(alpha: float, offsets, W: int, dedup: bool = True):
+    f = _offsets(offsets)
+    K = len(f)
+    d = np.zeros(K, np.float32); w = np.zeros(K, np.float32)
+    s0 = np.zeros(K, np.int32); act = np.zeros(K, np.int32)
+    _check(lib().fibattn_rung_params(float(alpha), _fptr(f), K, int(W), 0 if dedup else 1,
+                                     _fptr(d), _iptr(s0), _fptr(w), _iptr(act)))
+    return dict(d=d, s0=s0, w=w, active=act.astype(bool))
+
+
+# --------------------------------------------------------------- compute ----
+
+def fwd_workspace_bytes(B, H, T, W, K, dtype, Hkv=None, D=64) -> int:
+    o = _opts(Hkv=Hkv)
+    code = FIBATTN_BF16 if dtype == torch.bfloat16 else FIBATTN_F32
+    return int(lib().fibattn_fwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
+
+
+def bwd_workspace_bytes(B, H, T, W, K, dtype, Hkv=None, D=64) -> int:
+    o = _opts(Hkv=Hkv)
+    code = FIBATTN_BF16 if dtype == torch.bfloat16 else FIBATTN_F32
+    return int(lib().fibattn_bwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
+
+
+def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
+        out=None, lse=None, workspace=None, stream=None):
+    """Forward pass.  q [B,H,T,64]; k, v [B,Hkv,T,64] (fp32 or bf16, CUDA,
+    contiguous).  Returns (out, lse)."""
+    B, H, T, D = q.shape
+    Hkv = k.shape[1]
+    f = _offsets(offsets)
+    o = _opts(rope_base, scale, Hkv, dedup)
+    code = _dtype_code(q)
+    for t in (q, k, v):
+        if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
+            raise ValueError("q, k, v must be contiguous CUDA tensors of one dtype")
+    if out is None:
+        out = torch.empty_like(q)
+    if lse is None:
+        lse = torch.empty((B, H, T), dtype=torch.float32, device=q.device)
+    need = int(lib().fibattn_fwd_workspace_bytes(B, H, T, D, W, len(f), code, ctypes.byref(o)))
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
+    _check(lib().fibattn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), lse.data_ptr(),
+                             B, H, T, D, int(W), float(alpha), _fptr(f), len(f), code, ctypes.byref(o),
+                             workspace.data_ptr(), workspace.numel(), _stream_ptr(stream)))
+    return out, lse
+
+
+def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
+        dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None):
+    """Backward pass.  Returns (dq, dk, dv, dtheta [1], dd [K]) on the device."""
+    B, H, T, D = q.shape
+    Hkv = k.shape[1]
+    f = _offsets(offsets)
+    K = len(f)
+    o = _opts(rope_base, scale, Hkv, dedup)
+    code = _dtype_code(q)
+    for t in (q, k, v, dout):
+        if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
+            raise ValueError("q, k, v, dout must be contiguous CUDA tensors of one dtype")
+    dq = torch.empty_like(q) if dq is None else dq
+    dk = torch.empty_like(k) if dk is None else dk
+    dv = torch.empty_like(v) if dv is None else dv
+    dtheta = torch.empty(4, dtype=torch.float32, device=q.device) if dtheta is None else dtheta
+    dd = torch.empty(max(K, 1), dtype=torch.float32, device=q.device) if dd is None else dd
+    need = int(lib().fibattn_bwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
+    if workspace is None:
+        workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
+    _check(lib().fibattn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), lse.data_ptr(), dout.data_ptr(),
+                             dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), dtheta.data_ptr(), dd.data_ptr(),
+                             B, H, T, D, int(W), float(alpha), _fptr(f), K, code, ctypes.byref(o),
+                             workspace.data_ptr(), workspace.numel(), _stream_ptr(stream)))
+    return dq, dk, dv, dtheta[:1], dd[:K]
+
+
+# ------------------------------------------------------------- profiling ----
+
+def profile_enable(on: bool = True):
+    L = lib()
+    L.fibattn_profile_enable.argtypes = [ctypes.c_int]
+    L.fibattn_profile_enable.restype = ctypes.c_int
+    _check(L.fibattn_profile_enable(1 if on else 0))
+
+
+def profile_summary() -> dict:
+    """{kernel name: (total device ms, launches)} for launches since enable."""
+    L = lib()
+    L.fibattn_profile_summary.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_int,
+                                          ctypes.POINTER(ctypes.c_double), ctypes.POINTER(ctypes.c_int)]
+    L.fibattn_profile_summary.restype = ctypes.c_int
+    n = L.fibattn_profile_summary(-1, None, 0, None, None)
+    out = {}
+    for i in range(n):
+        buf = ctypes.create_string_buffer(64)
+        ms = ctypes.c_double()
+        cnt = ctypes.c_int()
+        _check(L.fibattn_profile_summary(i, buf, 64, ctypes.byref(ms), ctypes.byref(cnt)))
+        out[buf.value.decode()] = (ms.value, cnt.value)
+    return out

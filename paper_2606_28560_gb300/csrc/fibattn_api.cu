@@ -1,0 +1,373 @@
+// fibattn_api.cu -- the C ABI declared in include/fibattn.h: argument checks,
+// host-side parameter prep (rung distances, RoPE phase increments),
+// workspace layout, and the launches.  arXiv 2606.28560, Section 2.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <cstdint>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/fibattn.h"
+#include "fibattn_internal.cuh"
+
+using namespace fibattn;
+
+namespace {
+
+thread_local std::string g_err;
+
+int fail(int code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return code;
+}
+
+size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+size_t elem_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
+// rotated q/k rows in the workspace: fp32 (fp32 I/O) or fp16 (bf16 I/O)
+size_t rot_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
+
+struct Resolved {
+    float rope_base, scale;
+    int Hkv, dedup;
+};
+
+int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
+    r->rope_base = (o && o->rope_base != 0.f) ? o->rope_base : 1e4f;
+    r->scale = (o && o->scale > 0.f) ? o->scale : (float)(1.0 / std::sqrt((double)D));
+    r->Hkv = (o && o->Hkv > 0) ? o->Hkv : H;
+    r->dedup = (o && o->no_dedup) ? 0 : 1;
+    if (!(r->rope_base > 1.f) || !std::isfinite(r->rope_base))
+        return fail(FIBATTN_ERR_INVALID_ARG, "rope_base must be finite and > 1 (got %g)", (double)r->rope_base);
+    if (!std::isfinite(r->scale)) return fail(FIBATTN_ERR_INVALID_ARG, "scale must be finite");
+    if (r->Hkv <= 0 || H % r->Hkv) return fail(FIBATTN_ERR_INVALID_ARG, "H (%d) must be a multiple of Hkv (%d)", H, r->Hkv);
+    return FIBATTN_OK;
+}
+
+int check_shape(int B, int H, int T, int D, int W, int K, int dtype) {
+    if (dtype != FIBATTN_F32 && dtype != FIBATTN_BF16) return fail(FIBATTN_ERR_INVALID_ARG, "unknown dtype %d", dtype);
+    if (B < 0 || H <= 0 || T < 1 || T > (1 << 20)) return fail(FIBATTN_ERR_INVALID_ARG, "bad shape B=%d H=%d T=%d", B, H, T);
+    if (D != kHeadDim) return fail(FIBATTN_ERR_UNSUPPORTED, "only D == %d is built (got %d)", kHeadDim, D);
+    if (W < 0 || W > kMaxWindow) return fail(FIBATTN_ERR_INVALID_ARG, "W must be in [0, %d] (got %d)", kMaxWindow, W);
+    if (K < 0 || K > kMaxRungs) return fail(FIBATTN_ERR_INVALID_ARG, "K must be in [0, %d] (got %d)", kMaxRungs, K);
+    if ((long long)B * H * T > (1LL << 31) / 64) return fail(FIBATTN_ERR_INVALID_ARG, "B*H*T too large");
+    return FIBATTN_OK;
+}
+
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// Section 2: d_k = alpha f_k, rounded once to fp32; s0 = floor(d_k), w = d_k - s0.
+int prep_rungs(float alpha, const float* f, int K, int W, int dedup, int T, RungParams* r) {
+    if (!(alpha >= 0.5f && alpha <= 1.5f)) return fail(FIBATTN_ERR_INVALID_ARG, "alpha must be in [0.5, 1.5] (got %g)", (double)alpha);
+    if (K > 0 && !f) return fail(FIBATTN_ERR_INVALID_ARG, "offsets is NULL");
+    std::memset(r, 0, sizeof(*r));
+    r->K = K;
+    for (int k = 0; k < K; ++k) {
+        if (!std::isfinite(f[k]) || f[k] < 0.f) return fail(FIBATTN_ERR_INVALID_ARG, "offsets[%d] must be finite and >= 0", k);
+        volatile float d = alpha * f[k];        // one fp32 rounding
+        if (!std::isfinite(d)) return fail(FIBATTN_ERR_INVALID_ARG, "alpha*offsets[%d] overflows", k);
+        r->f[k] = f[k];
+        r->d[k] = d;
+        bool reach = d <= (float)(T - 1);       // otherwise masked for every query
+        bool keep = dedup ? (d > (float)W) : true;
+        if (reach && keep) {
+            float fl = std::floor(d);
+            r->s0[k] = (int)fl;
+            r->w[k] = d - fl;                   // exact in fp32
+            r->active |= 1u << k;
+        } else {
+            r->s0[k] = 0;
+            r->w[k] = 0.f;
+        }
+    }
+    return FIBATTN_OK;
+}
+
+// F[m] = round(2^64 * theta_m / (2 pi)), theta_m = base^(-2m/D)  (fp64 on the host)
+void prep_rope(float base, RopeParams* rp) {
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int m = 0; m < kHalf; ++m) {
+        double theta = std::pow((double)base, -2.0 * m / (double)kHeadDim);
+        double frac = theta / two_pi;           // in (0, 1)
+        long double scaled = std::ldexp((long double)frac, 64);
+        rp->F[m] = (unsigned long long)(scaled + 0.5L);
+    }
+}
+
+Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
+    Shape s;
+    s.B = B; s.H = H; s.Hkv = o.Hkv; s.T = T; s.W = W; s.G = H / o.Hkv; s.scale = o.scale;
+    return s;
+}
+
+struct BwdLayout {
+    size_t qt, kt, P, DS, partial, total;
+    int nblocks;
+};
+
+BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype) {
+    BwdLayout L;
+    size_t es = rot_size(dtype);
+    size_t S = (size_t)W + 1 + K;
+    Shape s; s.B = B; s.H = H; s.Hkv = Hkv; s.T = T; s.W = W; s.G = H / Hkv; s.scale = 1.f;
+    L.nblocks = bwd_simple_blocks(s);
+    size_t off = 0;
+    L.qt = off; off += align256((size_t)B * H * T * kHeadDim * es);
+    L.kt = off; off += align256((size_t)B * Hkv * T * kHeadDim * es);
+    L.P = off; off += align256((size_t)B * H * T * S * 4);
+    L.DS = off; off += align256((size_t)B * H * T * S * 4);
+    L.partial = off; off += align256((size_t)(L.nblocks > 0 ? L.nblocks : 1) * kMaxRungs * 4);
+    L.total = off;
+    return L;
+}
+
+int cuda_fail(cudaError_t e, const char* what) {
+    return fail(FIBATTN_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// ---------------------------------------------------------------- profiler --
+
+struct ProfRecord { std::string name; cudaEvent_t a, b; };
+std::mutex g_prof_mu;
+bool g_prof_on = false;
+std::vector<ProfRecord> g_prof_recs;
+std::vector<cudaEvent_t> g_prof_pool;
+
+cudaEvent_t prof_event() {
+    cudaEvent_t e = nullptr;
+    if (!g_prof_pool.empty()) { e = g_prof_pool.back(); g_prof_pool.pop_back(); return e; }
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+
+}  // namespace
+
+namespace fibattn {
+ProfScope::ProfScope(const char* name, cudaStream_t st) : name_(name), st_(st), start_(nullptr), on_(false) {
+    std::lock_guard<std::mutex> g(g_prof_mu);
+    if (!g_prof_on) return;
+    start_ = prof_event();
+    if (start_ && cudaEventRecord(start_, st_) == cudaSuccess) on_ = true;
+}
+ProfScope::~ProfScope() {
+    if (!on_) return;
+    std::lock_guard<std::mutex> g(g_prof_mu);
+    cudaEvent_t b = prof_event();
+    if (b && cudaEventRecord(b, st_) == cudaSuccess) g_prof_recs.push_back({name_, start_, b});
+}
+}  // namespace fibattn
+
+extern "C" {
+
+int fibattn_profile_enable(int on) {
+    std::lock_guard<std::mutex> g(g_prof_mu);
+    g_prof_on = on != 0;
+    for (auto& r : g_prof_recs) { g_prof_pool.push_back(r.a); g_prof_pool.push_back(r.b); }
+    g_prof_recs.clear();
+    return FIBATTN_OK;
+}
+
+int fibattn_profile_summary(int index, char* name, int name_len, double* total_ms, int* launches) {
+    std::lock_guard<std::mutex> g(g_prof_mu);
+    std::vector<std::string> names;
+    for (auto& r : g_prof_recs) {
+        bool seen = false;
+        for (auto& n : names) seen = seen || n == r.name;
+        if (!seen) names.push_back(r.name);
+    }
+    if (index < 0) return (int)names.size();
+    if (index >= (int)names.size()) return fail(FIBATTN_ERR_INVALID_ARG, "profile index out of range");
+    double tot = 0.0;
+    int cnt = 0;
+    for (auto& r : g_prof_recs) {
+        if (r.name != names[index]) continue;
+        cudaError_t e = cudaEventSynchronize(r.b);
+        if (e != cudaSuccess) return cuda_fail(e, "profile event sync");
+        float ms = 0.f;
+        e = cudaEventElapsedTime(&ms, r.a, r.b);
+        if (e != cudaSuccess) return cuda_fail(e, "profile elapsed time");
+        tot += ms;
+        ++cnt;
+    }
+    if (name && name_len > 0) { std::strncpy(name, names[index].c_str(), name_len - 1); name[name_len - 1] = 0; }
+    if (total_ms) *total_ms = tot;
+    if (launches) *launches = cnt;
+    return FIBATTN_OK;
+}
+
+const char* fibattn_last_error(void) { return g_err.c_str(); }
+
+int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup,
+                        float* d, int* s0, float* w, int* active) {
+    if (K < 0 || K > kMaxRungs) return fail(FIBATTN_ERR_INVALID_ARG, "K must be in [0, %d]", kMaxRungs);
+    if (W < 0) return fail(FIBATTN_ERR_INVALID_ARG, "W must be >= 0");
+    RungParams r;
+    int rc = prep_rungs(alpha, offsets, K, W, no_dedup ? 0 : 1, 1 << 30, &r);
+    if (rc) return rc;
+    for (int k = 0; k < K; ++k) {
+        if (d) d[k] = r.d[k];
+        float fl = std::floor(r.d[k]);
+        if (s0) s0[k] = (int)fl;
+        if (w) w[k] = r.d[k] - fl;
+        if (active) active[k] = (r.active >> k) & 1u;
+    }
+    return FIBATTN_OK;
+}
+
+int fibattn_base(int kind, int K, float* f) {
+    if (!f || K < 0 || K > 64) return fail(FIBATTN_ERR_INVALID_ARG, "bad arguments to fibattn_base");
+    if (kind == 0) {                            // Fibonacci 1, 2, 3, 5, ...
+        double a = 1, b = 2;
+        for (int k = 0; k < K; ++k) { f[k] = (float)a; double n = a + b; a = b; b = n; }
+    } else if (kind == 1) {                     // powers of two
+        for (int k = 0; k < K; ++k) f[k] = std::ldexp(1.f, k);
+    } else {
+        return fail(FIBATTN_ERR_INVALID_ARG, "unknown base kind %d", kind);
+    }
+    return FIBATTN_OK;
+}
+
+int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, float* alpha) {
+    if (!alpha || L < 1) return fail(FIBATTN_ERR_INVALID_ARG, "bad arguments to fibattn_alpha_schedule");
+    for (int l = 0; l < L; ++l) {
+        switch (kind) {
+        case 0: alpha[l] = 1.f; break;
+        case 1:
+            if (!theta) return fail(FIBATTN_ERR_INVALID_ARG, "learned schedule needs theta");
+            alpha[l] = (float)(0.5 + 1.0 / (1.0 + std::exp(-(double)theta[l])));
+            break;
+        case 2: alpha[l] = L > 1 ? (float)(0.5 + (double)l / (L - 1)) : 1.f; break;
+        case 3: {
+            int a = stride, b = L;              // gcd(stride, L) must be 1
+            while (b) { int t = a % b; a = b; b = t; }
+            if (stride <= 0 || a != 1) return fail(FIBATTN_ERR_INVALID_ARG, "stride %d not coprime to L=%d", stride, L);
+            int idx = (int)(((long long)stride * l) % L);
+            alpha[l] = L > 1 ? (float)(0.5 + (double)idx / (L - 1)) : 1.f;
+            break;
+        }
+        default: return fail(FIBATTN_ERR_INVALID_ARG, "unknown schedule kind %d", kind);
+        }
+    }
+    return FIBATTN_OK;
+}
+
+size_t fibattn_fwd_workspace_bytes(int B, int H, int T, int D, int W, int K, int dtype, const fibattn_opts* opts) {
+    Resolved o;
+    if (check_shape(B, H, T, D, W, K, dtype) || resolve_opts(opts, H, D, &o)) return 0;
+    return align256((size_t)B * o.Hkv * T * kHeadDim * rot_size(dtype));
+}
+
+int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* lse,
+                int B, int H, int T, int D, int W, float alpha, const float* offsets, int K,
+                int dtype, const fibattn_opts* opts, void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_shape(B, H, T, D, W, K, dtype);
+    if (rc) return rc;
+    Resolved o;
+    if ((rc = resolve_opts(opts, H, D, &o))) return rc;
+    FwdArgs a;
+    std::memset(&a, 0, sizeof(a));
+    if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
+    if (B == 0) return FIBATTN_OK;
+    if (!q || !k || !v || !out || !lse || !workspace) return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor or workspace pointer");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(lse) || !aligned16(workspace))
+        return fail(FIBATTN_ERR_INVALID_ARG, "tensor pointers must be 16-byte aligned");
+    size_t need = fibattn_fwd_workspace_bytes(B, H, T, D, W, K, dtype, opts);
+    if (workspace_bytes < need) return fail(FIBATTN_ERR_INVALID_ARG, "workspace too small: %zu < %zu", workspace_bytes, need);
+    prep_rope(o.rope_base, &a.rope);
+    a.s = make_shape(B, H, T, W, o);
+    a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.kt = workspace;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const bool bf16 = dtype == FIBATTN_BF16;
+    cudaError_t e;
+    {
+        ProfScope p("rope_k", st);
+        e = launch_rope_rows(k, workspace, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "rope prologue launch");
+    {
+        ProfScope p("fwd", st);
+        e = launch_fwd_simple(a, bf16, st);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "forward launch");
+    return FIBATTN_OK;
+}
+
+size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K, int dtype, const fibattn_opts* opts) {
+    Resolved o;
+    if (check_shape(B, H, T, D, W, K, dtype) || resolve_opts(opts, H, D, &o)) return 0;
+    return bwd_layout(B, H, o.Hkv, T, W, K, dtype).total;
+}
+
+int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, const void* dout,
+                void* dq, void* dk, void* dv, float* dtheta, float* dd,
+                int B, int H, int T, int D, int W, float alpha, const float* offsets, int K,
+                int dtype, const fibattn_opts* opts, void* workspace, size_t workspace_bytes, void* stream) {
+    int rc = check_shape(B, H, T, D, W, K, dtype);
+    if (rc) return rc;
+    Resolved o;
+    if ((rc = resolve_opts(opts, H, D, &o))) return rc;
+    BwdArgs a;
+    std::memset(&a, 0, sizeof(a));
+    if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
+    if (!dtheta) return fail(FIBATTN_ERR_INVALID_ARG, "dtheta is NULL");
+    if (!workspace) return fail(FIBATTN_ERR_INVALID_ARG, "workspace is NULL");
+    if (B > 0 && (!q || !k || !v || !lse || !dout || !dq || !dk || !dv))
+        return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor pointer");
+    if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(lse) || !aligned16(dout) || !aligned16(dq) ||
+        !aligned16(dk) || !aligned16(dv) || !aligned16(workspace) || ((uintptr_t)dtheta & 3u) || ((uintptr_t)dd & 3u))
+        return fail(FIBATTN_ERR_INVALID_ARG, "pointers must be 16-byte aligned (dtheta, dd: 4-byte)");
+    BwdLayout L = bwd_layout(B, H, o.Hkv, T, W, K, dtype);
+    if (workspace_bytes < L.total) return fail(FIBATTN_ERR_INVALID_ARG, "workspace too small: %zu < %zu", workspace_bytes, L.total);
+    prep_rope(o.rope_base, &a.rope);
+    a.s = make_shape(B, H, T, W, o);
+    char* ws = reinterpret_cast<char*>(workspace);
+    a.q = q; a.k = k; a.v = v; a.lse = lse; a.dout = dout; a.dq = dq; a.dk = dk; a.dv = dv;
+    a.dtheta = dtheta; a.dd = dd;
+    a.qt = ws + L.qt; a.kt = ws + L.kt;
+    a.P = reinterpret_cast<float*>(ws + L.P); a.DS = reinterpret_cast<float*>(ws + L.DS);
+    a.partial = reinterpret_cast<float*>(ws + L.partial);
+    a.nblocks_a = B > 0 ? L.nblocks : 0;
+    a.S = W + 1 + K;
+    a.alpha = alpha;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    const bool bf16 = dtype == FIBATTN_BF16;
+    cudaError_t e;
+    if (B > 0) {
+        {
+            ProfScope p("rope_q", st);
+            e = launch_rope_rows(q, a.qt, (long long)B * H * T, T, a.rope, bf16, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "rope prologue (q) launch");
+        {
+            ProfScope p("rope_k", st);
+            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "rope prologue (k) launch");
+        {
+            ProfScope p("bwd_query", st);
+            e = launch_bwd_query(a, bf16, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "backward query-pass launch");
+        {
+            ProfScope p("bwd_key", st);
+            e = launch_bwd_key(a, bf16, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "backward key-pass launch");
+    }
+    {
+        ProfScope p("bwd_finalize", st);
+        e = launch_bwd_finalize(a, st);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "backward finalize launch");
+    return FIBATTN_OK;
+}
+
+}  // extern "C"

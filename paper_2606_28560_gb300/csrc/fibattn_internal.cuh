@@ -1,0 +1,209 @@
+// fibattn_internal.cuh -- shared definitions of the CUDA library (not part of
+// the C ABI).  Depth-staggered scaled-Fibonacci sparse attention,
+// arXiv 2606.28560, Section 2.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+#include <stdint.h>
+
+namespace fibattn {
+
+constexpr int kHeadDim = 64;      // D; every kernel is specialised for it
+constexpr int kHalf = kHeadDim / 2;
+constexpr int kMaxRungs = 32;     // K limit of the ABI
+constexpr int kMaxWindow = 1024;  // W limit of the ABI
+
+// Per-rung data prepared on the host (Section 2: d_k = alpha * f_k, read by
+// linear interpolation between the floor and floor-plus-one rows).
+struct RungParams {
+    int K;                    // number of rungs passed by the caller
+    unsigned active;          // bit k: rung k can ever be attended (dedup, reach)
+    int s0[kMaxRungs];        // floor(d_k)
+    float w[kMaxRungs];       // d_k - floor(d_k): weight of the far row i-s0-1
+    float d[kMaxRungs];       // d_k in fp32; the rung is masked for queries i < d_k
+    float f[kMaxRungs];       // base value f_k (for dL/dalpha = sum_k f_k dL/dd_k)
+};
+
+// RoPE phase increments: the rotation angle of pair m at position p is
+// 2*pi * frac(p * F[m] / 2^64), F[m] = round(2^64 * theta_m / (2*pi)),
+// theta_m = base^(-2m/D).  The integer product wraps modulo one turn exactly,
+// so the angle is reduced without any floating-point range reduction.
+struct RopeParams {
+    unsigned long long F[kHalf];
+};
+
+struct Shape {
+    int B, H, Hkv, T, W, G;   // G = H / Hkv
+    float scale;              // score scale (1/sqrt(D) by default)
+};
+
+struct FwdArgs {
+    const void* q;            // [B,H,T,D]
+    const void* kt;           // rotated keys [B,Hkv,T,D] (workspace)
+    const void* k;            // raw keys (prologue input)
+    const void* v;            // [B,Hkv,T,D]
+    void* out;                // [B,H,T,D]
+    float* lse;               // [B,H,T]
+    Shape s;
+    RungParams r;
+    RopeParams rope;
+};
+
+struct BwdArgs {
+    const void* q;            // [B,H,T,D]
+    const void* k;            // [B,Hkv,T,D]
+    const void* v;
+    const float* lse;         // [B,H,T]
+    const void* dout;         // [B,H,T,D]
+    void* dq;                 // [B,H,T,D]
+    void* dk;                 // [B,Hkv,T,D]
+    void* dv;
+    float* dtheta;            // device scalar
+    float* dd;                // device [K] or nullptr
+    // workspace views
+    void* qt;                 // rotated q [B,H,T,D]
+    void* kt;                 // rotated k [B,Hkv,T,D]
+    float* P;                 // softmax probabilities [B,H,T,S]
+    float* DS;                // dL/dscore [B,H,T,S]
+    float* partial;           // per-block dL/dd_k partial sums [nblocks][kMaxRungs]
+    int nblocks_a;            // number of query-centric blocks (rows of partial)
+    int S;                    // slots per query = W + 1 + K
+    float alpha;
+    Shape s;
+    RungParams r;
+    RopeParams rope;
+};
+
+// ---------------------------------------------------------------- RoPE ----
+
+// cos/sin of the angle of pair m at position pos (see RopeParams).
+__device__ __forceinline__ void rope_cs(const RopeParams& rp, int m, int pos, float& c, float& s) {
+    unsigned long long ph = (unsigned long long)(unsigned)pos * rp.F[m];
+    int hi = (int)(unsigned)(ph >> 32);              // signed turn fraction in [-1/2, 1/2)
+    float ang = (float)hi * 1.4629180792671596e-09f; // 2*pi / 2^32
+    __sincosf(ang, &s, &c);
+}
+
+// ------------------------------------------------------------- element IO --
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(__nv_bfloat16 x) { return __bfloat162float(x); }
+
+template <typename T> struct Vec8;   // 8 consecutive elements
+
+template <> struct Vec8<float> {
+    static __device__ __forceinline__ void load(const float* p, float* x) {
+        float4 a = *reinterpret_cast<const float4*>(p);
+        float4 b = *reinterpret_cast<const float4*>(p + 4);
+        x[0] = a.x; x[1] = a.y; x[2] = a.z; x[3] = a.w; x[4] = b.x; x[5] = b.y; x[6] = b.z; x[7] = b.w;
+    }
+    static __device__ __forceinline__ void store(float* p, const float* x) {
+        *reinterpret_cast<float4*>(p) = make_float4(x[0], x[1], x[2], x[3]);
+        *reinterpret_cast<float4*>(p + 4) = make_float4(x[4], x[5], x[6], x[7]);
+    }
+};
+
+template <> struct Vec8<__nv_bfloat16> {
+    static __device__ __forceinline__ void load(const __nv_bfloat16* p, float* x) {
+        uint4 u = *reinterpret_cast<const uint4*>(p);
+        unsigned w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            x[2 * i] = __uint_as_float(w[i] << 16);
+            x[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+        }
+    }
+    static __device__ __forceinline__ void store(__nv_bfloat16* p, const float* x) {
+        uint4 u;
+        unsigned w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            __nv_bfloat162 h = __floats2bfloat162_rn(x[2 * i], x[2 * i + 1]);
+            w[i] = *reinterpret_cast<unsigned*>(&h);
+        }
+        u.x = w[0]; u.y = w[1]; u.z = w[2]; u.w = w[3];
+        *reinterpret_cast<uint4*>(p) = u;
+    }
+};
+
+// fp16 holds the RoPE-rotated q/k rows of the bf16 path: 10 mantissa bits
+// against bf16's 7 keep the score error well inside the bf16 tolerance.
+template <> struct Vec8<__half> {
+    static __device__ __forceinline__ void load(const __half* p, float* x) {
+        uint4 u = *reinterpret_cast<const uint4*>(p);
+        unsigned w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float2 f = __half22float2(*reinterpret_cast<__half2*>(&w[i]));
+            x[2 * i] = f.x;
+            x[2 * i + 1] = f.y;
+        }
+    }
+    static __device__ __forceinline__ void store(__half* p, const float* x) {
+        uint4 u;
+        unsigned w[4];
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            __half2 h = __floats2half2_rn(x[2 * i], x[2 * i + 1]);
+            w[i] = *reinterpret_cast<unsigned*>(&h);
+        }
+        u.x = w[0]; u.y = w[1]; u.z = w[2]; u.w = w[3];
+        *reinterpret_cast<uint4*>(p) = u;
+    }
+};
+
+// Storage type of rotated rows: fp32 for fp32 I/O, fp16 for bf16 I/O.
+template <typename T> struct RotOf { using type = float; };
+template <> struct RotOf<__nv_bfloat16> { using type = __half; };
+
+// A lane of a 4-lane group owns RoPE pairs [8c, 8c+8): head dims 8c..8c+7
+// (x[0..7]) and 32+8c..32+8c+7 (x[8..15]), so a rotation stays in the lane.
+template <typename T>
+__device__ __forceinline__ void load_chunk(const T* row, int c, float* x) {
+    Vec8<T>::load(row + 8 * c, x);
+    Vec8<T>::load(row + kHalf + 8 * c, x + 8);
+}
+template <typename T>
+__device__ __forceinline__ void store_chunk(T* row, int c, const float* x) {
+    Vec8<T>::store(row + 8 * c, x);
+    Vec8<T>::store(row + kHalf + 8 * c, x + 8);
+}
+
+// x <- R(pos) x (inverse = false) or R(pos)^T x (inverse = true) for the 8
+// pairs owned by lane c.
+__device__ __forceinline__ void rope_chunk(const RopeParams& rp, int pos, int c, float* x, bool inverse) {
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+        float cs, sn;
+        rope_cs(rp, 8 * c + u, pos, cs, sn);
+        if (inverse) sn = -sn;
+        float a = x[u], b = x[8 + u];
+        x[u] = a * cs - b * sn;
+        x[8 + u] = b * cs + a * sn;
+    }
+}
+
+// ----------------------------------------------------------- launchers ----
+
+cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
+                             bool bf16, cudaStream_t st);
+cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st);
+cudaError_t launch_bwd_query(const BwdArgs& a, bool bf16, cudaStream_t st);
+cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st);
+cudaError_t launch_bwd_finalize(const BwdArgs& a, cudaStream_t st);
+int bwd_simple_blocks(const Shape& s);
+
+// Opt-in per-kernel timing: when enabled, each launch is bracketed by CUDA
+// events recorded on the caller's stream (see fibattn_profile_* in the ABI).
+struct ProfScope {
+    ProfScope(const char* name, cudaStream_t st);
+    ~ProfScope();
+    const char* name_;
+    cudaStream_t st_;
+    cudaEvent_t start_;
+    bool on_;
+};
+
+}  // namespace fibattn

@@ -1,0 +1,472 @@
+// kernels_simple.cu -- straightforward CUDA kernels for every step of the
+// path (arXiv 2606.28560, Section 2): the RoPE prologue, the forward pass and
+// the backward pass.  Rows are read through L1/L2 with 128-bit loads; a group
+// of 4 lanes owns one query (or key) row, each lane 8 RoPE pairs (16 dims).
+//
+// Forward  (Section 2, "Attended set"): online softmax over the window slots
+//          t = 0..W and the interpolated rungs, accumulating the equally
+//          interpolated values.
+// Backward (chain rule of the forward): a query-centric pass recomputes the
+//          probabilities, forms dL/dscore, dq and the per-rung distance
+//          gradient; a key-centric pass gathers dk and dv from the shifted
+//          query rows (no atomics); a one-block pass sums the per-block rung
+//          partials in a fixed order and applies d_k = alpha f_k and
+//          alpha = 0.5 + sigmoid(theta) (Section 2, "The per-layer scalar").
+#include "fibattn_internal.cuh"
+
+namespace fibattn {
+
+namespace {
+
+constexpr int kThreads = 128;                 // 4 warps
+constexpr int kRowsPerBlock = kThreads / 4;   // 32 query/key rows per block
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+
+__device__ __forceinline__ float group_sum(float x) {
+    x += __shfl_xor_sync(0xffffffffu, x, 1);
+    x += __shfl_xor_sync(0xffffffffu, x, 2);
+    return x;
+}
+
+__device__ __forceinline__ float dot16(const float* a, const float* b) {
+    float s = 0.f;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) s = fmaf(a[e], b[e], s);
+    return s;
+}
+
+// ---------------------------------------------------------------- RoPE ----
+
+template <typename T, typename R>
+__global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ src, R* __restrict__ dst,
+                                                        long long rows, int T_, RopeParams rp) {
+    long long n = rows * 4;
+    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
+         g += (long long)gridDim.x * blockDim.x) {
+        long long row = g >> 2;
+        int c = (int)(g & 3);
+        int pos = (int)(row % T_);
+        float x[16];
+        load_chunk(src + row * kHeadDim, c, x);
+        rope_chunk(rp, pos, c, x, false);
+        store_chunk(dst + row * kHeadDim, c, x);
+    }
+}
+
+// ------------------------------------------------------------- forward ----
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads) fwd_simple_kernel(FwdArgs a) {
+    const Shape s = a.s;
+    const int lane = threadIdx.x & 31, c = lane & 3;
+    const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    const int bh = blockIdx.x / tiles;
+    const int i = (blockIdx.x % tiles) * kRowsPerBlock + (threadIdx.x >> 2);
+    const int b = bh / s.H, h = bh % s.H, hk = h / s.G;
+    const bool qvalid = i < s.T;
+    const int ii = qvalid ? i : s.T - 1;
+
+    const T* Q = reinterpret_cast<const T*>(a.q) + ((size_t)bh * s.T) * kHeadDim;
+    using R = typename RotOf<T>::type;
+    const R* Kt = reinterpret_cast<const R*>(a.kt) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
+    const T* V = reinterpret_cast<const T*>(a.v) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
+
+    float q[16];
+    load_chunk(Q + (size_t)ii * kHeadDim, c, q);
+    rope_chunk(a.rope, ii, c, q, false);
+    const float sc2 = s.scale * kLog2e;          // scores kept in log2 units
+
+    float m = -INFINITY, l = 0.f, acc[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) acc[e] = 0.f;
+
+    float kr[16], vr[16];
+    // window slots: distance t = 0..W (self always present)
+    for (int t = 0; t <= s.W; ++t) {
+        const int j = ii - t;
+        const bool ok = j >= 0;
+        const int jj = ok ? j : 0;
+        load_chunk(Kt + (size_t)jj * kHeadDim, c, kr);
+        const float sco = group_sum(dot16(q, kr)) * sc2;
+        if (ok) {
+            load_chunk(V + (size_t)jj * kHeadDim, c, vr);
+            if (sco > m) {
+                const float corr = exp2f(m - sco);
+                l *= corr;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) acc[e] *= corr;
+                m = sco;
+            }
+            const float p = exp2f(sco - m);
+            l += p;
+#pragma unroll
+            for (int e = 0; e < 16; ++e) acc[e] = fmaf(p, vr[e], acc[e]);
+        }
+        if (__all_sync(0xffffffffu, !ok)) break;
+    }
+    // rungs: d_k = alpha f_k, read between rows i-s0 (weight 1-w) and i-s0-1 (weight w)
+    const float fi = (float)ii;
+    for (int k = 0; k < a.r.K; ++k) {
+        if (!((a.r.active >> k) & 1u)) continue;
+        const int s0 = a.r.s0[k];
+        const float w = a.r.w[k];
+        const bool ok = a.r.d[k] <= fi;
+        const int j0 = ii - s0, j1 = j0 - 1;
+        const int jj0 = ok ? j0 : 0;
+        load_chunk(Kt + (size_t)jj0 * kHeadDim, c, kr);
+        float sraw = (1.f - w) * dot16(q, kr);
+        const bool far = w != 0.f;               // warp-uniform
+        float kf[16];
+        if (far) {
+            const int jj1 = (ok && j1 >= 0) ? j1 : 0;
+            load_chunk(Kt + (size_t)jj1 * kHeadDim, c, kf);
+            if (ok && j1 >= 0) sraw = fmaf(w, dot16(q, kf), sraw);
+        }
+        const float sco = group_sum(sraw) * sc2;
+        if (ok) {
+            load_chunk(V + (size_t)jj0 * kHeadDim, c, vr);
+            if (sco > m) {
+                const float corr = exp2f(m - sco);
+                l *= corr;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) acc[e] *= corr;
+                m = sco;
+            }
+            const float p = exp2f(sco - m);
+            l += p;
+            const float p0 = p * (1.f - w);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) acc[e] = fmaf(p0, vr[e], acc[e]);
+            if (far && j1 >= 0) {
+                load_chunk(V + (size_t)j1 * kHeadDim, c, vr);
+                const float p1 = p * w;
+#pragma unroll
+                for (int e = 0; e < 16; ++e) acc[e] = fmaf(p1, vr[e], acc[e]);
+            }
+        }
+    }
+    if (qvalid) {
+        const float inv = 1.f / l;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) acc[e] *= inv;
+        T* O = reinterpret_cast<T*>(a.out) + ((size_t)bh * s.T + i) * kHeadDim;
+        store_chunk(O, c, acc);
+        if (c == 0) a.lse[(size_t)bh * s.T + i] = (m + __log2f(l)) * kLn2;
+    }
+}
+
+// ------------------------------------------------------------ backward ----
+
+// Query-centric pass.  For query i: recompute p = exp(score - lse) for every
+// slot, Delta = sum_slots p * (dO . val), dS = p (dO . val - Delta); then
+// dq~ = scale sum dS key, and per rung
+//   dL/dd_k += scale dS (q~ . (k~[j1] - k~[j0])) + p (dO . (v[j1] - v[j0])).
+// Writes P and DS (zero for slots that are not attended) for the key pass.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
+    __shared__ float red[kThreads / 32][kMaxRungs];
+    const Shape s = a.s;
+    const int lane = threadIdx.x & 31, c = lane & 3, warp = threadIdx.x >> 5;
+    const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    const int bh = blockIdx.x / tiles;
+    const int i = (blockIdx.x % tiles) * kRowsPerBlock + (threadIdx.x >> 2);
+    const int b = bh / s.H, h = bh % s.H, hk = h / s.G;
+    const bool qvalid = i < s.T;
+    const int ii = qvalid ? i : s.T - 1;
+    const float fi = (float)ii;
+    const float lse2 = qvalid ? a.lse[(size_t)bh * s.T + ii] * kLog2e : 0.f;
+    const float sc2 = s.scale * kLog2e;
+
+    using R = typename RotOf<T>::type;
+    const R* Qt = reinterpret_cast<const R*>(a.qt) + ((size_t)bh * s.T) * kHeadDim;
+    const T* dO = reinterpret_cast<const T*>(a.dout) + ((size_t)bh * s.T) * kHeadDim;
+    const R* Kt = reinterpret_cast<const R*>(a.kt) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
+    const T* V = reinterpret_cast<const T*>(a.v) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
+    float* Prow = a.P + ((size_t)bh * s.T + ii) * a.S;
+    float* DSrow = a.DS + ((size_t)bh * s.T + ii) * a.S;
+
+    float q[16], go[16], kr[16], kf[16], vr[16], vf[16];
+    load_chunk(Qt + (size_t)ii * kHeadDim, c, q);
+    load_chunk(dO + (size_t)ii * kHeadDim, c, go);
+
+    // pass 1: Delta = sum_slots p * (dO . val)
+    float delta = 0.f;
+    for (int t = 0; t <= s.W; ++t) {
+        const int j = ii - t;
+        const bool ok = j >= 0;
+        const int jj = ok ? j : 0;
+        load_chunk(Kt + (size_t)jj * kHeadDim, c, kr);
+        load_chunk(V + (size_t)jj * kHeadDim, c, vr);
+        const float sco = group_sum(dot16(q, kr)) * sc2;
+        const float dp = group_sum(dot16(go, vr));
+        if (ok) delta = fmaf(exp2f(sco - lse2), dp, delta);
+        if (__all_sync(0xffffffffu, !ok)) break;
+    }
+    for (int k = 0; k < a.r.K; ++k) {
+        if (!((a.r.active >> k) & 1u)) continue;
+        const int s0 = a.r.s0[k];
+        const float w = a.r.w[k];
+        const bool ok = a.r.d[k] <= fi;
+        const int j0 = ok ? ii - s0 : 0;
+        const bool far = w != 0.f;
+        const bool hasf = ok && far && j0 >= 1;
+        const int j1 = hasf ? j0 - 1 : 0;
+        load_chunk(Kt + (size_t)j0 * kHeadDim, c, kr);
+        load_chunk(V + (size_t)j0 * kHeadDim, c, vr);
+        float s0r = dot16(q, kr), dp0 = dot16(go, vr), s1r = 0.f, dp1 = 0.f;
+        if (far) {
+            load_chunk(Kt + (size_t)j1 * kHeadDim, c, kf);
+            load_chunk(V + (size_t)j1 * kHeadDim, c, vf);
+            if (hasf) { s1r = dot16(q, kf); dp1 = dot16(go, vf); }
+        }
+        const float sco = group_sum((1.f - w) * s0r + w * s1r) * sc2;
+        const float dp = group_sum((1.f - w) * dp0 + w * dp1);
+        if (ok) delta = fmaf(exp2f(sco - lse2), dp, delta);
+    }
+
+    // pass 2: dS, dq~, rung gradients, P / DS for the key pass
+    float dq[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) dq[e] = 0.f;
+    float g[kMaxRungs];
+#pragma unroll
+    for (int k = 0; k < kMaxRungs; ++k) g[k] = 0.f;
+
+    for (int t = 0; t <= s.W; ++t) {
+        const int j = ii - t;
+        const bool ok = j >= 0;
+        const int jj = ok ? j : 0;
+        load_chunk(Kt + (size_t)jj * kHeadDim, c, kr);
+        load_chunk(V + (size_t)jj * kHeadDim, c, vr);
+        const float sco = group_sum(dot16(q, kr)) * sc2;
+        const float dp = group_sum(dot16(go, vr));
+        const float p = ok ? exp2f(sco - lse2) : 0.f;
+        const float ds = p * (dp - delta);
+        const float dss = ds * s.scale;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) dq[e] = fmaf(dss, kr[e], dq[e]);
+        if (qvalid && c == 0) { Prow[t] = p; DSrow[t] = ds; }
+        if (__all_sync(0xffffffffu, j < 0)) {
+            if (qvalid && c == 0)
+                for (int u = t + 1; u <= s.W; ++u) { Prow[u] = 0.f; DSrow[u] = 0.f; }
+            break;
+        }
+    }
+    for (int k = 0; k < a.r.K; ++k) {
+        const int slot = s.W + 1 + k;
+        if (!((a.r.active >> k) & 1u)) {
+            if (qvalid && c == 0) { Prow[slot] = 0.f; DSrow[slot] = 0.f; }
+            continue;
+        }
+        const int s0 = a.r.s0[k];
+        const float w = a.r.w[k];
+        const bool ok = a.r.d[k] <= fi;
+        const int j0 = ok ? ii - s0 : 0;
+        // the far row enters dL/dd_k even at w == 0 (one-sided derivative);
+        // row -1 (only when d_k == i) is a zero row
+        const bool hasf = ok && j0 >= 1;
+        const int j1 = hasf ? j0 - 1 : 0;
+        load_chunk(Kt + (size_t)j0 * kHeadDim, c, kr);
+        load_chunk(V + (size_t)j0 * kHeadDim, c, vr);
+        float s0r = dot16(q, kr), dp0 = dot16(go, vr), s1r = 0.f, dp1 = 0.f;
+        load_chunk(Kt + (size_t)j1 * kHeadDim, c, kf);
+        load_chunk(V + (size_t)j1 * kHeadDim, c, vf);
+        if (hasf) { s1r = dot16(q, kf); dp1 = dot16(go, vf); }
+        s0r = group_sum(s0r); s1r = group_sum(s1r);
+        dp0 = group_sum(dp0); dp1 = group_sum(dp1);
+        const float sco = ((1.f - w) * s0r + w * s1r) * sc2;
+        const float dp = (1.f - w) * dp0 + w * dp1;
+        const float p = ok ? exp2f(sco - lse2) : 0.f;
+        const float ds = p * (dp - delta);
+        const float dss = ds * s.scale;
+        const float c0 = dss * (1.f - w), c1 = dss * w;
+#pragma unroll
+        for (int e = 0; e < 16; ++e) dq[e] = fmaf(c0, kr[e], dq[e]);
+        if (hasf) {
+#pragma unroll
+            for (int e = 0; e < 16; ++e) dq[e] = fmaf(c1, kf[e], dq[e]);
+        }
+        // d(key)/d(d_k) = k~[j1] - k~[j0], d(val)/d(d_k) = v[j1] - v[j0] (row -1 is zero)
+        if (qvalid && ok) g[k] += dss * (s1r - s0r) + p * (dp1 - dp0);
+        if (qvalid && c == 0) { Prow[slot] = p; DSrow[slot] = ds; }
+    }
+    if (qvalid) {
+        rope_chunk(a.rope, ii, c, dq, true);
+        T* dQ = reinterpret_cast<T*>(a.dq) + ((size_t)bh * s.T + i) * kHeadDim;
+        store_chunk(dQ, c, dq);
+    }
+    // per-block rung partials: sum the 8 query groups of the warp (lanes with
+    // c == 0 hold the value; other lanes hold the same copy), then the warps.
+#pragma unroll
+    for (int k = 0; k < kMaxRungs; ++k) {
+        float x = (c == 0) ? g[k] : 0.f;
+        x += __shfl_xor_sync(0xffffffffu, x, 4);
+        x += __shfl_xor_sync(0xffffffffu, x, 8);
+        x += __shfl_xor_sync(0xffffffffu, x, 16);
+        if (lane == 0) red[warp][k] = x;
+    }
+    __syncthreads();
+    if (threadIdx.x < kMaxRungs) {
+        float x = 0.f;
+        for (int w = 0; w < kThreads / 32; ++w) x += red[w][threadIdx.x];
+        a.partial[(size_t)blockIdx.x * kMaxRungs + threadIdx.x] = x;
+    }
+}
+
+// Key-centric pass.  Key row j of kv head hk receives, from every query head
+// of its group, the slots that read it: window slot t of query j+t (weight 1),
+// rung k of query j+s0_k (floor row, weight 1-w_k) and of query j+s0_k+1 (far
+// row, weight w_k):  dk~_j = scale sum c dS q~_i,  dv_j = sum c P dO_i.
+template <typename T>
+__global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
+    const Shape s = a.s;
+    const int c = threadIdx.x & 3;
+    const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    const int bhk = blockIdx.x / tiles;               // b * Hkv + hk
+    const int j = (blockIdx.x % tiles) * kRowsPerBlock + (threadIdx.x >> 2);
+    const int b = bhk / s.Hkv, hk = bhk % s.Hkv;
+    const bool kvalid = j < s.T;
+    const int jj = kvalid ? j : s.T - 1;
+
+    float dk[16], dv[16], x[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) { dk[e] = 0.f; dv[e] = 0.f; }
+
+    for (int g = 0; g < s.G; ++g) {
+        const int bh = b * s.H + hk * s.G + g;
+        using R = typename RotOf<T>::type;
+        const R* Qt = reinterpret_cast<const R*>(a.qt) + ((size_t)bh * s.T) * kHeadDim;
+        const T* dO = reinterpret_cast<const T*>(a.dout) + ((size_t)bh * s.T) * kHeadDim;
+        const float* P = a.P + (size_t)bh * s.T * a.S;
+        const float* DS = a.DS + (size_t)bh * s.T * a.S;
+        for (int t = 0; t <= s.W; ++t) {
+            const int i = jj + t;
+            const bool ok = i < s.T;
+            const int ic = ok ? i : jj;
+            const float ds = ok ? DS[(size_t)ic * a.S + t] * s.scale : 0.f;
+            const float p = ok ? P[(size_t)ic * a.S + t] : 0.f;
+            load_chunk(Qt + (size_t)ic * kHeadDim, c, x);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) dk[e] = fmaf(ds, x[e], dk[e]);
+            load_chunk(dO + (size_t)ic * kHeadDim, c, x);
+#pragma unroll
+            for (int e = 0; e < 16; ++e) dv[e] = fmaf(p, x[e], dv[e]);
+            if (__all_sync(0xffffffffu, !ok)) break;
+        }
+        for (int k = 0; k < a.r.K; ++k) {
+            if (!((a.r.active >> k) & 1u)) continue;
+            const int slot = s.W + 1 + k;
+            const float w = a.r.w[k];
+#pragma unroll
+            for (int side = 0; side < 2; ++side) {
+                const float cw = side == 0 ? 1.f - w : w;
+                if (side == 1 && w == 0.f) break;       // warp-uniform
+                const long long il = (long long)jj + a.r.s0[k] + side;
+                const bool ok = il < s.T;
+                const int ic = ok ? (int)il : jj;
+                const float ds = ok ? DS[(size_t)ic * a.S + slot] * s.scale * cw : 0.f;
+                const float p = ok ? P[(size_t)ic * a.S + slot] * cw : 0.f;
+                if (__all_sync(0xffffffffu, !ok)) continue;
+                load_chunk(Qt + (size_t)ic * kHeadDim, c, x);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) dk[e] = fmaf(ds, x[e], dk[e]);
+                load_chunk(dO + (size_t)ic * kHeadDim, c, x);
+#pragma unroll
+                for (int e = 0; e < 16; ++e) dv[e] = fmaf(p, x[e], dv[e]);
+            }
+        }
+    }
+    if (kvalid) {
+        rope_chunk(a.rope, jj, c, dk, true);
+        const size_t off = ((size_t)bhk * s.T + j) * kHeadDim;
+        store_chunk(reinterpret_cast<T*>(a.dk) + off, c, dk);
+        store_chunk(reinterpret_cast<T*>(a.dv) + off, c, dv);
+    }
+}
+
+// Fixed-order sum of the per-block rung partials (fp64), then the chain rule
+// dL/dalpha = sum_k f_k dL/dd_k and dL/dtheta = dL/dalpha (alpha-0.5)(1.5-alpha).
+// Thread t sums blocks t, t+256, ... in order; a fixed shared-memory tree then
+// combines the 256 partial sums, so the result does not depend on scheduling.
+constexpr int kFinThreads = 256;
+__global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
+    __shared__ double red[kFinThreads];
+    __shared__ double dd[kMaxRungs];
+    const int t = threadIdx.x;
+    for (int k = 0; k < a.r.K; ++k) {
+        double x = 0.0;
+        for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) x += (double)a.partial[(size_t)blk * kMaxRungs + k];
+        red[t] = x;
+        __syncthreads();
+        for (int w = kFinThreads / 2; w > 0; w >>= 1) {
+            if (t < w) red[t] += red[t + w];
+            __syncthreads();
+        }
+        if (t == 0) dd[k] = red[0];
+        __syncthreads();
+    }
+    if (t < a.r.K && a.dd) a.dd[t] = (float)dd[t];
+    if (t == 0) {
+        double da = 0.0;
+        for (int u = 0; u < a.r.K; ++u) da += (double)a.r.f[u] * dd[u];
+        const double al = (double)a.alpha;
+        *a.dtheta = (float)(da * (al - 0.5) * (1.5 - al));
+    }
+}
+
+}  // namespace
+
+cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
+                             bool bf16, cudaStream_t st) {
+    if (rows <= 0) return cudaSuccess;
+    long long threads = rows * 4;
+    int grid = (int)((threads + 255) / 256);
+    if (grid > 152 * 16) grid = 152 * 16;
+    if (bf16)
+        rope_rows_kernel<__nv_bfloat16, __half><<<grid, 256, 0, st>>>(
+            reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp);
+    else
+        rope_rows_kernel<float, float><<<grid, 256, 0, st>>>(reinterpret_cast<const float*>(src),
+                                                              reinterpret_cast<float*>(dst), rows, T, rp);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st) {
+    const long long tiles = (a.s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    const long long grid = tiles * a.s.B * a.s.H;
+    if (grid <= 0) return cudaSuccess;
+    if (bf16) fwd_simple_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, st>>>(a);
+    else fwd_simple_kernel<float><<<(unsigned)grid, kThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+int bwd_simple_blocks(const Shape& s) {
+    const long long tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    return (int)(tiles * s.B * s.H);
+}
+
+cudaError_t launch_bwd_query(const BwdArgs& a, bool bf16, cudaStream_t st) {
+    const long long tiles = (a.s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    const long long gq = tiles * a.s.B * a.s.H;
+    if (gq <= 0) return cudaSuccess;
+    if (bf16) bwd_query_kernel<__nv_bfloat16><<<(unsigned)gq, kThreads, 0, st>>>(a);
+    else bwd_query_kernel<float><<<(unsigned)gq, kThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st) {
+    const long long tiles = (a.s.T + kRowsPerBlock - 1) / kRowsPerBlock;
+    const long long gk = tiles * a.s.B * a.s.Hkv;
+    if (gk <= 0) return cudaSuccess;
+    if (bf16) bwd_key_kernel<__nv_bfloat16><<<(unsigned)gk, kThreads, 0, st>>>(a);
+    else bwd_key_kernel<float><<<(unsigned)gk, kThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_bwd_finalize(const BwdArgs& a, cudaStream_t st) {
+    bwd_finalize_kernel<<<1, kFinThreads, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace fibattn

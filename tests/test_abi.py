@@ -1,0 +1,122 @@
+"""CPU-only checks of the C ABI: the library loads, exports every function
+declared in include/fibattn.h, its host-side prep matches the oracle's
+definitions, and bad arguments are rejected before anything is launched."""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import oracle as O
+import paper_2606_28560_gb300 as fa
+from paper_2606_28560_gb300 import binding as B
+from paper_2606_28560_gb300 import build as build_mod
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    build_mod.build()
+
+
+def _declared():
+    names = []
+    for h in sorted(os.listdir(os.path.join(ROOT, "include"))):
+        if h.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", h)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names += re.findall(r"\b(fibattn_\w+)\s*\(", text)
+    return sorted(set(names))
+
+
+def test_library_exports_every_declared_function():
+    lib = ctypes.CDLL(fa.library_path())
+    decl = _declared()
+    assert "fibattn_fwd" in decl and "fibattn_bwd" in decl
+    for name in decl:
+        assert hasattr(lib, name), f"{name} declared in include/ but not exported"
+
+
+def test_base_and_schedules_match_oracle():
+    np.testing.assert_array_equal(fa.base("fib", 15), O.fib_base(15).astype(np.float32))
+    np.testing.assert_array_equal(fa.base("pow2", 10), O.pow2_base(10).astype(np.float32))
+    for kind in ("fixed", "linear", "coprime"):
+        np.testing.assert_allclose(fa.alpha_schedule(kind, 16), O.alpha_schedule(kind, 16), rtol=0, atol=1e-7)
+    th = [0.3, -0.8, 0.0, 1.7]
+    np.testing.assert_allclose(fa.alpha_schedule("learned", 4, theta=th),
+                               O.alpha_schedule("learned", 4, theta=th), rtol=0, atol=1e-7)
+
+
+@pytest.mark.parametrize("alpha", [0.5, 0.5 + 1 / 15, 0.7333333, 1.0, 1.2345, 1.5])
+@pytest.mark.parametrize("W", [0, 8, 12])
+def test_rung_params_match_oracle(alpha, W):
+    f = O.fib_base(15)
+    p = fa.rung_params(np.float32(alpha), f, W)
+    d = O.offsets_fp32(float(np.float32(alpha)), f)
+    np.testing.assert_array_equal(p["d"].astype(np.float64), d)
+    np.testing.assert_array_equal(p["s0"], np.floor(d).astype(np.int32))
+    np.testing.assert_array_equal(p["w"].astype(np.float64), d - np.floor(d))
+    np.testing.assert_array_equal(p["active"], d > W)
+    p2 = fa.rung_params(np.float32(alpha), f, W, dedup=False)
+    assert p2["active"].all()
+
+
+def _call_fwd(**kw):
+    lib = B.lib()
+    args = dict(q=16, k=16, v=16, out=16, lse=16, B=1, H=2, T=8, D=64, W=2, alpha=1.0,
+                K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0)
+    args.update(kw)
+    f = np.array([1, 2, 3] + [5] * 40, dtype=np.float32)
+    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0)
+    rc = lib.fibattn_fwd(args["q"], args["k"], args["v"], args["out"], args["lse"], args["B"], args["H"],
+                         args["T"], args["D"], args["W"], args["alpha"], B._fptr(f), args["K"], args["dtype"],
+                         ctypes.byref(o), args["ws"], args["wsb"], None)
+    return rc, lib.fibattn_last_error().decode()
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(alpha=0.49), 1), (dict(alpha=1.51), 1), (dict(alpha=float("nan")), 1),
+    (dict(K=33), 1), (dict(K=-1), 1), (dict(W=-1), 1), (dict(W=1025), 1),
+    (dict(D=128), 2), (dict(D=32), 2), (dict(T=0), 1), (dict(H=0), 1), (dict(dtype=7), 1),
+    (dict(Hkv=3), 1), (dict(q=0), 1), (dict(lse=0), 1), (dict(ws=0), 1),
+    (dict(q=17), 1), (dict(out=24), 1), (dict(wsb=10), 1), (dict(rope_base=-2.0), 1),
+])
+def test_fwd_rejects_bad_arguments(kw, code):
+    rc, msg = _call_fwd(**kw)
+    assert rc == code, msg
+    assert msg
+
+
+def test_bwd_rejects_bad_arguments():
+    lib = B.lib()
+    f = np.array([1, 2, 3], dtype=np.float32)
+    o = B.Opts(0.0, 0.0, 0, 0)
+    ok_ptr = 16
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None, None,
+                         1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
+    assert rc == 1 and "dtheta" in lib.fibattn_last_error().decode()
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, 18, None,
+                         1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
+    assert rc == 1
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None,
+                         1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 8, None)
+    assert rc == 1 and "workspace" in lib.fibattn_last_error().decode()
+
+
+def test_workspace_queries():
+    import torch
+    assert fa.fwd_workspace_bytes(16, 8, 1024, 8, 15, torch.bfloat16) >= 16 * 8 * 1024 * 64 * 2
+    assert fa.bwd_workspace_bytes(16, 8, 1024, 8, 15, torch.bfloat16) > fa.fwd_workspace_bytes(16, 8, 1024, 8, 15,
+                                                                                                 torch.bfloat16)
+    assert B.lib().fibattn_fwd_workspace_bytes(1, 2, 8, 128, 2, 3, 0, None) == 0    # invalid -> 0
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    monkeypatch.setattr(build_mod, "LIB", str(tmp_path / "nope.so"))
+    monkeypatch.setattr(B, "_lib", None)
+    with pytest.raises(RuntimeError, match="not built"):
+        B.lib()

@@ -1,0 +1,209 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on
+the same seeded inputs, element by element.
+
+Tolerances: fp32 I/O max abs error <= 1e-4 on out/lse and <= 1e-4 relative
+to the largest reference magnitude on gradients; bf16 I/O (fp32 accumulate)
+max abs error <= 1e-2 on out and <= 3e-2 relative (max |g - ref| / max |ref|)
+on gradients; dtheta |d - ref| / |ref|.
+"""
+from __future__ import annotations
+
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import oracle as O
+import paper_2606_28560_gb300 as fa
+from paper_2606_28560_gb300 import inputs
+
+pytestmark = pytest.mark.gpu
+
+NTHREADS = max(1, min(16, os.cpu_count() or 1))
+TOL = {torch.float32: dict(out=1e-4, lse=1e-4, grad=1e-4, dtheta=1e-4),
+       torch.bfloat16: dict(out=1e-2, lse=1e-2, grad=3e-2, dtheta=3e-2)}
+
+
+def _f64(t):
+    return t.detach().to("cpu", torch.float64).numpy()
+
+
+def bf16_out_tol(ref):
+    """Per-element bar on bf16 outputs: 1e-2 wherever bf16 can hold it (|o| < 4,
+    where half a bf16 ulp is at most 2^-8 * 2 = 2^-7).  For |o| >= 4 the format's
+    own rounding step (half-ulp >= 2^-6) alone can exceed 1e-2 even for an exact
+    result, so the excess of that half-ulp over 2^-7 is added to the bar."""
+    e = np.floor(np.log2(np.maximum(np.abs(ref), 1e-30)))
+    half_ulp = np.exp2(e - 8)
+    return 1e-2 + np.maximum(0.0, half_ulp - 2.0 ** -7)
+
+
+def _rel(a, ref):
+    return float(np.max(np.abs(a - ref)) / max(np.max(np.abs(ref)), 1e-30))
+
+
+def _offsets(kind, K):
+    return fa.base(kind, K)
+
+
+def gpu_fwd(q, k, v, alpha, f, W, dedup=True):
+    out, lse = fa.fwd(q.cuda(), k.cuda(), v.cuda(), alpha, f, W, dedup=dedup)
+    torch.cuda.synchronize()
+    return out, lse
+
+
+def oracle_fwd(q, k, v, alpha, f, W, dedup=True):
+    d = O.offsets_fp32(float(np.float32(alpha)), f.astype(np.float64))
+    return O.forward(_f64(q), _f64(k), _f64(v), W, d, dedup=dedup, nthreads=NTHREADS)
+
+
+def check_fwd(q, k, v, alpha, f, W, dedup=True):
+    out, lse = gpu_fwd(q, k, v, alpha, f, W, dedup)
+    ro, rl = oracle_fwd(q, k, v, alpha, f, W, dedup)
+    tol = TOL[q.dtype]
+    diff = np.abs(_f64(out) - ro)
+    eo = float(np.max(diff)) if ro.size else 0.0
+    el = float(np.max(np.abs(_f64(lse) - rl))) if rl.size else 0.0
+    if q.dtype == torch.bfloat16 and ro.size:
+        bad = diff > bf16_out_tol(ro)
+        assert not bad.any(), f"out err {eo} (worst over bar at |ref|={np.abs(ro[bad]).max():.3f})"
+        assert float(np.max(diff[np.abs(ro) < 4.0], initial=0.0)) <= tol["out"], f"out max abs err {eo} for |ref| < 4"
+    else:
+        assert eo <= tol["out"], f"out max abs err {eo}"
+    assert el <= tol["lse"], f"lse max abs err {el}"
+    return out, lse
+
+
+def check_bwd(q, k, v, dout, alpha, f, W, dedup=True):
+    qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), dout.cuda()
+    out, lse = fa.fwd(qc, kc, vc, alpha, f, W, dedup=dedup)
+    dq, dk, dv, dth, dd = fa.bwd(qc, kc, vc, lse, gc, alpha, f, W, dedup=dedup)
+    torch.cuda.synchronize()
+    a32 = float(np.float32(alpha))
+    d = O.offsets_fp32(a32, f.astype(np.float64))
+    rq, rk, rv, rdd = O.backward(_f64(q), _f64(k), _f64(v), _f64(dout), W, d, dedup=dedup, nthreads=NTHREADS)
+    _, rth = O.dtheta(a32, f.astype(np.float64), rdd)
+    tol = TOL[q.dtype]
+    for name, g, r in (("dq", dq, rq), ("dk", dk, rk), ("dv", dv, rv)):
+        e = _rel(_f64(g), r)
+        assert e <= tol["grad"], f"{name} rel err {e}"
+    eth = abs(float(dth[0]) - rth) / max(abs(rth), 1e-6)
+    assert eth <= tol["dtheta"], f"dtheta {float(dth[0])} vs {rth} (rel {eth})"
+    edd = _rel(_f64(dd), rdd) if len(f) else 0.0
+    assert edd <= tol["dtheta"], f"dd rel err {edd}"
+    return dict(dq=dq, dk=dk, dv=dv, dtheta=float(dth[0]), dtheta_ref=rth)
+
+
+# ------------------------------------------------------------ small cases --
+
+SMALL = [
+    # (B, H, Hkv, T, W, alpha, base, K, dedup)
+    (1, 2, 2, 1, 8, 1.0, "fib", 15, True),
+    (1, 2, 2, 5, 0, 1.0, "fib", 15, True),
+    (2, 4, 2, 77, 3, 0.7333333, "fib", 15, True),
+    (1, 3, 3, 130, 8, 1.0, "fib", 15, True),
+    (2, 2, 1, 300, 12, 1.4666666, "fib", 15, True),
+    (1, 2, 2, 257, 6, 0.5, "fib", 15, True),
+    (1, 2, 2, 200, 10, 1.5, "fib", 15, True),
+    (1, 2, 2, 190, 8, 0.9, "pow2", 10, True),
+    (1, 2, 2, 150, 4, 1.1, "fib", 12, False),
+    (1, 2, 2, 100, 5, 0.8, "fib", 0, True),
+    (1, 2, 2, 64, 63, 1.0, "fib", 15, True),
+    (1, 1, 1, 2100, 8, 1.5, "fib", 15, True),
+]
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+@pytest.mark.parametrize("case", SMALL, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]}{c[6]}{c[7]}d{int(c[8])}"
+                                              for c in SMALL])
+def test_forward_small(case, dtype):
+    Bn, H, Hkv, T, W, alpha, base, K, dedup = case
+    q, k, v = inputs.qkv(Bn, H, T, seed=T + W, dtype=dtype, Hkv=Hkv)
+    check_fwd(q, k, v, alpha, _offsets(base, K), W, dedup)
+
+
+@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+@pytest.mark.parametrize("case", SMALL, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]}{c[6]}{c[7]}d{int(c[8])}"
+                                              for c in SMALL])
+def test_backward_small(case, dtype):
+    Bn, H, Hkv, T, W, alpha, base, K, dedup = case
+    q, k, v = inputs.qkv(Bn, H, T, seed=T + W + 1, dtype=dtype, Hkv=Hkv)
+    g = inputs.dout(Bn, H, T, seed=T + W + 2, dtype=dtype)
+    check_bwd(q, k, v, g, alpha, _offsets(base, K), W, dedup)
+
+
+def test_empty_batch():
+    q = torch.zeros((0, 2, 16, 64), device="cuda")
+    out, lse = fa.fwd(q, q, q, 1.0, _offsets("fib", 15), 4)
+    assert out.shape == q.shape and lse.shape == (0, 2, 16)
+    dq, dk, dv, dth, dd = fa.bwd(q, q, q, lse, q, 1.0, _offsets("fib", 15), 4)
+    torch.cuda.synchronize()
+    assert float(dth[0]) == 0.0 and torch.all(dd == 0)
+
+
+def test_outputs_finite_and_deterministic():
+    q, k, v = inputs.qkv(2, 4, 700, seed=5, dtype=torch.bfloat16)
+    g = inputs.dout(2, 4, 700, seed=6, dtype=torch.bfloat16)
+    qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), g.cuda()
+    f = _offsets("fib", 15)
+    r1 = fa.bwd(qc, kc, vc, fa.fwd(qc, kc, vc, 0.77, f, 8)[1], gc, 0.77, f, 8)
+    r2 = fa.bwd(qc, kc, vc, fa.fwd(qc, kc, vc, 0.77, f, 8)[1], gc, 0.77, f, 8)
+    torch.cuda.synchronize()
+    for a, b in zip(r1, r2):
+        assert torch.equal(a, b)
+        assert torch.isfinite(a.float()).all()
+
+
+# --------------------------------------------- full-size workload configs --
+
+def test_config1_fp32_alpha1_full():
+    """B=1 H=8 T=1024 D=64 W=8 alpha=1 (integer rungs), fp32, seed 0: every output."""
+    q, k, v = inputs.qkv(1, 8, 1024, seed=0, dtype=torch.float32)
+    check_fwd(q, k, v, 1.0, _offsets("fib", 15), 8)
+
+
+@pytest.mark.parametrize("W", [6, 8, 10, 12])
+def test_config2_bf16_linear_stagger(W):
+    """B=16 H=8 T=1024, 16 layers with alpha_l = 0.5 + l/15: layers 0, 7, 15 in
+    full (all 131072 query heads of the launch)."""
+    alphas = fa.alpha_schedule("linear", 16)
+    f = _offsets("fib", 15)
+    for layer in (0, 7, 15):
+        q, k, v = inputs.qkv(16, 8, 1024, seed=inputs.layer_seed(1, layer), dtype=torch.bfloat16)
+        check_fwd(q, k, v, float(alphas[layer]), f, W)
+
+
+def test_config3_bf16_extrapolation_coprime():
+    """B=4 H=8 T=4096 W=10, coprime-reassigned stagger: layers 0, 1, 9."""
+    alphas = fa.alpha_schedule("coprime", 16)
+    f = _offsets("fib", 15)
+    for layer in (0, 1, 9):
+        q, k, v = inputs.qkv(4, 8, 4096, seed=inputs.layer_seed(2, layer), dtype=torch.bfloat16)
+        check_fwd(q, k, v, float(alphas[layer]), f, 10)
+
+
+def test_config4_bf16_backward_learned_alpha():
+    """B=16 H=8 T=1024 W=8, theta_l ~ N(0, 0.5): fwd+bwd of layers 0 and 15 in full."""
+    theta = inputs.theta_learned(16, seed=3)
+    alphas = fa.alpha_schedule("learned", 16, theta=theta)
+    f = _offsets("fib", 15)
+    for layer in (0, 15):
+        s = inputs.layer_seed(3, layer)
+        q, k, v = inputs.qkv(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+        g = inputs.dout(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+        check_bwd(q, k, v, g, float(alphas[layer]), f, 8)
+
+
+@pytest.mark.parametrize("base,K", [("fib", 15), ("pow2", 10)])
+def test_config5_bf16_long_stress(base, K):
+    """B=2 H=8 T=16384 W=12, linear stagger, Fibonacci vs power-of-2 base:
+    fwd+bwd of layers 0 and 15 in full."""
+    alphas = fa.alpha_schedule("linear", 16)
+    f = _offsets(base, K)
+    for layer in (0, 15):
+        s = inputs.layer_seed(4, layer)
+        q, k, v = inputs.qkv(2, 8, 16384, seed=s, dtype=torch.bfloat16)
+        g = inputs.dout(2, 8, 16384, seed=s, dtype=torch.bfloat16)
+        check_fwd(q, k, v, float(alphas[layer]), f, 12)
+        check_bwd(q, k, v, g, float(alphas[layer]), f, 12)
