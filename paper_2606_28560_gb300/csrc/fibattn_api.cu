@@ -109,7 +109,7 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
 }
 
 struct BwdLayout {
-    size_t qt, kt, P, DS, partial, total;
+    size_t qt, kt, P, DS, partial, colsum, ticket, total;
     int nblocks;
 };
 
@@ -125,6 +125,8 @@ BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype) {
     L.P = off; off += align256((size_t)B * H * T * S * 4);
     L.DS = off; off += align256((size_t)B * H * T * S * 4);
     L.partial = off; off += align256((size_t)(L.nblocks > 0 ? L.nblocks : 1) * kMaxRungs * 4);
+    L.colsum = off; off += align256((size_t)kMaxRungs * 8);
+    L.ticket = off; off += 256;
     L.total = off;
     return L;
 }
@@ -334,6 +336,8 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, c
     a.qt = ws + L.qt; a.kt = ws + L.kt;
     a.P = reinterpret_cast<float*>(ws + L.P); a.DS = reinterpret_cast<float*>(ws + L.DS);
     a.partial = reinterpret_cast<float*>(ws + L.partial);
+    a.colsum = reinterpret_cast<double*>(ws + L.colsum);
+    a.ticket = reinterpret_cast<unsigned*>(ws + L.ticket);
     a.nblocks_a = B > 0 ? L.nblocks : 0;
     a.S = W + 1 + K;
     a.alpha = alpha;
@@ -361,6 +365,12 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, c
             e = launch_bwd_key(a, bf16, st);
         }
         if (e != cudaSuccess) return cuda_fail(e, "backward key-pass launch");
+    }
+    if (B == 0) {                                // no queries: every gradient is zero
+        e = cudaMemsetAsync(dtheta, 0, sizeof(float), st);
+        if (e == cudaSuccess && dd && K > 0) e = cudaMemsetAsync(dd, 0, sizeof(float) * K, st);
+        if (e != cudaSuccess) return cuda_fail(e, "zero gradients for an empty batch");
+        return FIBATTN_OK;
     }
     {
         ProfScope p("bwd_finalize", st);

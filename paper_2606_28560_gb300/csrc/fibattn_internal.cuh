@@ -68,6 +68,8 @@ struct BwdArgs {
     float* P;                 // softmax probabilities [B,H,T,S]
     float* DS;                // dL/dscore [B,H,T,S]
     float* partial;           // per-block dL/dd_k partial sums [nblocks][kMaxRungs]
+    double* colsum;           // dL/dd_k column sums [kMaxRungs]
+    unsigned* ticket;         // finalize completion counter (reset by the query pass)
     int nblocks_a;            // number of query-centric blocks (rows of partial)
     int S;                    // slots per query = W + 1 + K
     float alpha;

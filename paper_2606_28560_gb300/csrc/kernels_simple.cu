@@ -312,6 +312,7 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
         for (int w = 0; w < kThreads / 32; ++w) x += red[w][threadIdx.x];
         a.partial[(size_t)blockIdx.x * kMaxRungs + threadIdx.x] = x;
     }
+    if (blockIdx.x == 0 && threadIdx.x == 0) *a.ticket = 0u;
 }
 
 // Key-centric pass.  Key row j of kv head hk receives, from every query head
@@ -385,33 +386,41 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
     }
 }
 
-// Fixed-order sum of the per-block rung partials (fp64), then the chain rule
+// Fixed-order sum of the per-block rung partials, then the chain rule
 // dL/dalpha = sum_k f_k dL/dd_k and dL/dtheta = dL/dalpha (alpha-0.5)(1.5-alpha).
-// Thread t sums blocks t, t+256, ... in order; a fixed shared-memory tree then
-// combines the 256 partial sums, so the result does not depend on scheduling.
+// Block k sums column k: thread t adds rows t, t+256, ... in order, then a
+// fixed shared-memory tree combines the 256 sums (fp64), so the result does
+// not depend on scheduling.  The last block to finish (ticket counter, no
+// waiting) forms dL/dalpha and dL/dtheta from the K column sums and resets the
+// ticket for the next call.
 constexpr int kFinThreads = 256;
 __global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
     __shared__ double red[kFinThreads];
-    __shared__ double dd[kMaxRungs];
-    const int t = threadIdx.x;
-    for (int k = 0; k < a.r.K; ++k) {
-        double x = 0.0;
-        for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) x += (double)a.partial[(size_t)blk * kMaxRungs + k];
-        red[t] = x;
-        __syncthreads();
-        for (int w = kFinThreads / 2; w > 0; w >>= 1) {
-            if (t < w) red[t] += red[t + w];
-            __syncthreads();
-        }
-        if (t == 0) dd[k] = red[0];
+    __shared__ bool last;
+    const int t = threadIdx.x, k = blockIdx.x;
+    double x = 0.0;
+#pragma unroll 8
+    for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) x += (double)a.partial[(size_t)blk * kMaxRungs + k];
+    red[t] = x;
+    __syncthreads();
+    for (int w = kFinThreads / 2; w > 0; w >>= 1) {
+        if (t < w) red[t] += red[t + w];
         __syncthreads();
     }
-    if (t < a.r.K && a.dd) a.dd[t] = (float)dd[t];
     if (t == 0) {
+        a.colsum[k] = red[0];
+        if (a.dd) a.dd[k] = (float)red[0];
+        __threadfence();
+        last = atomicAdd(a.ticket, 1u) == (unsigned)(gridDim.x - 1);
+    }
+    __syncthreads();
+    if (last && t == 0) {
+        __threadfence();
         double da = 0.0;
-        for (int u = 0; u < a.r.K; ++u) da += (double)a.r.f[u] * dd[u];
+        for (int u = 0; u < a.r.K; ++u) da += (double)a.r.f[u] * ((volatile double*)a.colsum)[u];
         const double al = (double)a.alpha;
         *a.dtheta = (float)(da * (al - 0.5) * (1.5 - al));
+        *a.ticket = 0u;
     }
 }
 
@@ -465,7 +474,11 @@ cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st) {
 }
 
 cudaError_t launch_bwd_finalize(const BwdArgs& a, cudaStream_t st) {
-    bwd_finalize_kernel<<<1, kFinThreads, 0, st>>>(a);
+    if (a.r.K == 0) {                            // no rungs: dL/dtheta = 0
+        cudaError_t e = cudaMemsetAsync(a.dtheta, 0, sizeof(float), st);
+        return e != cudaSuccess ? e : cudaGetLastError();
+    }
+    bwd_finalize_kernel<<<a.r.K, kFinThreads, 0, st>>>(a);
     return cudaGetLastError();
 }
 
