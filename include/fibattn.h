@@ -122,6 +122,27 @@ int fibattn_base(int kind, int K, float* f);
 int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, float* alpha);
 
 /* ---------------------------------------------------------------------------
+ * Forward without a caller-provided workspace.  The paper has no counterpart;
+ * this serves callers that cannot allocate device memory -- a host framework
+ * that owns all device memory and gives its plugins only tensors, or a hot
+ * path where cudaMalloc's implicit device synchronisation is not allowed.
+ * Same arguments and results as fibattn_fwd without workspace/workspace_bytes.
+ * Scratch: one library-owned device array of FIBATTN_NOALLOC_SCRATCH_BYTES
+ * (32 MiB, enough for B*Hkv*T <= 262144 bf16 rows or 131072 fp32 rows), held
+ * by every GPU that loads the library until the process exits.  Calls that
+ * need more are rejected with FIBATTN_ERR_INVALID_ARG before any device work.
+ * The call allocates nothing (no cudaMalloc / cudaFree).  The first call on
+ * each device looks up the array's device address with that device current;
+ * make that first call before any stream capture.  Every call shares the one
+ * array and leaves its contents behind: calls that overlap on the GPU (other
+ * streams, other host threads) race on it and must be serialised by the caller.
+ * ------------------------------------------------------------------------- */
+#define FIBATTN_NOALLOC_SCRATCH_BYTES (32u << 20)
+int fibattn_fwd_noalloc(const void* q, const void* k, const void* v, void* out, float* lse,
+                        int B, int H, int T, int D, int W, float alpha, const float* offsets, int K,
+                        int dtype, const fibattn_opts* opts, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Opt-in kernel timing (no counterpart in the paper; used to attribute time
  * to kernels).  fibattn_profile_enable(1) clears the record and brackets every
  * later launch with CUDA events on the launch stream; (0) stops and clears.

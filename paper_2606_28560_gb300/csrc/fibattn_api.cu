@@ -153,6 +153,8 @@ cudaEvent_t prof_event() {
 }  // namespace
 
 namespace fibattn {
+int set_error(int code, const char* msg) { return fail(code, "%s", msg); }
+
 ProfScope::ProfScope(const char* name, cudaStream_t st) : name_(name), st_(st), start_(nullptr), on_(false) {
     std::lock_guard<std::mutex> g(g_prof_mu);
     if (!g_prof_on) return;

@@ -197,6 +197,9 @@ cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_finalize(const BwdArgs& a, cudaStream_t st);
 int bwd_simple_blocks(const Shape& s);
 
+// Records a message for fibattn_last_error() and returns `code`.
+int set_error(int code, const char* msg);
+
 // Opt-in per-kernel timing: when enabled, each launch is bracketed by CUDA
 // events recorded on the caller's stream (see fibattn_profile_* in the ABI).
 struct ProfScope {
