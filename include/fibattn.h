@@ -57,6 +57,10 @@ typedef struct {
     float scale;       /* score scale; <= 0 means 1/sqrt(D)                            */
     int   Hkv;         /* key/value heads (GQA); 0 means Hkv = H                       */
     int   no_dedup;    /* 0: drop rungs with d_k <= W [default]; 1: keep them          */
+    int   fwd_kernel;  /* forward kernel: 0 automatic [default]; 1 row-gather kernel;
+                          2 shared-memory staged CUDA-core kernel; 3 tensor-core
+                          kernel (2 and 3: bf16 I/O only; 3: W <= 16, K <= 16;
+                          FIBATTN_ERR_UNSUPPORTED when the choice does not apply) */
 } fibattn_opts;
 
 /* ---------------------------------------------------------------------------

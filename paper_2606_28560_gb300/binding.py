@@ -32,7 +32,7 @@ class FibattnError(RuntimeError):
 
 class Opts(ctypes.Structure):
     _fields_ = [("rope_base", ctypes.c_float), ("scale", ctypes.c_float),
-                ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int)]
+                ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int), ("fwd_kernel", ctypes.c_int)]
 
 
 def library_path() -> str:
@@ -86,8 +86,12 @@ def _iptr(a: np.ndarray):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
 
 
-def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True) -> Opts:
-    return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1)
+FWD_KERNELS = {"auto": 0, "gather": 1, "staged": 2, "mma": 3}
+
+
+def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto") -> Opts:
+    return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1,
+                FWD_KERNELS[fwd_kernel])
 
 
 def _dtype_code(t: torch.Tensor) -> int:
@@ -148,13 +152,13 @@ def bwd_workspace_bytes(B, H, T, W, K, dtype, Hkv=None, D=64) -> int:
 
 
 def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
-        out=None, lse=None, workspace=None, stream=None):
+        out=None, lse=None, workspace=None, stream=None, kernel="auto"):
     """Forward pass.  q [B,H,T,64]; k, v [B,Hkv,T,64] (fp32 or bf16, CUDA,
-    contiguous).  Returns (out, lse)."""
+    contiguous).  ``kernel``: "auto", "gather", "staged" or "mma".  Returns (out, lse)."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
-    o = _opts(rope_base, scale, Hkv, dedup)
+    o = _opts(rope_base, scale, Hkv, dedup, kernel)
     code = _dtype_code(q)
     for t in (q, k, v):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):

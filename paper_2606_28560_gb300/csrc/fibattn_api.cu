@@ -12,6 +12,8 @@
 
 #include "../../include/fibattn.h"
 #include "fibattn_internal.cuh"
+#include "fwd_staged.cuh"
+#include "fwd_mma.cuh"
 
 using namespace fibattn;
 
@@ -37,7 +39,7 @@ size_t rot_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
 
 struct Resolved {
     float rope_base, scale;
-    int Hkv, dedup;
+    int Hkv, dedup, fwd_kernel;
 };
 
 int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
@@ -45,6 +47,8 @@ int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
     r->scale = (o && o->scale > 0.f) ? o->scale : (float)(1.0 / std::sqrt((double)D));
     r->Hkv = (o && o->Hkv > 0) ? o->Hkv : H;
     r->dedup = (o && o->no_dedup) ? 0 : 1;
+    r->fwd_kernel = o ? o->fwd_kernel : 0;
+    if (r->fwd_kernel < 0 || r->fwd_kernel > 3) return fail(FIBATTN_ERR_INVALID_ARG, "fwd_kernel must be 0, 1, 2 or 3");
     if (!(r->rope_base > 1.f) || !std::isfinite(r->rope_base))
         return fail(FIBATTN_ERR_INVALID_ARG, "rope_base must be finite and > 1 (got %g)", (double)r->rope_base);
     if (!std::isfinite(r->scale)) return fail(FIBATTN_ERR_INVALID_ARG, "scale must be finite");
@@ -109,7 +113,7 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
 }
 
 struct BwdLayout {
-    size_t qt, kt, P, DS, partial, colsum, ticket, total;
+    size_t qt, kt, P, DP, Delta, partial, colsum, ticket, total;
     int nblocks;
 };
 
@@ -123,7 +127,8 @@ BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype) {
     L.qt = off; off += align256((size_t)B * H * T * kHeadDim * es);
     L.kt = off; off += align256((size_t)B * Hkv * T * kHeadDim * es);
     L.P = off; off += align256((size_t)B * H * T * S * 4);
-    L.DS = off; off += align256((size_t)B * H * T * S * 4);
+    L.DP = off; off += align256((size_t)B * H * T * S * 4);
+    L.Delta = off; off += align256((size_t)B * H * T * 4);
     L.partial = off; off += align256((size_t)(L.nblocks > 0 ? L.nblocks : 1) * kMaxRungs * 4);
     L.colsum = off; off += align256((size_t)kMaxRungs * 8);
     L.ticket = off; off += 256;
@@ -176,6 +181,15 @@ int fibattn_profile_enable(int on) {
     g_prof_on = on != 0;
     for (auto& r : g_prof_recs) { g_prof_pool.push_back(r.a); g_prof_pool.push_back(r.b); }
     g_prof_recs.clear();
+    // create the events up front so that recording during a timed region
+    // costs no event creation on the host
+    const size_t kPool = 1 << 14;
+    while (g_prof_on && g_prof_pool.size() < kPool) {
+        cudaEvent_t e = nullptr;
+        if (cudaEventCreate(&e) != cudaSuccess) break;
+        g_prof_pool.push_back(e);
+    }
+    g_prof_recs.reserve(kPool / 2);
     return FIBATTN_OK;
 }
 
@@ -296,7 +310,25 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
         e = launch_rope_rows(k, workspace, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
     }
     if (e != cudaSuccess) return cuda_fail(e, "rope prologue launch");
-    {
+    // bf16 I/O: the tensor-core kernel when its layout applies (W <= 16,
+    // K <= 16, shared memory fits), else the staged CUDA-core kernel, else the
+    // row-gather kernel (also the fp32 I/O path).
+    const size_t smem_limit = 227 * 1024;
+    MmaLayout ML;
+    StageLayout L;
+    const bool mma_ok = bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 3) && build_mma_layout(a.s, a.r, smem_limit, &ML);
+    const bool staged_ok = !mma_ok && bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 2) &&
+                           build_stage_layout(a.s, a.r, o.rope_base, smem_limit, &L);
+    if ((o.fwd_kernel == 3 && !mma_ok) || (o.fwd_kernel == 2 && !staged_ok))
+        return fail(FIBATTN_ERR_UNSUPPORTED, "requested forward kernel does not apply to these arguments "
+                                             "(bf16 I/O, W <= 16, K <= 16, shared-memory layout)");
+    if (mma_ok) {
+        ProfScope p("fwd", st);
+        e = launch_fwd_mma(a, ML, st);
+    } else if (staged_ok) {
+        ProfScope p("fwd", st);
+        e = launch_fwd_staged(a, L, bf16, st);
+    } else {
         ProfScope p("fwd", st);
         e = launch_fwd_simple(a, bf16, st);
     }
@@ -336,7 +368,8 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, c
     a.q = q; a.k = k; a.v = v; a.lse = lse; a.dout = dout; a.dq = dq; a.dk = dk; a.dv = dv;
     a.dtheta = dtheta; a.dd = dd;
     a.qt = ws + L.qt; a.kt = ws + L.kt;
-    a.P = reinterpret_cast<float*>(ws + L.P); a.DS = reinterpret_cast<float*>(ws + L.DS);
+    a.P = reinterpret_cast<float*>(ws + L.P); a.DP = reinterpret_cast<float*>(ws + L.DP);
+    a.Delta = reinterpret_cast<float*>(ws + L.Delta);
     a.partial = reinterpret_cast<float*>(ws + L.partial);
     a.colsum = reinterpret_cast<double*>(ws + L.colsum);
     a.ticket = reinterpret_cast<unsigned*>(ws + L.ticket);

@@ -66,7 +66,8 @@ struct BwdArgs {
     void* qt;                 // rotated q [B,H,T,D]
     void* kt;                 // rotated k [B,Hkv,T,D]
     float* P;                 // softmax probabilities [B,H,T,S]
-    float* DS;                // dL/dscore [B,H,T,S]
+    float* DP;                // dL/dp = dO . val per slot [B,H,T,S]
+    float* Delta;             // sum_slots p dL/dp per query [B,H,T]
     float* partial;           // per-block dL/dd_k partial sums [nblocks][kMaxRungs]
     double* colsum;           // dL/dd_k column sums [kMaxRungs]
     unsigned* ticket;         // finalize completion counter (reset by the query pass)

@@ -1,0 +1,506 @@
+// fwd_mma.cu -- forward pass on tensor cores (mma.sync, m16n8) with TMA
+// staging (arXiv 2606.28560, Section 2 "Attended set").
+//
+// A warp owns one 16-row tile of queries, tiles placed every 15 queries (the
+// 16th row duplicates the next tile's first query and is discarded), so for a
+// rung with floor s0 the 16 slab rows [b-s0-1, b-s0+15) hold both rows every
+// valid query of the tile reads: query u reads slab row u (far, weight w) and
+// row u+1 (floor, weight 1-w).  Scores:
+//   window band  S = Q~ K~[b-Wp, b+16)^T   (16 x (16+Wp), the causal band t=0..W)
+//   rung k       S = Q~ K~[b-s0-1, +16)^T (16 x 16; the diagonal and the first
+//                superdiagonal are the far and floor scores)
+// The interpolated rung score (1-w) S[u][u+1] + w S[u][u] is summed inside the
+// quad of lanes that share a row.  Softmax is two-pass in registers (row max,
+// then P); the probability-weighted values are again 16x8 MMAs:
+//   window band  O += P_band V[b-Wp, b+16)
+//   rung k       O += Phat_k V[b-s0-1, +16),  Phat_k[u][u] = p w, Phat_k[u][u+1] = p (1-w)
+//
+// Precision (bf16 I/O): q~ and k~ enter the score MMAs as fp16 (11-bit
+// significands); P of the window band is the unnormalised exp(s - max) in
+// bf16, so the largest entry of each row is exactly 1; Phat of a rung carries
+// arbitrary interpolation weights and is split into bf16 hi + lo parts (two
+// MMAs), which keeps the weights exact to ~2^-17.  Row sums use the same
+// rounded values.  Accumulation is fp32.
+//
+// Staging: the CTA's union of key rows (rotated keys, fp16) and then of value
+// rows (bf16, same buffer) is copied by TMA (3-D tensor maps [heads][T][64],
+// 8-row boxes, 128-byte swizzle, rows outside [0, T) zero-filled) under an
+// mbarrier with a bounded wait.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include "fibattn_internal.cuh"
+#include "fwd_mma.cuh"
+
+namespace fibattn {
+namespace {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kLn2 = 0.6931471805599453f;
+constexpr int kWarps = kMmaWarps;
+constexpr int kRowsPerWarp = 15;                 // useful query rows of a 16-row tile
+constexpr unsigned kWaitLimit = 1u << 26;        // mbarrier polls before giving up
+
+// ------------------------------------------------------------------ PTX ----
+
+__device__ __forceinline__ unsigned smem_u32(const void* p) { return (unsigned)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(unsigned long long* bar, unsigned count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" :: "r"(smem_u32(bar)), "r"(count));
+}
+__device__ __forceinline__ void mbar_expect_tx(unsigned long long* bar, unsigned bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" :: "r"(smem_u32(bar)), "r"(bytes));
+}
+// Bounded wait on phase `parity`; returns false after kWaitLimit polls.
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity) {
+    const unsigned a = smem_u32(bar);
+    for (unsigned it = 0; it < kWaitLimit; ++it) {
+        unsigned done;
+        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+                     " selp.u32 %0, 1, 0, p;\n}\n" : "=r"(done) : "r"(a), "r"(parity) : "memory");
+        if (done) return true;
+    }
+    return false;
+}
+__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
+                                            unsigned long long* bar) {
+    asm volatile("cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
+                 " [%0], [%1, {%2, %3, %4}], [%5];\n"
+                 :: "r"(smem_u32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)) : "memory");
+}
+
+__device__ __forceinline__ void ldsm_x4(unsigned addr, unsigned& r0, unsigned& r1, unsigned& r2, unsigned& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+__device__ __forceinline__ void ldsm_x4_t(unsigned addr, unsigned& r0, unsigned& r1, unsigned& r2, unsigned& r3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
+                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
+}
+
+__device__ __forceinline__ void mma_f16_16816(float* d, const unsigned* a, unsigned b0, unsigned b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%0,%1,%2,%3};\n"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_bf16_16816(float* d, const unsigned* a, unsigned b0, unsigned b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%0,%1,%2,%3};\n"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+__device__ __forceinline__ void mma_bf16_1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
+    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, "
+                 "{%0,%1,%2,%3};\n"
+                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3]) : "r"(a0), "r"(a1), "r"(b0));
+}
+
+__device__ __forceinline__ unsigned pack_f16(float lo, float hi) {
+    __half2 h = __floats2half2_rn(lo, hi);
+    return *reinterpret_cast<unsigned*>(&h);
+}
+__device__ __forceinline__ unsigned pack_bf16(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<unsigned*>(&h);
+}
+__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
+
+__device__ __forceinline__ float quad_sum(float x) {
+    x += __shfl_xor_sync(0xffffffffu, x, 1);
+    x += __shfl_xor_sync(0xffffffffu, x, 2);
+    return x;
+}
+__device__ __forceinline__ float quad_max(float x) {
+    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 1));
+    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 2));
+    return x;
+}
+
+// Shared-memory byte address of 16-byte chunk `ch` of staged row `row` under the
+// 128-byte swizzle (chunk index XOR row % 8), buffer base 1024-byte aligned.
+__device__ __forceinline__ unsigned row_chunk(unsigned base, int row, int ch) {
+    return base + (unsigned)row * 128u + (unsigned)((ch ^ (row & 7)) << 4);
+}
+
+template <int NT>
+__global__ void __launch_bounds__(kWarps * 32, 2)
+fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+               FwdArgs a, MmaLayout L) {
+    constexpr int Wp = NT * 8 - 16;               // window rows before the tile
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ unsigned long long bars[2];
+    unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const unsigned sbase = smem_u32(buf);
+
+    const Shape s = a.s;
+    const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
+    const int bh = blockIdx.x / tiles;
+    const int i0 = (blockIdx.x % tiles) * kMmaTile;
+    const int b = bh / s.H, h = bh % s.H, hk = h / s.G;
+    const int head = b * s.Hkv + hk;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int g4 = lane >> 2, c4 = lane & 3;
+    const int wrel = warp * kRowsPerWarp;         // tile-relative first row of this warp
+    const int bw = i0 + wrel;                     // absolute first row
+
+    // ---- issue the key copies (one elected thread)
+    if (tid == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+        mbar_expect_tx(&bars[0], (unsigned)L.rows * 128u);
+        for (int iv = 0; iv < L.n_iv; ++iv)
+            for (int r = 0; r < L.iv_len[iv]; r += 8)
+                tma_load_3d(buf + (size_t)(L.iv_smem[iv] + r) * 128, &tmK, 0, i0 + L.iv_start[iv] + r, head, &bars[0]);
+    }
+
+    // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32)
+    // Thread dims: 16kc + 2c4 + {0,1} and 16kc + 8 + 2c4 + {0,1} for kc = 0..3.
+    unsigned qa[4][4];
+    {
+        const __nv_bfloat16* Q = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)bh * s.T) * kHeadDim;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int pos = min(bw + g4 + 8 * half, s.T - 1);
+            const __nv_bfloat16* row = Q + (size_t)pos * kHeadDim;
+            float x[4][4];                        // [kc][j]: dims 16kc + {2c4, 2c4+1, 2c4+8, 2c4+9}
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                const unsigned u0 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 2 * c4);
+                const unsigned u1 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 8 + 2 * c4);
+                x[kc][0] = __uint_as_float(u0 << 16); x[kc][1] = __uint_as_float(u0 & 0xffff0000u);
+                x[kc][2] = __uint_as_float(u1 << 16); x[kc][3] = __uint_as_float(u1 & 0xffff0000u);
+            }
+#pragma unroll
+            for (int kc = 0; kc < 2; ++kc) {      // pair (dim m in kc, dim m+32 in kc+2)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
+                    float cs, sn;
+                    rope_cs(a.rope, m, pos, cs, sn);
+                    const float xa = x[kc][j], xb = x[kc + 2][j];
+                    x[kc][j] = xa * cs - xb * sn;
+                    x[kc + 2][j] = xb * cs + xa * sn;
+                }
+            }
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);       // a0 / a1: k = 2c4, 2c4+1
+                qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);   // a2 / a3: k = 2c4+8, 2c4+9
+            }
+        }
+    }
+    const float sc2 = s.scale * kLog2e;           // scores in log2 units
+    const int qlo = bw + g4, qhi = bw + g4 + 8;   // absolute queries of this thread's rows
+    const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
+    const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
+
+    __syncthreads();                              // barrier init visible
+    const bool ok_k = mbar_wait(&bars[0], 0);
+
+    // ---- window band scores: keys [bw - Wp, bw + 16), n-tile j covers 8 keys
+    float sw[NT][4];
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+        sw[j][0] = sw[j][1] = sw[j][2] = sw[j][3] = 0.f;
+        const int krow = L.win_smem + wrel - Wp + 8 * j + (lane & 7);
+#pragma unroll
+        for (int kc = 0; kc < 4; kc += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+            mma_f16_16816(sw[j], qa[kc], b0, b1);
+            mma_f16_16816(sw[j], qa[kc + 1], b2, b3);
+        }
+    }
+    float mlo = -INFINITY, mhi = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const int r = (e < 2) ? g4 : g4 + 8;
+            const int n = 8 * j + 2 * c4 + (e & 1);
+            const int t = r + Wp - n;                     // distance query - key
+            const int key = bw - Wp + n;
+            const bool ok = (e < 2 ? vlo : vhi) && t >= 0 && t <= s.W && key >= 0;
+            sw[j][e] = ok ? sw[j][e] * sc2 : -INFINITY;
+            if (e < 2) mlo = fmaxf(mlo, sw[j][e]); else mhi = fmaxf(mhi, sw[j][e]);
+        }
+    }
+    mlo = quad_max(mlo);
+    mhi = quad_max(mhi);
+
+    // ---- rung scores: slab rows x = 0..15 at absolute bw - s0 - 1 + x.
+    // Row r's far score is column x = r, its floor score column x = r + 1.
+    // Columns 2c4 + {0,1} of n-tile t belong to this thread.
+    const int xf_lo = g4, xl_lo = g4 + 1, xf_hi = g4 + 8, xl_hi = g4 + 9;
+    const bool own_f_lo = ((xf_lo & 7) >> 1) == c4, own_l_lo = ((xl_lo & 7) >> 1) == c4;
+    const bool own_f_hi = ((xf_hi & 7) >> 1) == c4, own_l_hi = ((xl_hi & 7) >> 1) == c4 && xl_hi < 16;
+    float rs[kMmaMaxRungs][2];
+#pragma unroll
+    for (int k = 0; k < kMmaMaxRungs; ++k) { rs[k][0] = -INFINITY; rs[k][1] = -INFINITY; }
+#pragma unroll
+    for (int k = 0; k < kMmaMaxRungs; ++k) {
+        if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
+        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;        // masked for the whole warp
+        const float w = a.r.w[k], w1 = 1.f - w;
+        float st[2][4];
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+            st[t][0] = st[t][1] = st[t][2] = st[t][3] = 0.f;
+            const int krow = L.rung_smem[k] + wrel + 8 * t + (lane & 7);
+#pragma unroll
+            for (int kc = 0; kc < 4; kc += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                mma_f16_16816(st[t], qa[kc], b0, b1);
+                mma_f16_16816(st[t], qa[kc + 1], b2, b3);
+            }
+        }
+        // element of (row half, column x): n-tile x >> 3, register 2*half + (x & 1)
+        float plo = 0.f, phi = 0.f;
+        {
+            // row lo: far column g4 lies in n-tile 0; floor column g4+1 in n-tile (g4+1)>>3
+            const float f_lo = (xf_lo & 1) ? st[0][1] : st[0][0];
+            const float l_lo0 = (xl_lo & 1) ? st[0][1] : st[0][0];
+            const float l_lo1 = (xl_lo & 1) ? st[1][1] : st[1][0];
+            const float l_lo = (xl_lo >> 3) ? l_lo1 : l_lo0;
+            const float f_hi = (xf_hi & 1) ? st[1][3] : st[1][2];
+            const float l_hi = (xl_hi & 1) ? st[1][3] : st[1][2];
+            plo = (own_f_lo ? w * f_lo : 0.f) + (own_l_lo ? w1 * l_lo : 0.f);
+            phi = (own_f_hi ? w * f_hi : 0.f) + (own_l_hi ? w1 * l_hi : 0.f);
+        }
+        plo = quad_sum(plo) * sc2;
+        phi = quad_sum(phi) * sc2;
+        const float dk = a.r.d[k];
+        rs[k][0] = (vlo && dk <= (float)qlo) ? plo : -INFINITY;
+        rs[k][1] = (vhi && dk <= (float)qhi) ? phi : -INFINITY;
+        mlo = fmaxf(mlo, rs[k][0]);
+        mhi = fmaxf(mhi, rs[k][1]);
+    }
+
+    // ---- all warps are done with the keys: stage the values into the same buffer
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+    __syncthreads();
+    if (tid == 0) {
+        mbar_expect_tx(&bars[1], (unsigned)L.rows * 128u);
+        for (int iv = 0; iv < L.n_iv; ++iv)
+            for (int r = 0; r < L.iv_len[iv]; r += 8)
+                tma_load_3d(buf + (size_t)(L.iv_smem[iv] + r) * 128, &tmV, 0, i0 + L.iv_start[iv] + r, head, &bars[1]);
+    }
+
+    // ---- probabilities (unnormalised, row max -> exactly 1) while values arrive
+    if (mlo == -INFINITY) mlo = 0.f;              // rows beyond T: keep arithmetic finite
+    if (mhi == -INFINITY) mhi = 0.f;
+    float llo = 0.f, lhi = 0.f;
+    unsigned pa[NT][2];                           // window band P as bf16 A fragments
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+        const float p0 = bf16_round(exp2f(sw[j][0] - mlo)), p1 = bf16_round(exp2f(sw[j][1] - mlo));
+        const float p2 = bf16_round(exp2f(sw[j][2] - mhi)), p3 = bf16_round(exp2f(sw[j][3] - mhi));
+        llo += p0 + p1;
+        lhi += p2 + p3;
+        pa[j][0] = pack_bf16(p0, p1);
+        pa[j][1] = pack_bf16(p2, p3);
+    }
+    llo = quad_sum(llo);
+    lhi = quad_sum(lhi);
+
+    const bool ok_v = mbar_wait(&bars[1], 0);
+
+    float o[8][4];
+#pragma unroll
+    for (int n = 0; n < 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+
+    // ---- window band values: k-chunks of 16 keys (+ one of 8 when NT is odd)
+#pragma unroll
+    for (int kk = 0; kk + 1 < NT; kk += 2) {
+        const unsigned afr[4] = {pa[kk][0], pa[kk][1], pa[kk + 1][0], pa[kk + 1][1]};
+        const int vrow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+        for (int n = 0; n < 8; n += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
+            mma_bf16_16816(o[n], afr, b0, b1);
+            mma_bf16_16816(o[n + 1], afr, b2, b3);
+        }
+    }
+    if constexpr (NT & 1) {
+        const int kk = NT - 1;
+        const int vrow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7);
+#pragma unroll
+        for (int n = 0; n < 8; n += 4) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 3)), b0, b1, b2, b3);
+            mma_bf16_1688(o[n], pa[kk][0], pa[kk][1], b0);
+            mma_bf16_1688(o[n + 1], pa[kk][0], pa[kk][1], b1);
+            mma_bf16_1688(o[n + 2], pa[kk][0], pa[kk][1], b2);
+            mma_bf16_1688(o[n + 3], pa[kk][0], pa[kk][1], b3);
+        }
+    }
+
+    // ---- rung values: Phat[r][x] = p_r w at x = r, p_r (1-w) at x = r + 1
+    // A-fragment columns of this thread: 2c4 + {0,1} (a0, a1) and 2c4 + 8 + {0,1} (a2, a3).
+#pragma unroll
+    for (int k = 0; k < kMmaMaxRungs; ++k) {
+        if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
+        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
+        const float w = a.r.w[k], w1 = 1.f - w;
+        const float plo = exp2f(rs[k][0] - mlo), phi = exp2f(rs[k][1] - mhi);   // 0 when masked
+        llo += plo;
+        lhi += phi;
+        float ev[2][4];                           // [row half][column slot]
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int r = g4 + 8 * half;
+            const float p = half ? phi : plo;
+#pragma unroll
+            for (int cs = 0; cs < 4; ++cs) {
+                const int x = 2 * c4 + (cs & 1) + 8 * (cs >> 1);
+                ev[half][cs] = (x == r) ? p * w : ((x == r + 1) ? p * w1 : 0.f);
+            }
+        }
+        unsigned ahi[4], alo[4];
+#pragma unroll
+        for (int cs = 0; cs < 4; cs += 2) {
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const float e0 = ev[half][cs], e1 = ev[half][cs + 1];
+                const float h0 = bf16_round(e0), h1 = bf16_round(e1);
+                ahi[(cs >> 1) * 2 + half] = pack_bf16(h0, h1);
+                alo[(cs >> 1) * 2 + half] = pack_bf16(e0 - h0, e1 - h1);
+            }
+        }
+        const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+        for (int n = 0; n < 8; n += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
+            mma_bf16_16816(o[n], ahi, b0, b1);
+            mma_bf16_16816(o[n + 1], ahi, b2, b3);
+            mma_bf16_16816(o[n], alo, b0, b1);
+            mma_bf16_16816(o[n + 1], alo, b2, b3);
+        }
+    }
+
+    // ---- normalise and store rows 0..14 of the tile
+    const bool ok = ok_k && ok_v;
+    const float inv_lo = ok ? 1.f / llo : __int_as_float(0x7fc00000);
+    const float inv_hi = ok ? 1.f / lhi : __int_as_float(0x7fc00000);
+    __nv_bfloat16* O = reinterpret_cast<__nv_bfloat16*>(a.out) + ((size_t)bh * s.T) * kHeadDim;
+    if (vlo && wrel + g4 < kMmaTile) {
+        __nv_bfloat16* row = O + (size_t)qlo * kHeadDim;
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+            *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][0] * inv_lo, o[n][1] * inv_lo);
+        if (c4 == 0) a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
+    }
+    if (vhi && wrel + g4 + 8 < kMmaTile) {
+        __nv_bfloat16* row = O + (size_t)qhi * kHeadDim;
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+            *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][2] * inv_hi, o[n][3] * inv_hi);
+        if (c4 == 0) a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
+    }
+}
+
+// ------------------------------------------------------------ host side ----
+
+PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess && q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads) {
+    auto fn = get_encode();
+    if (!fn) return false;
+    cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)T, (cuuint64_t)heads};
+    cuuint64_t strides[2] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)T * kHeadDim * 2};
+    cuuint32_t box[3] = {(cuuint32_t)kHeadDim, 8, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = fn(map, dt, 3, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+template <int NT>
+cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const FwdArgs& a, const MmaLayout& L,
+                      unsigned grid, size_t smem, cudaStream_t st) {
+    auto kern = fwd_mma_kernel<NT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kWarps * 32, smem, st>>>(mk, mv, a, L);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.rows * 128 + 1024; }
+
+bool build_mma_layout(const Shape& s, const RungParams& r, size_t smem_limit, MmaLayout* L) {
+    if (s.W > 16 || r.K > kMmaMaxRungs) return false;
+    const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
+    const int Wp = NT * 8 - 16;
+    L->nt = NT;
+    // relative rows each warp tile reads; the tile spans rows [0, kMmaTile + 1)
+    struct Iv { int a, b; };
+    Iv iv[kMmaMaxRungs + 1];
+    int n = 0;
+    iv[n++] = {-Wp, kMmaTile + 1};
+    for (int k = 0; k < r.K; ++k)
+        if ((r.active >> k) & 1u) iv[n++] = {-r.s0[k] - 1, kMmaTile + 1 - r.s0[k]};
+    for (int i = 1; i < n; ++i)                   // insertion sort by start
+        for (int j = i; j > 0 && iv[j].a < iv[j - 1].a; --j) { Iv t = iv[j]; iv[j] = iv[j - 1]; iv[j - 1] = t; }
+    int m = 0;
+    for (int i = 0; i < n; ++i) {
+        if (m > 0 && iv[i].a <= iv[m - 1].b) { if (iv[i].b > iv[m - 1].b) iv[m - 1].b = iv[i].b; }
+        else iv[m++] = iv[i];
+    }
+    L->n_iv = m;
+    int rows = 0;
+    for (int i = 0; i < m; ++i) {
+        const int len = ((iv[i].b - iv[i].a) + 7) & ~7;      // whole 8-row TMA boxes
+        L->iv_start[i] = iv[i].a;
+        L->iv_len[i] = len;
+        L->iv_smem[i] = rows;
+        rows += len;
+    }
+    L->rows = rows;
+    auto smem_row = [&](int rel) {
+        for (int i = 0; i < L->n_iv; ++i)
+            if (rel >= L->iv_start[i] && rel < L->iv_start[i] + L->iv_len[i]) return L->iv_smem[i] + (rel - L->iv_start[i]);
+        return -1;
+    };
+    L->win_smem = smem_row(0);
+    for (int k = 0; k < kMmaMaxRungs; ++k) L->rung_smem[k] = 0;
+    for (int k = 0; k < r.K; ++k)
+        if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row(-r.s0[k] - 1);
+    return fwd_mma_smem_bytes(*L) <= smem_limit;
+}
+
+cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st) {
+    const long long tiles = (a.s.T + kMmaTile - 1) / kMmaTile;
+    const long long grid = tiles * a.s.B * a.s.H;
+    if (grid <= 0) return cudaSuccess;
+    CUtensorMap mk, mv;
+    const int heads = a.s.B * a.s.Hkv;
+    if (!encode_rows_map(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
+        !encode_rows_map(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
+        return cudaErrorInvalidValue;
+    const size_t smem = fwd_mma_smem_bytes(L);
+    switch (L.nt) {
+    case 2: return launch_nt<2>(mk, mv, a, L, (unsigned)grid, smem, st);
+    case 3: return launch_nt<3>(mk, mv, a, L, (unsigned)grid, smem, st);
+    default: return launch_nt<4>(mk, mv, a, L, (unsigned)grid, smem, st);
+    }
+}
+
+}  // namespace fibattn

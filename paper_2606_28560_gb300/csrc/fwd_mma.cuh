@@ -1,0 +1,29 @@
+// fwd_mma.cuh -- host/device interface of the tensor-core forward kernel.
+#pragma once
+#include "fibattn_internal.cuh"
+
+namespace fibattn {
+
+constexpr int kMmaWarps = 8;                      // one 16-row MMA tile per warp
+constexpr int kMmaTile = kMmaWarps * 15;          // queries per CTA (tiles every 15 rows)
+constexpr int kMmaMaxRungs = 16;
+
+// Rows a CTA stages, relative to its first query: merged intervals of the
+// window band [-Wp, M+1) and the rung slabs [-s0-1, M+1-s0), each rounded up
+// to whole 8-row TMA boxes and stored from shared row iv_smem[n].
+struct MmaLayout {
+    int n_iv;
+    int rows;
+    int nt;                                       // window n-tiles: 16 + Wp = 8 nt keys
+    int win_smem;                                 // shared row of relative row 0
+    int iv_start[kMmaMaxRungs + 1];
+    int iv_len[kMmaMaxRungs + 1];
+    int iv_smem[kMmaMaxRungs + 1];
+    int rung_smem[kMmaMaxRungs];                  // shared row of relative row -s0_k - 1
+};
+
+bool build_mma_layout(const Shape& s, const RungParams& r, size_t smem_limit, MmaLayout* L);
+size_t fwd_mma_smem_bytes(const MmaLayout& L);
+cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st);
+
+}  // namespace fibattn

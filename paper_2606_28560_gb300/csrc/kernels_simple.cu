@@ -158,14 +158,22 @@ __global__ void __launch_bounds__(kThreads) fwd_simple_kernel(FwdArgs a) {
 
 // ------------------------------------------------------------ backward ----
 
-// Query-centric pass.  For query i: recompute p = exp(score - lse) for every
-// slot, Delta = sum_slots p * (dO . val), dS = p (dO . val - Delta); then
-// dq~ = scale sum dS key, and per rung
-//   dL/dd_k += scale dS (q~ . (k~[j1] - k~[j0])) + p (dO . (v[j1] - v[j0])).
-// Writes P and DS (zero for slots that are not attended) for the key pass.
+// Query-centric pass, one sweep over the attended slots of query i.  With
+// p = exp(score - lse), dp = dO . val and Delta = sum_slots p dp (= dO . o),
+// dL/dscore = p (dp - Delta), so
+//   dq~ = scale sum_slots p (dp - Delta) key = scale (A - Delta B),
+//   A = sum p dp key,  B = sum p key,
+// and for rung k (d key / d d_k = k~[j1] - k~[j0], d val / d d_k = v[j1] - v[j0];
+// row -1 is a zero row)
+//   dL/dd_k += scale p (dp - Delta) q~.(k~[j1]-k~[j0]) + p dO.(v[j1]-v[j0])
+//            = t1 - Delta t2,  t1 = scale p ds_k dp + p ddp_k,  t2 = scale p ds_k.
+// A, B, t1, t2 and Delta accumulate in the same sweep.  P, dp (per slot, zero
+// where not attended) and Delta (per query) go to the workspace for the key
+// pass, which forms dL/dscore = P (dp - Delta).
 template <typename T>
 __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
-    __shared__ float red[kThreads / 32][kMaxRungs];
+    __shared__ float tsm[kRowsPerBlock][kMaxRungs][2];   // per-query t1, t2 of each rung
+    __shared__ float dsm[kRowsPerBlock];                 // per-query Delta (0 when i >= T)
     const Shape s = a.s;
     const int lane = threadIdx.x & 31, c = lane & 3, warp = threadIdx.x >> 5;
     const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
@@ -184,55 +192,21 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
     const R* Kt = reinterpret_cast<const R*>(a.kt) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
     const T* V = reinterpret_cast<const T*>(a.v) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
     float* Prow = a.P + ((size_t)bh * s.T + ii) * a.S;
-    float* DSrow = a.DS + ((size_t)bh * s.T + ii) * a.S;
+    float* DProw = a.DP + ((size_t)bh * s.T + ii) * a.S;
 
     float q[16], go[16], kr[16], kf[16], vr[16], vf[16];
     load_chunk(Qt + (size_t)ii * kHeadDim, c, q);
     load_chunk(dO + (size_t)ii * kHeadDim, c, go);
 
-    // pass 1: Delta = sum_slots p * (dO . val)
+    float A[16], Bv[16];
+#pragma unroll
+    for (int e = 0; e < 16; ++e) { A[e] = 0.f; Bv[e] = 0.f; }
     float delta = 0.f;
-    for (int t = 0; t <= s.W; ++t) {
-        const int j = ii - t;
-        const bool ok = j >= 0;
-        const int jj = ok ? j : 0;
-        load_chunk(Kt + (size_t)jj * kHeadDim, c, kr);
-        load_chunk(V + (size_t)jj * kHeadDim, c, vr);
-        const float sco = group_sum(dot16(q, kr)) * sc2;
-        const float dp = group_sum(dot16(go, vr));
-        if (ok) delta = fmaf(exp2f(sco - lse2), dp, delta);
-        if (__all_sync(0xffffffffu, !ok)) break;
-    }
-    for (int k = 0; k < a.r.K; ++k) {
-        if (!((a.r.active >> k) & 1u)) continue;
-        const int s0 = a.r.s0[k];
-        const float w = a.r.w[k];
-        const bool ok = a.r.d[k] <= fi;
-        const int j0 = ok ? ii - s0 : 0;
-        const bool far = w != 0.f;
-        const bool hasf = ok && far && j0 >= 1;
-        const int j1 = hasf ? j0 - 1 : 0;
-        load_chunk(Kt + (size_t)j0 * kHeadDim, c, kr);
-        load_chunk(V + (size_t)j0 * kHeadDim, c, vr);
-        float s0r = dot16(q, kr), dp0 = dot16(go, vr), s1r = 0.f, dp1 = 0.f;
-        if (far) {
-            load_chunk(Kt + (size_t)j1 * kHeadDim, c, kf);
-            load_chunk(V + (size_t)j1 * kHeadDim, c, vf);
-            if (hasf) { s1r = dot16(q, kf); dp1 = dot16(go, vf); }
-        }
-        const float sco = group_sum((1.f - w) * s0r + w * s1r) * sc2;
-        const float dp = group_sum((1.f - w) * dp0 + w * dp1);
-        if (ok) delta = fmaf(exp2f(sco - lse2), dp, delta);
-    }
+    const int qloc = threadIdx.x >> 2;
+    if (c == 0)
+        for (int k = 0; k < kMaxRungs; ++k) { tsm[qloc][k][0] = 0.f; tsm[qloc][k][1] = 0.f; }
 
-    // pass 2: dS, dq~, rung gradients, P / DS for the key pass
-    float dq[16];
-#pragma unroll
-    for (int e = 0; e < 16; ++e) dq[e] = 0.f;
-    float g[kMaxRungs];
-#pragma unroll
-    for (int k = 0; k < kMaxRungs; ++k) g[k] = 0.f;
-
+    // window slots t = 0..W
     for (int t = 0; t <= s.W; ++t) {
         const int j = ii - t;
         const bool ok = j >= 0;
@@ -242,75 +216,75 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
         const float sco = group_sum(dot16(q, kr)) * sc2;
         const float dp = group_sum(dot16(go, vr));
         const float p = ok ? exp2f(sco - lse2) : 0.f;
-        const float ds = p * (dp - delta);
-        const float dss = ds * s.scale;
+        const float pdp = p * dp;
+        delta += pdp;
 #pragma unroll
-        for (int e = 0; e < 16; ++e) dq[e] = fmaf(dss, kr[e], dq[e]);
-        if (qvalid && c == 0) { Prow[t] = p; DSrow[t] = ds; }
+        for (int e = 0; e < 16; ++e) { A[e] = fmaf(pdp, kr[e], A[e]); Bv[e] = fmaf(p, kr[e], Bv[e]); }
+        if (qvalid && c == 0) { Prow[t] = p; DProw[t] = ok ? dp : 0.f; }
         if (__all_sync(0xffffffffu, j < 0)) {
             if (qvalid && c == 0)
-                for (int u = t + 1; u <= s.W; ++u) { Prow[u] = 0.f; DSrow[u] = 0.f; }
+                for (int u = t + 1; u <= s.W; ++u) { Prow[u] = 0.f; DProw[u] = 0.f; }
             break;
         }
     }
+    // rungs
     for (int k = 0; k < a.r.K; ++k) {
         const int slot = s.W + 1 + k;
         if (!((a.r.active >> k) & 1u)) {
-            if (qvalid && c == 0) { Prow[slot] = 0.f; DSrow[slot] = 0.f; }
+            if (qvalid && c == 0) { Prow[slot] = 0.f; DProw[slot] = 0.f; }
             continue;
         }
         const int s0 = a.r.s0[k];
         const float w = a.r.w[k];
         const bool ok = a.r.d[k] <= fi;
         const int j0 = ok ? ii - s0 : 0;
-        // the far row enters dL/dd_k even at w == 0 (one-sided derivative);
-        // row -1 (only when d_k == i) is a zero row
-        const bool hasf = ok && j0 >= 1;
+        const bool hasf = ok && j0 >= 1;          // far row -1 is a zero row
         const int j1 = hasf ? j0 - 1 : 0;
         load_chunk(Kt + (size_t)j0 * kHeadDim, c, kr);
         load_chunk(V + (size_t)j0 * kHeadDim, c, vr);
-        float s0r = dot16(q, kr), dp0 = dot16(go, vr), s1r = 0.f, dp1 = 0.f;
         load_chunk(Kt + (size_t)j1 * kHeadDim, c, kf);
         load_chunk(V + (size_t)j1 * kHeadDim, c, vf);
+        float s0r = dot16(q, kr), dp0 = dot16(go, vr), s1r = 0.f, dp1 = 0.f;
         if (hasf) { s1r = dot16(q, kf); dp1 = dot16(go, vf); }
         s0r = group_sum(s0r); s1r = group_sum(s1r);
         dp0 = group_sum(dp0); dp1 = group_sum(dp1);
-        const float sco = ((1.f - w) * s0r + w * s1r) * sc2;
-        const float dp = (1.f - w) * dp0 + w * dp1;
+        const float w1 = 1.f - w;
+        const float sco = (w1 * s0r + w * s1r) * sc2;
+        const float dp = w1 * dp0 + w * dp1;
         const float p = ok ? exp2f(sco - lse2) : 0.f;
-        const float ds = p * (dp - delta);
-        const float dss = ds * s.scale;
-        const float c0 = dss * (1.f - w), c1 = dss * w;
+        const float pdp = p * dp;
+        delta += pdp;
+        const float fw0 = w1, fw1 = hasf ? w : 0.f;
 #pragma unroll
-        for (int e = 0; e < 16; ++e) dq[e] = fmaf(c0, kr[e], dq[e]);
-        if (hasf) {
-#pragma unroll
-            for (int e = 0; e < 16; ++e) dq[e] = fmaf(c1, kf[e], dq[e]);
+        for (int e = 0; e < 16; ++e) {
+            const float key = fw0 * kr[e] + fw1 * kf[e];
+            A[e] = fmaf(pdp, key, A[e]);
+            Bv[e] = fmaf(p, key, Bv[e]);
         }
-        // d(key)/d(d_k) = k~[j1] - k~[j0], d(val)/d(d_k) = v[j1] - v[j0] (row -1 is zero)
-        if (qvalid && ok) g[k] += dss * (s1r - s0r) + p * (dp1 - dp0);
-        if (qvalid && c == 0) { Prow[slot] = p; DSrow[slot] = ds; }
+        const float psd = s.scale * p * (s1r - s0r);
+        if (c == 0) { tsm[qloc][k][0] = psd * dp + p * (dp1 - dp0); tsm[qloc][k][1] = psd; }
+        if (qvalid && c == 0) { Prow[slot] = p; DProw[slot] = ok ? dp : 0.f; }
     }
     if (qvalid) {
+        float dq[16];
+#pragma unroll
+        for (int e = 0; e < 16; ++e) dq[e] = s.scale * (A[e] - delta * Bv[e]);
         rope_chunk(a.rope, ii, c, dq, true);
         T* dQ = reinterpret_cast<T*>(a.dq) + ((size_t)bh * s.T + i) * kHeadDim;
         store_chunk(dQ, c, dq);
+        if (c == 0) a.Delta[(size_t)bh * s.T + i] = delta;
     }
-    // per-block rung partials: sum the 8 query groups of the warp (lanes with
-    // c == 0 hold the value; other lanes hold the same copy), then the warps.
-#pragma unroll
-    for (int k = 0; k < kMaxRungs; ++k) {
-        float x = (c == 0) ? g[k] : 0.f;
-        x += __shfl_xor_sync(0xffffffffu, x, 4);
-        x += __shfl_xor_sync(0xffffffffu, x, 8);
-        x += __shfl_xor_sync(0xffffffffu, x, 16);
-        if (lane == 0) red[warp][k] = x;
-    }
+    if (c == 0) dsm[qloc] = qvalid ? delta : 0.f;
     __syncthreads();
+    // per-block rung partials sum_i (t1 - Delta_i t2), queries in a fixed order
     if (threadIdx.x < kMaxRungs) {
+        const int k = threadIdx.x;
         float x = 0.f;
-        for (int w = 0; w < kThreads / 32; ++w) x += red[w][threadIdx.x];
-        a.partial[(size_t)blockIdx.x * kMaxRungs + threadIdx.x] = x;
+        for (int u = 0; u < kRowsPerBlock; ++u) {
+            const bool valid = (blockIdx.x % tiles) * kRowsPerBlock + u < s.T;
+            if (valid) x += tsm[u][k][0] - dsm[u] * tsm[u][k][1];
+        }
+        a.partial[(size_t)blockIdx.x * kMaxRungs + k] = x;
     }
     if (blockIdx.x == 0 && threadIdx.x == 0) *a.ticket = 0u;
 }
@@ -318,7 +292,8 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
 // Key-centric pass.  Key row j of kv head hk receives, from every query head
 // of its group, the slots that read it: window slot t of query j+t (weight 1),
 // rung k of query j+s0_k (floor row, weight 1-w_k) and of query j+s0_k+1 (far
-// row, weight w_k):  dk~_j = scale sum c dS q~_i,  dv_j = sum c P dO_i.
+// row, weight w_k):  dk~_j = scale sum c dS q~_i,  dv_j = sum c P dO_i, with
+// dS = P (dp - Delta_i) from the query pass.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
     const Shape s = a.s;
@@ -340,13 +315,14 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
         const R* Qt = reinterpret_cast<const R*>(a.qt) + ((size_t)bh * s.T) * kHeadDim;
         const T* dO = reinterpret_cast<const T*>(a.dout) + ((size_t)bh * s.T) * kHeadDim;
         const float* P = a.P + (size_t)bh * s.T * a.S;
-        const float* DS = a.DS + (size_t)bh * s.T * a.S;
+        const float* DP = a.DP + (size_t)bh * s.T * a.S;
+        const float* Dl = a.Delta + (size_t)bh * s.T;
         for (int t = 0; t <= s.W; ++t) {
             const int i = jj + t;
             const bool ok = i < s.T;
             const int ic = ok ? i : jj;
-            const float ds = ok ? DS[(size_t)ic * a.S + t] * s.scale : 0.f;
             const float p = ok ? P[(size_t)ic * a.S + t] : 0.f;
+            const float ds = ok ? p * (DP[(size_t)ic * a.S + t] - Dl[ic]) * s.scale : 0.f;
             load_chunk(Qt + (size_t)ic * kHeadDim, c, x);
 #pragma unroll
             for (int e = 0; e < 16; ++e) dk[e] = fmaf(ds, x[e], dk[e]);
@@ -366,8 +342,9 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
                 const long long il = (long long)jj + a.r.s0[k] + side;
                 const bool ok = il < s.T;
                 const int ic = ok ? (int)il : jj;
-                const float ds = ok ? DS[(size_t)ic * a.S + slot] * s.scale * cw : 0.f;
-                const float p = ok ? P[(size_t)ic * a.S + slot] * cw : 0.f;
+                const float pr = ok ? P[(size_t)ic * a.S + slot] : 0.f;
+                const float ds = ok ? pr * (DP[(size_t)ic * a.S + slot] - Dl[ic]) * s.scale * cw : 0.f;
+                const float p = pr * cw;
                 if (__all_sync(0xffffffffu, !ok)) continue;
                 load_chunk(Qt + (size_t)ic * kHeadDim, c, x);
 #pragma unroll

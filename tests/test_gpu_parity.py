@@ -3,8 +3,8 @@ the same seeded inputs, element by element.
 
 Tolerances: fp32 I/O max abs error <= 1e-4 on out/lse and <= 1e-4 relative
 to the largest reference magnitude on gradients; bf16 I/O (fp32 accumulate)
-max abs error <= 1e-2 on out and <= 3e-2 relative (max |g - ref| / max |ref|)
-on gradients; dtheta |d - ref| / |ref|.
+max abs error <= 1e-2 on out and <= 3e-2 relative (max |g - ref| / max |ref|,
+denominator floored at 1e-3) on gradients; dtheta |d - ref| / |ref|.
 """
 from __future__ import annotations
 
@@ -40,15 +40,17 @@ def bf16_out_tol(ref):
 
 
 def _rel(a, ref):
-    return float(np.max(np.abs(a - ref)) / max(np.max(np.abs(ref)), 1e-30))
+    """max |a - ref| / max |ref|, the denominator floored at 1e-3: some exact
+    gradients are identically zero (e.g. dq with a single attended slot)."""
+    return float(np.max(np.abs(a - ref)) / max(np.max(np.abs(ref)), 1e-3))
 
 
 def _offsets(kind, K):
     return fa.base(kind, K)
 
 
-def gpu_fwd(q, k, v, alpha, f, W, dedup=True):
-    out, lse = fa.fwd(q.cuda(), k.cuda(), v.cuda(), alpha, f, W, dedup=dedup)
+def gpu_fwd(q, k, v, alpha, f, W, dedup=True, kernel="auto"):
+    out, lse = fa.fwd(q.cuda(), k.cuda(), v.cuda(), alpha, f, W, dedup=dedup, kernel=kernel)
     torch.cuda.synchronize()
     return out, lse
 
@@ -58,8 +60,8 @@ def oracle_fwd(q, k, v, alpha, f, W, dedup=True):
     return O.forward(_f64(q), _f64(k), _f64(v), W, d, dedup=dedup, nthreads=NTHREADS)
 
 
-def check_fwd(q, k, v, alpha, f, W, dedup=True):
-    out, lse = gpu_fwd(q, k, v, alpha, f, W, dedup)
+def check_fwd(q, k, v, alpha, f, W, dedup=True, kernel="auto"):
+    out, lse = gpu_fwd(q, k, v, alpha, f, W, dedup, kernel)
     ro, rl = oracle_fwd(q, k, v, alpha, f, W, dedup)
     tol = TOL[q.dtype]
     diff = np.abs(_f64(out) - ro)
@@ -114,13 +116,22 @@ SMALL = [
 ]
 
 
-@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+FWD_KERNELS = [(torch.float32, "auto"), (torch.bfloat16, "gather"), (torch.bfloat16, "staged"),
+               (torch.bfloat16, "mma")]
+
+
+@pytest.mark.parametrize("dtype,kernel", FWD_KERNELS, ids=["f32", "bf16-gather", "bf16-staged", "bf16-mma"])
 @pytest.mark.parametrize("case", SMALL, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]}{c[6]}{c[7]}d{int(c[8])}"
                                               for c in SMALL])
-def test_forward_small(case, dtype):
+def test_forward_small(case, dtype, kernel):
     Bn, H, Hkv, T, W, alpha, base, K, dedup = case
     q, k, v = inputs.qkv(Bn, H, T, seed=T + W, dtype=dtype, Hkv=Hkv)
-    check_fwd(q, k, v, alpha, _offsets(base, K), W, dedup)
+    try:
+        check_fwd(q, k, v, alpha, _offsets(base, K), W, dedup, kernel)
+    except fa.FibattnError as e:
+        if e.status == 2:                        # kernel does not apply to this shape
+            pytest.skip(str(e))
+        raise
 
 
 @pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
@@ -172,6 +183,8 @@ def test_config2_bf16_linear_stagger(W):
     for layer in (0, 7, 15):
         q, k, v = inputs.qkv(16, 8, 1024, seed=inputs.layer_seed(1, layer), dtype=torch.bfloat16)
         check_fwd(q, k, v, float(alphas[layer]), f, W)
+        if layer == 7:
+            check_fwd(q, k, v, float(alphas[layer]), f, W, kernel="staged")
 
 
 def test_config3_bf16_extrapolation_coprime():
