@@ -150,6 +150,8 @@ int fibattn_fwd_noalloc(const void* q, const void* k, const void* v, void* out, 
  * Opt-in kernel timing (no counterpart in the paper; used to attribute time
  * to kernels).  fibattn_profile_enable(1) clears the record and brackets every
  * later launch with CUDA events on the launch stream; (0) stops and clears.
+ * Launches made while the stream is being captured into a CUDA graph record
+ * external event nodes, so the summary then reports the graph's last replay.
  * fibattn_profile_summary(-1, ...) returns the number of distinct kernels
  * recorded; with index i >= 0 it synchronises on those events and writes the
  * kernel name, its summed device time in ms and its launch count.

@@ -160,17 +160,26 @@ cudaEvent_t prof_event() {
 namespace fibattn {
 int set_error(int code, const char* msg) { return fail(code, "%s", msg); }
 
+// During stream capture the records become external event nodes of the
+// graph, so every replay of the graph re-times the kernel.
+static cudaError_t prof_record(cudaEvent_t e, cudaStream_t st) {
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(st, &cs) == cudaSuccess && cs == cudaStreamCaptureStatusActive)
+        return cudaEventRecordWithFlags(e, st, cudaEventRecordExternal);
+    return cudaEventRecord(e, st);
+}
+
 ProfScope::ProfScope(const char* name, cudaStream_t st) : name_(name), st_(st), start_(nullptr), on_(false) {
     std::lock_guard<std::mutex> g(g_prof_mu);
     if (!g_prof_on) return;
     start_ = prof_event();
-    if (start_ && cudaEventRecord(start_, st_) == cudaSuccess) on_ = true;
+    if (start_ && prof_record(start_, st_) == cudaSuccess) on_ = true;
 }
 ProfScope::~ProfScope() {
     if (!on_) return;
     std::lock_guard<std::mutex> g(g_prof_mu);
     cudaEvent_t b = prof_event();
-    if (b && cudaEventRecord(b, st_) == cudaSuccess) g_prof_recs.push_back({name_, start_, b});
+    if (b && prof_record(b, st_) == cudaSuccess) g_prof_recs.push_back({name_, start_, b});
 }
 }  // namespace fibattn
 

@@ -68,7 +68,7 @@ struct BwdArgs {
     float* P;                 // softmax probabilities [B,H,T,S]
     float* DP;                // dL/dp = dO . val per slot [B,H,T,S]
     float* Delta;             // sum_slots p dL/dp per query [B,H,T]
-    float* partial;           // per-block dL/dd_k partial sums [nblocks][kMaxRungs]
+    float* partial;           // per-block dL/dd_k partial sums [kMaxRungs][nblocks]
     double* colsum;           // dL/dd_k column sums [kMaxRungs]
     unsigned* ticket;         // finalize completion counter (reset by the query pass)
     int nblocks_a;            // number of query-centric blocks (rows of partial)

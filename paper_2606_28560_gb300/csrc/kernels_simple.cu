@@ -41,16 +41,28 @@ __device__ __forceinline__ float dot16(const float* a, const float* b) {
 template <typename T, typename R>
 __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ src, R* __restrict__ dst,
                                                         long long rows, int T_, RopeParams rp) {
-    long long n = rows * 4;
-    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
-         g += (long long)gridDim.x * blockDim.x) {
-        long long row = g >> 2;
-        int c = (int)(g & 3);
-        int pos = (int)(row % T_);
-        float x[16];
-        load_chunk(src + row * kHeadDim, c, x);
-        rope_chunk(rp, pos, c, x, false);
-        store_chunk(dst + row * kHeadDim, c, x);
+    // Each thread rotates two (row, 8-pair chunk) items; both loads are issued
+    // before any arithmetic.
+    constexpr int kItems = 2;
+    const long long n = rows * 4;
+    const long long stride = (long long)gridDim.x * blockDim.x;
+    for (long long g0 = blockIdx.x * (long long)blockDim.x + threadIdx.x; g0 < n; g0 += stride * kItems) {
+        float x[kItems][16];
+#pragma unroll
+        for (int it = 0; it < kItems; ++it) {
+            const long long g = g0 + it * stride;
+            if (g < n) load_chunk(src + (g >> 2) * kHeadDim, (int)(g & 3), x[it]);
+        }
+#pragma unroll
+        for (int it = 0; it < kItems; ++it) {
+            const long long g = g0 + it * stride;
+            if (g < n) {
+                const long long row = g >> 2;
+                const int c = (int)(g & 3);
+                rope_chunk(rp, (int)(row % T_), c, x[it], false);
+                store_chunk(dst + row * kHeadDim, c, x[it]);
+            }
+        }
     }
 }
 
@@ -284,7 +296,7 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
             const bool valid = (blockIdx.x % tiles) * kRowsPerBlock + u < s.T;
             if (valid) x += tsm[u][k][0] - dsm[u] * tsm[u][k][1];
         }
-        a.partial[(size_t)blockIdx.x * kMaxRungs + k] = x;
+        a.partial[(size_t)k * a.nblocks_a + blockIdx.x] = x;
     }
     if (blockIdx.x == 0 && threadIdx.x == 0) *a.ticket = 0u;
 }
@@ -377,7 +389,8 @@ __global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
     const int t = threadIdx.x, k = blockIdx.x;
     double x = 0.0;
 #pragma unroll 8
-    for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) x += (double)a.partial[(size_t)blk * kMaxRungs + k];
+    const float* col = a.partial + (size_t)k * a.nblocks_a;
+    for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) x += (double)col[blk];
     red[t] = x;
     __syncthreads();
     for (int w = kFinThreads / 2; w > 0; w >>= 1) {
@@ -391,13 +404,18 @@ __global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
         last = atomicAdd(a.ticket, 1u) == (unsigned)(gridDim.x - 1);
     }
     __syncthreads();
-    if (last && t == 0) {
+    if (last) {                                  // block-uniform
         __threadfence();
-        double da = 0.0;
-        for (int u = 0; u < a.r.K; ++u) da += (double)a.r.f[u] * ((volatile double*)a.colsum)[u];
-        const double al = (double)a.alpha;
-        *a.dtheta = (float)(da * (al - 0.5) * (1.5 - al));
-        *a.ticket = 0u;
+        // every column sum is now visible; load them in parallel, sum in order
+        if (t < a.r.K) red[t] = (double)a.r.f[t] * __ldcg(a.colsum + t);
+        __syncthreads();
+        if (t == 0) {
+            double da = 0.0;
+            for (int u = 0; u < a.r.K; ++u) da += red[u];
+            const double al = (double)a.alpha;
+            *a.dtheta = (float)(da * (al - 0.5) * (1.5 - al));
+            *a.ticket = 0u;
+        }
     }
 }
 
@@ -406,14 +424,14 @@ __global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
                              bool bf16, cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
-    long long threads = rows * 4;
-    int grid = (int)((threads + 255) / 256);
-    if (grid > 152 * 16) grid = 152 * 16;
+    const long long items = rows * 4;
+    long long grid = (items + 256 * 2 - 1) / (256 * 2);
+    if (grid < 1) grid = 1;
     if (bf16)
-        rope_rows_kernel<__nv_bfloat16, __half><<<grid, 256, 0, st>>>(
+        rope_rows_kernel<__nv_bfloat16, __half><<<(unsigned)grid, 256, 0, st>>>(
             reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp);
     else
-        rope_rows_kernel<float, float><<<grid, 256, 0, st>>>(reinterpret_cast<const float*>(src),
+        rope_rows_kernel<float, float><<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const float*>(src),
                                                               reinterpret_cast<float*>(dst), rows, T, rp);
     return cudaGetLastError();
 }
