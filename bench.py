@@ -42,6 +42,24 @@ ESIZE = 2                     # bf16
 ROW_BYTES = D * ESIZE
 
 
+def max_over_ranks(x: float, device=None) -> float:
+    """Slowest rank's time: all-reduce MAX over the process group (NCCL on
+    GPUs, gloo on CPU); the identity when not distributed."""
+    dist = torch.distributed
+    if not (dist.is_available() and dist.is_initialized()) or dist.get_world_size() == 1:
+        return float(x)
+    on_gpu = dist.get_backend() == "nccl"
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device if on_gpu else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, steps: int, ms_max: float) -> float:
+    """Whole-job query-heads per second: every rank processes its own copy of
+    the per-rank workload (weak scaling), timed by the slowest rank."""
+    return world * steps * L * B * H * T / (ms_max / 1e3)
+
+
 def workload_config():
     return {"workload": "fwd+bwd, 16 layers, learned alpha (theta_l ~ N(0,0.5)), Fibonacci K=15",
             "B": B, "H": H, "Hkv": H, "T": T, "D": D, "W": W, "layers": L, "K": K, "seed": SEED,
@@ -244,12 +262,8 @@ def run_gpu(args, rank, world, device):
     clk = clocks.stop() if rank == 0 else None
     launches_per_step = sum(v[1] for v in prof.values())
 
-    t = torch.tensor([ms], dtype=torch.float64, device=device)
-    if dist:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-    ms_max = float(t.item())
-    queries = world * args.steps * L * B * H * T
-    value = queries / (ms_max / 1e3)
+    ms_max = max_over_ranks(ms, device)
+    value = job_throughput(world, args.steps, ms_max)
 
     # roofline of the dominant kernel (largest share of device time)
     hbm, peak_kind = peaks()
@@ -333,12 +347,9 @@ def run_e2e(args, wl, device, dist):
         one()
     e1.record(stream)
     torch.cuda.synchronize(device)
-    ms = e0.elapsed_time(e1)
-    t = torch.tensor([ms], dtype=torch.float64, device=device)
-    if dist:
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    ms = max_over_ranks(e0.elapsed_time(e1), device)
     world = torch.distributed.get_world_size() if dist else 1
-    value = world * steps * L * B * H * T / (float(t.item()) / 1e3)
+    value = job_throughput(world, steps, ms)
     bi = n_in * B * H * T * ROW_BYTES
     bo = 4 * L * B * H * T * ROW_BYTES + L * 4 * 4
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo}

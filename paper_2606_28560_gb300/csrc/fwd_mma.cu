@@ -26,6 +26,8 @@
 // rows (bf16, same buffer) is copied by TMA (3-D tensor maps [heads][T][64],
 // 8-row boxes, 128-byte swizzle, rows outside [0, T) zero-filled) under an
 // mbarrier with a bounded wait.
+#include <cmath>
+
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -123,6 +125,23 @@ __device__ __forceinline__ unsigned row_chunk(unsigned base, int row, int ch) {
     return base + (unsigned)row * 128u + (unsigned)((ch ^ (row & 7)) << 4);
 }
 
+// Warp 0 issues the copies of one staged tensor: box b fills shared rows
+// [8b, 8b+8) from the interval that contains them.  Lane 0 announces the byte
+// count first; the boxes are then spread over the 32 lanes.
+__device__ __forceinline__ void issue_rows(unsigned char* dst, const CUtensorMap* map, const MmaLayout& L,
+                                           int i0, int head, unsigned long long* bar, int lane) {
+    if (lane == 0) mbar_expect_tx(bar, (unsigned)L.rows * 128u);
+    __syncwarp();
+    const int nbox = L.rows >> 3;
+    for (int bx = lane; bx < nbox; bx += 32) {
+        const int srow = bx * 8;
+        int iv = 0;
+        while (iv + 1 < L.n_iv && srow >= L.iv_smem[iv + 1]) ++iv;
+        const int rel = L.iv_start[iv] + (srow - L.iv_smem[iv]);
+        tma_load_3d(dst + (size_t)srow * 128, map, 0, i0 + rel, head, bar);
+    }
+}
+
 template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
@@ -144,15 +163,15 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
     const int wrel = warp * kRowsPerWarp;         // tile-relative first row of this warp
     const int bw = i0 + wrel;                     // absolute first row
 
-    // ---- issue the key copies (one elected thread)
+    // ---- issue the key copies (warp 0)
     if (tid == 0) {
         mbar_init(&bars[0], 1);
         mbar_init(&bars[1], 1);
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
-        mbar_expect_tx(&bars[0], (unsigned)L.rows * 128u);
-        for (int iv = 0; iv < L.n_iv; ++iv)
-            for (int r = 0; r < L.iv_len[iv]; r += 8)
-                tma_load_3d(buf + (size_t)(L.iv_smem[iv] + r) * 128, &tmK, 0, i0 + L.iv_start[iv] + r, head, &bars[0]);
+    }
+    if (warp == 0) {
+        __syncwarp();
+        issue_rows(buf, &tmK, L, i0, head, &bars[0], lane);
     }
 
     // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32)
@@ -160,9 +179,20 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
     unsigned qa[4][4];
     {
         const __nv_bfloat16* Q = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)bh * s.T) * kHeadDim;
+        // cos/sin of the 8 pairs at position bw+g4, then advanced by 8 positions
+        // for row g4+8 with the host's fp64 cos/sin(8 theta_m)
+        float cs[2][4], sn[2][4];
+        const int pos0 = bw + g4;
+#pragma unroll
+        for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
+                rope_cs(a.rope, m, pos0, cs[kc][j], sn[kc][j]);
+            }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-            const int pos = min(bw + g4 + 8 * half, s.T - 1);
+            const int pos = min(pos0 + 8 * half, s.T - 1);
             const __nv_bfloat16* row = Q + (size_t)pos * kHeadDim;
             float x[4][4];                        // [kc][j]: dims 16kc + {2c4, 2c4+1, 2c4+8, 2c4+9}
 #pragma unroll
@@ -172,16 +202,25 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
                 x[kc][0] = __uint_as_float(u0 << 16); x[kc][1] = __uint_as_float(u0 & 0xffff0000u);
                 x[kc][2] = __uint_as_float(u1 << 16); x[kc][3] = __uint_as_float(u1 & 0xffff0000u);
             }
+            if (half == 1) {
+#pragma unroll
+                for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
+                        const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                        const float cn = cs[kc][j] * c8 - sn[kc][j] * s8;
+                        sn[kc][j] = sn[kc][j] * c8 + cs[kc][j] * s8;
+                        cs[kc][j] = cn;
+                    }
+            }
 #pragma unroll
             for (int kc = 0; kc < 2; ++kc) {      // pair (dim m in kc, dim m+32 in kc+2)
 #pragma unroll
                 for (int j = 0; j < 4; ++j) {
-                    const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
-                    float cs, sn;
-                    rope_cs(a.rope, m, pos, cs, sn);
                     const float xa = x[kc][j], xb = x[kc + 2][j];
-                    x[kc][j] = xa * cs - xb * sn;
-                    x[kc + 2][j] = xb * cs + xa * sn;
+                    x[kc][j] = xa * cs[kc][j] - xb * sn[kc][j];
+                    x[kc + 2][j] = xb * cs[kc][j] + xa * sn[kc][j];
                 }
             }
 #pragma unroll
@@ -282,12 +321,7 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
     // ---- all warps are done with the keys: stage the values into the same buffer
     asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
     __syncthreads();
-    if (tid == 0) {
-        mbar_expect_tx(&bars[1], (unsigned)L.rows * 128u);
-        for (int iv = 0; iv < L.n_iv; ++iv)
-            for (int r = 0; r < L.iv_len[iv]; r += 8)
-                tma_load_3d(buf + (size_t)(L.iv_smem[iv] + r) * 128, &tmV, 0, i0 + L.iv_start[iv] + r, head, &bars[1]);
-    }
+    if (warp == 0) issue_rows(buf, &tmV, L, i0, head, &bars[1], lane);
 
     // ---- probabilities (unnormalised, row max -> exactly 1) while values arrive
     if (mlo == -INFINITY) mlo = 0.f;              // rows beyond T: keep arithmetic finite
@@ -445,7 +479,7 @@ cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const FwdArg
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.rows * 128 + 1024; }
 
-bool build_mma_layout(const Shape& s, const RungParams& r, size_t smem_limit, MmaLayout* L) {
+bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L) {
     if (s.W > 16 || r.K > kMmaMaxRungs) return false;
     const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
     const int Wp = NT * 8 - 16;
@@ -480,6 +514,11 @@ bool build_mma_layout(const Shape& s, const RungParams& r, size_t smem_limit, Mm
         return -1;
     };
     L->win_smem = smem_row(0);
+    for (int m = 0; m < kHalf; ++m) {
+        const double theta = std::pow(rope_base, -2.0 * m / (double)kHeadDim);
+        L->rope_c8[m] = (float)std::cos(8.0 * theta);
+        L->rope_s8[m] = (float)std::sin(8.0 * theta);
+    }
     for (int k = 0; k < kMmaMaxRungs; ++k) L->rung_smem[k] = 0;
     for (int k = 0; k < r.K; ++k)
         if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row(-r.s0[k] - 1);

@@ -20,9 +20,11 @@ struct MmaLayout {
     int iv_len[kMmaMaxRungs + 1];
     int iv_smem[kMmaMaxRungs + 1];
     int rung_smem[kMmaMaxRungs];                  // shared row of relative row -s0_k - 1
+    float rope_c8[kHalf];                         // cos, sin of 8 position steps of pair m
+    float rope_s8[kHalf];
 };
 
-bool build_mma_layout(const Shape& s, const RungParams& r, size_t smem_limit, MmaLayout* L);
+bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
 size_t fwd_mma_smem_bytes(const MmaLayout& L);
 cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st);
 

@@ -377,29 +377,40 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
 
 // Fixed-order sum of the per-block rung partials, then the chain rule
 // dL/dalpha = sum_k f_k dL/dd_k and dL/dtheta = dL/dalpha (alpha-0.5)(1.5-alpha).
-// Block k sums column k: thread t adds rows t, t+256, ... in order, then a
-// fixed shared-memory tree combines the 256 sums (fp64), so the result does
-// not depend on scheduling.  The last block to finish (ticket counter, no
-// waiting) forms dL/dalpha and dL/dtheta from the K column sums and resets the
-// ticket for the next call.
+// Block k sums column k: thread t adds rows t, t+256, ... in order with
+// compensated (Kahan) fp32 sums, then a fixed shared-memory tree combines the
+// 256 (sum, compensation) pairs, so the result does not depend on scheduling.
+// (fp64 arithmetic is avoided: it runs on a slow pipe on this part.)  The last
+// block to finish (ticket counter, no waiting) forms dL/dalpha and dL/dtheta
+// from the K column sums and resets the ticket for the next call.
 constexpr int kFinThreads = 256;
 __global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
-    __shared__ double red[kFinThreads];
+    __shared__ float red[kFinThreads], cmp[kFinThreads];
     __shared__ bool last;
     const int t = threadIdx.x, k = blockIdx.x;
-    double x = 0.0;
-#pragma unroll 8
     const float* col = a.partial + (size_t)k * a.nblocks_a;
-    for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) x += (double)col[blk];
-    red[t] = x;
+    float sum = 0.f, c = 0.f;
+    for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) {
+        const float y = col[blk] - c;
+        const float tt = sum + y;
+        c = (tt - sum) - y;
+        sum = tt;
+    }
+    red[t] = sum;
+    cmp[t] = c;
     __syncthreads();
     for (int w = kFinThreads / 2; w > 0; w >>= 1) {
-        if (t < w) red[t] += red[t + w];
+        if (t < w) {
+            const float y = red[t + w] - (cmp[t] + cmp[t + w]);
+            const float tt = red[t] + y;
+            cmp[t] = (tt - red[t]) - y;
+            red[t] = tt;
+        }
         __syncthreads();
     }
     if (t == 0) {
-        a.colsum[k] = red[0];
-        if (a.dd) a.dd[k] = (float)red[0];
+        a.colsum[k] = (double)red[0];
+        if (a.dd) a.dd[k] = red[0];
         __threadfence();
         last = atomicAdd(a.ticket, 1u) == (unsigned)(gridDim.x - 1);
     }
@@ -407,13 +418,12 @@ __global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
     if (last) {                                  // block-uniform
         __threadfence();
         // every column sum is now visible; load them in parallel, sum in order
-        if (t < a.r.K) red[t] = (double)a.r.f[t] * __ldcg(a.colsum + t);
+        if (t < a.r.K) red[t] = a.r.f[t] * (float)__ldcg(a.colsum + t);
         __syncthreads();
         if (t == 0) {
-            double da = 0.0;
+            float da = 0.f;
             for (int u = 0; u < a.r.K; ++u) da += red[u];
-            const double al = (double)a.alpha;
-            *a.dtheta = (float)(da * (al - 0.5) * (1.5 - al));
+            *a.dtheta = da * (a.alpha - 0.5f) * (1.5f - a.alpha);
             *a.ticket = 0u;
         }
     }
