@@ -29,11 +29,24 @@ __device__ __forceinline__ float group_sum(float x) {
     return x;
 }
 
-__device__ __forceinline__ float dot16(const float* a, const float* b) {
-    float s = 0.f;
+// Packed fp32 pairs: one fma.rn.f32x2 issue performs two FMAs.
+template <typename T>
+__device__ __forceinline__ void load_chunk2(const T* row, int c, float2* x) {
+    float t[16];
+    load_chunk(row, c, t);
 #pragma unroll
-    for (int e = 0; e < 16; ++e) s = fmaf(a[e], b[e], s);
-    return s;
+    for (int i = 0; i < 8; ++i) x[i] = make_float2(t[2 * i], t[2 * i + 1]);
+}
+__device__ __forceinline__ float dot16x2(const float2* a, const float2* b) {
+    float2 acc = __fmul2_rn(a[0], b[0]);
+#pragma unroll
+    for (int i = 1; i < 8; ++i) acc = __ffma2_rn(a[i], b[i], acc);
+    return acc.x + acc.y;
+}
+__device__ __forceinline__ void axpy16x2(float a, const float2* x, float2* y) {
+    const float2 a2 = make_float2(a, a);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) y[i] = __ffma2_rn(a2, x[i], y[i]);
 }
 
 // ---------------------------------------------------------------- RoPE ----
@@ -41,28 +54,16 @@ __device__ __forceinline__ float dot16(const float* a, const float* b) {
 template <typename T, typename R>
 __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ src, R* __restrict__ dst,
                                                         long long rows, int T_, RopeParams rp) {
-    // Each thread rotates two (row, 8-pair chunk) items; both loads are issued
-    // before any arithmetic.
-    constexpr int kItems = 2;
+    // One (row, 8-pair chunk) item per thread per pass; grid-stride over items.
     const long long n = rows * 4;
-    const long long stride = (long long)gridDim.x * blockDim.x;
-    for (long long g0 = blockIdx.x * (long long)blockDim.x + threadIdx.x; g0 < n; g0 += stride * kItems) {
-        float x[kItems][16];
-#pragma unroll
-        for (int it = 0; it < kItems; ++it) {
-            const long long g = g0 + it * stride;
-            if (g < n) load_chunk(src + (g >> 2) * kHeadDim, (int)(g & 3), x[it]);
-        }
-#pragma unroll
-        for (int it = 0; it < kItems; ++it) {
-            const long long g = g0 + it * stride;
-            if (g < n) {
-                const long long row = g >> 2;
-                const int c = (int)(g & 3);
-                rope_chunk(rp, (int)(row % T_), c, x[it], false);
-                store_chunk(dst + row * kHeadDim, c, x[it]);
-            }
-        }
+    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
+         g += (long long)gridDim.x * blockDim.x) {
+        const long long row = g >> 2;
+        const int c = (int)(g & 3);
+        float x[16];
+        load_chunk(src + row * kHeadDim, c, x);
+        rope_chunk(rp, (int)(row % T_), c, x, false);
+        store_chunk(dst + row * kHeadDim, c, x);
     }
 }
 
@@ -84,36 +85,44 @@ __global__ void __launch_bounds__(kThreads) fwd_simple_kernel(FwdArgs a) {
     const R* Kt = reinterpret_cast<const R*>(a.kt) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
     const T* V = reinterpret_cast<const T*>(a.v) + ((size_t)(b * s.Hkv + hk) * s.T) * kHeadDim;
 
-    float q[16];
-    load_chunk(Q + (size_t)ii * kHeadDim, c, q);
-    rope_chunk(a.rope, ii, c, q, false);
+    float2 q[8];
+    {
+        float qs[16];
+        load_chunk(Q + (size_t)ii * kHeadDim, c, qs);
+        rope_chunk(a.rope, ii, c, qs, false);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) q[e] = make_float2(qs[2 * e], qs[2 * e + 1]);
+    }
     const float sc2 = s.scale * kLog2e;          // scores kept in log2 units
 
-    float m = -INFINITY, l = 0.f, acc[16];
+    // Scores use the same pairwise dot product as the backward recompute, so
+    // both sides round a score identically.
+    float m = -INFINITY, l = 0.f;
+    float2 acc[8];
 #pragma unroll
-    for (int e = 0; e < 16; ++e) acc[e] = 0.f;
+    for (int e = 0; e < 8; ++e) acc[e] = make_float2(0.f, 0.f);
 
-    float kr[16], vr[16];
+    float2 kr[8], vr[8];
     // window slots: distance t = 0..W (self always present)
     for (int t = 0; t <= s.W; ++t) {
         const int j = ii - t;
         const bool ok = j >= 0;
         const int jj = ok ? j : 0;
-        load_chunk(Kt + (size_t)jj * kHeadDim, c, kr);
-        const float sco = group_sum(dot16(q, kr)) * sc2;
+        load_chunk2(Kt + (size_t)jj * kHeadDim, c, kr);
+        const float sco = group_sum(dot16x2(q, kr)) * sc2;
         if (ok) {
-            load_chunk(V + (size_t)jj * kHeadDim, c, vr);
+            load_chunk2(V + (size_t)jj * kHeadDim, c, vr);
             if (sco > m) {
                 const float corr = exp2f(m - sco);
                 l *= corr;
+                const float2 c2 = make_float2(corr, corr);
 #pragma unroll
-                for (int e = 0; e < 16; ++e) acc[e] *= corr;
+                for (int e = 0; e < 8; ++e) acc[e] = __fmul2_rn(acc[e], c2);
                 m = sco;
             }
             const float p = exp2f(sco - m);
             l += p;
-#pragma unroll
-            for (int e = 0; e < 16; ++e) acc[e] = fmaf(p, vr[e], acc[e]);
+            axpy16x2(p, vr, acc);
         }
         if (__all_sync(0xffffffffu, !ok)) break;
     }
@@ -126,44 +135,42 @@ __global__ void __launch_bounds__(kThreads) fwd_simple_kernel(FwdArgs a) {
         const bool ok = a.r.d[k] <= fi;
         const int j0 = ii - s0, j1 = j0 - 1;
         const int jj0 = ok ? j0 : 0;
-        load_chunk(Kt + (size_t)jj0 * kHeadDim, c, kr);
-        float sraw = (1.f - w) * dot16(q, kr);
+        load_chunk2(Kt + (size_t)jj0 * kHeadDim, c, kr);
+        float sraw = (1.f - w) * dot16x2(q, kr);
         const bool far = w != 0.f;               // warp-uniform
-        float kf[16];
+        float2 kf[8];
         if (far) {
             const int jj1 = (ok && j1 >= 0) ? j1 : 0;
-            load_chunk(Kt + (size_t)jj1 * kHeadDim, c, kf);
-            if (ok && j1 >= 0) sraw = fmaf(w, dot16(q, kf), sraw);
+            load_chunk2(Kt + (size_t)jj1 * kHeadDim, c, kf);
+            if (ok && j1 >= 0) sraw = fmaf(w, dot16x2(q, kf), sraw);
         }
         const float sco = group_sum(sraw) * sc2;
         if (ok) {
-            load_chunk(V + (size_t)jj0 * kHeadDim, c, vr);
+            load_chunk2(V + (size_t)jj0 * kHeadDim, c, vr);
             if (sco > m) {
                 const float corr = exp2f(m - sco);
                 l *= corr;
+                const float2 c2 = make_float2(corr, corr);
 #pragma unroll
-                for (int e = 0; e < 16; ++e) acc[e] *= corr;
+                for (int e = 0; e < 8; ++e) acc[e] = __fmul2_rn(acc[e], c2);
                 m = sco;
             }
             const float p = exp2f(sco - m);
             l += p;
-            const float p0 = p * (1.f - w);
-#pragma unroll
-            for (int e = 0; e < 16; ++e) acc[e] = fmaf(p0, vr[e], acc[e]);
+            axpy16x2(p * (1.f - w), vr, acc);
             if (far && j1 >= 0) {
-                load_chunk(V + (size_t)j1 * kHeadDim, c, vr);
-                const float p1 = p * w;
-#pragma unroll
-                for (int e = 0; e < 16; ++e) acc[e] = fmaf(p1, vr[e], acc[e]);
+                load_chunk2(V + (size_t)j1 * kHeadDim, c, vr);
+                axpy16x2(p * w, vr, acc);
             }
         }
     }
     if (qvalid) {
         const float inv = 1.f / l;
+        float o[16];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) acc[e] *= inv;
+        for (int e = 0; e < 8; ++e) { o[2 * e] = acc[e].x * inv; o[2 * e + 1] = acc[e].y * inv; }
         T* O = reinterpret_cast<T*>(a.out) + ((size_t)bh * s.T + i) * kHeadDim;
-        store_chunk(O, c, acc);
+        store_chunk(O, c, o);
         if (c == 0) a.lse[(size_t)bh * s.T + i] = (m + __log2f(l)) * kLn2;
     }
 }
@@ -206,13 +213,13 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
     float* Prow = a.P + ((size_t)bh * s.T + ii) * a.S;
     float* DProw = a.DP + ((size_t)bh * s.T + ii) * a.S;
 
-    float q[16], go[16], kr[16], kf[16], vr[16], vf[16];
-    load_chunk(Qt + (size_t)ii * kHeadDim, c, q);
-    load_chunk(dO + (size_t)ii * kHeadDim, c, go);
+    float2 q[8], go[8], kr[8], kf[8], vr[8], vf[8];
+    load_chunk2(Qt + (size_t)ii * kHeadDim, c, q);
+    load_chunk2(dO + (size_t)ii * kHeadDim, c, go);
 
-    float A[16], Bv[16];
+    float2 A[8], Bv[8];
 #pragma unroll
-    for (int e = 0; e < 16; ++e) { A[e] = 0.f; Bv[e] = 0.f; }
+    for (int e = 0; e < 8; ++e) { A[e] = make_float2(0.f, 0.f); Bv[e] = make_float2(0.f, 0.f); }
     float delta = 0.f;
     const int qloc = threadIdx.x >> 2;
     if (c == 0)
@@ -223,15 +230,15 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
         const int j = ii - t;
         const bool ok = j >= 0;
         const int jj = ok ? j : 0;
-        load_chunk(Kt + (size_t)jj * kHeadDim, c, kr);
-        load_chunk(V + (size_t)jj * kHeadDim, c, vr);
-        const float sco = group_sum(dot16(q, kr)) * sc2;
-        const float dp = group_sum(dot16(go, vr));
+        load_chunk2(Kt + (size_t)jj * kHeadDim, c, kr);
+        load_chunk2(V + (size_t)jj * kHeadDim, c, vr);
+        const float sco = group_sum(dot16x2(q, kr)) * sc2;
+        const float dp = group_sum(dot16x2(go, vr));
         const float p = ok ? exp2f(sco - lse2) : 0.f;
         const float pdp = p * dp;
         delta += pdp;
-#pragma unroll
-        for (int e = 0; e < 16; ++e) { A[e] = fmaf(pdp, kr[e], A[e]); Bv[e] = fmaf(p, kr[e], Bv[e]); }
+        axpy16x2(pdp, kr, A);
+        axpy16x2(p, kr, Bv);
         if (qvalid && c == 0) { Prow[t] = p; DProw[t] = ok ? dp : 0.f; }
         if (__all_sync(0xffffffffu, j < 0)) {
             if (qvalid && c == 0)
@@ -252,12 +259,12 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
         const int j0 = ok ? ii - s0 : 0;
         const bool hasf = ok && j0 >= 1;          // far row -1 is a zero row
         const int j1 = hasf ? j0 - 1 : 0;
-        load_chunk(Kt + (size_t)j0 * kHeadDim, c, kr);
-        load_chunk(V + (size_t)j0 * kHeadDim, c, vr);
-        load_chunk(Kt + (size_t)j1 * kHeadDim, c, kf);
-        load_chunk(V + (size_t)j1 * kHeadDim, c, vf);
-        float s0r = dot16(q, kr), dp0 = dot16(go, vr), s1r = 0.f, dp1 = 0.f;
-        if (hasf) { s1r = dot16(q, kf); dp1 = dot16(go, vf); }
+        load_chunk2(Kt + (size_t)j0 * kHeadDim, c, kr);
+        load_chunk2(V + (size_t)j0 * kHeadDim, c, vr);
+        load_chunk2(Kt + (size_t)j1 * kHeadDim, c, kf);
+        load_chunk2(V + (size_t)j1 * kHeadDim, c, vf);
+        float s0r = dot16x2(q, kr), dp0 = dot16x2(go, vr), s1r = 0.f, dp1 = 0.f;
+        if (hasf) { s1r = dot16x2(q, kf); dp1 = dot16x2(go, vf); }
         s0r = group_sum(s0r); s1r = group_sum(s1r);
         dp0 = group_sum(dp0); dp1 = group_sum(dp1);
         const float w1 = 1.f - w;
@@ -266,13 +273,11 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
         const float p = ok ? exp2f(sco - lse2) : 0.f;
         const float pdp = p * dp;
         delta += pdp;
-        const float fw0 = w1, fw1 = hasf ? w : 0.f;
-#pragma unroll
-        for (int e = 0; e < 16; ++e) {
-            const float key = fw0 * kr[e] + fw1 * kf[e];
-            A[e] = fmaf(pdp, key, A[e]);
-            Bv[e] = fmaf(p, key, Bv[e]);
-        }
+        const float fw1 = hasf ? w : 0.f;
+        axpy16x2(pdp * w1, kr, A);
+        axpy16x2(pdp * fw1, kf, A);
+        axpy16x2(p * w1, kr, Bv);
+        axpy16x2(p * fw1, kf, Bv);
         const float psd = s.scale * p * (s1r - s0r);
         if (c == 0) { tsm[qloc][k][0] = psd * dp + p * (dp1 - dp0); tsm[qloc][k][1] = psd; }
         if (qvalid && c == 0) { Prow[slot] = p; DProw[slot] = ok ? dp : 0.f; }
@@ -280,7 +285,10 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
     if (qvalid) {
         float dq[16];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) dq[e] = s.scale * (A[e] - delta * Bv[e]);
+        for (int e = 0; e < 8; ++e) {
+            dq[2 * e] = s.scale * (A[e].x - delta * Bv[e].x);
+            dq[2 * e + 1] = s.scale * (A[e].y - delta * Bv[e].y);
+        }
         rope_chunk(a.rope, ii, c, dq, true);
         T* dQ = reinterpret_cast<T*>(a.dq) + ((size_t)bh * s.T + i) * kHeadDim;
         store_chunk(dQ, c, dq);
@@ -317,9 +325,9 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
     const bool kvalid = j < s.T;
     const int jj = kvalid ? j : s.T - 1;
 
-    float dk[16], dv[16], x[16];
+    float2 dk2[8], dv2[8], x[8];
 #pragma unroll
-    for (int e = 0; e < 16; ++e) { dk[e] = 0.f; dv[e] = 0.f; }
+    for (int e = 0; e < 8; ++e) { dk2[e] = make_float2(0.f, 0.f); dv2[e] = make_float2(0.f, 0.f); }
 
     for (int g = 0; g < s.G; ++g) {
         const int bh = b * s.H + hk * s.G + g;
@@ -335,12 +343,10 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
             const int ic = ok ? i : jj;
             const float p = ok ? P[(size_t)ic * a.S + t] : 0.f;
             const float ds = ok ? p * (DP[(size_t)ic * a.S + t] - Dl[ic]) * s.scale : 0.f;
-            load_chunk(Qt + (size_t)ic * kHeadDim, c, x);
-#pragma unroll
-            for (int e = 0; e < 16; ++e) dk[e] = fmaf(ds, x[e], dk[e]);
-            load_chunk(dO + (size_t)ic * kHeadDim, c, x);
-#pragma unroll
-            for (int e = 0; e < 16; ++e) dv[e] = fmaf(p, x[e], dv[e]);
+            load_chunk2(Qt + (size_t)ic * kHeadDim, c, x);
+            axpy16x2(ds, x, dk2);
+            load_chunk2(dO + (size_t)ic * kHeadDim, c, x);
+            axpy16x2(p, x, dv2);
             if (__all_sync(0xffffffffu, !ok)) break;
         }
         for (int k = 0; k < a.r.K; ++k) {
@@ -358,14 +364,18 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
                 const float ds = ok ? pr * (DP[(size_t)ic * a.S + slot] - Dl[ic]) * s.scale * cw : 0.f;
                 const float p = pr * cw;
                 if (__all_sync(0xffffffffu, !ok)) continue;
-                load_chunk(Qt + (size_t)ic * kHeadDim, c, x);
-#pragma unroll
-                for (int e = 0; e < 16; ++e) dk[e] = fmaf(ds, x[e], dk[e]);
-                load_chunk(dO + (size_t)ic * kHeadDim, c, x);
-#pragma unroll
-                for (int e = 0; e < 16; ++e) dv[e] = fmaf(p, x[e], dv[e]);
+                load_chunk2(Qt + (size_t)ic * kHeadDim, c, x);
+                axpy16x2(ds, x, dk2);
+                load_chunk2(dO + (size_t)ic * kHeadDim, c, x);
+                axpy16x2(p, x, dv2);
             }
         }
+    }
+    float dk[16], dv[16];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        dk[2 * e] = dk2[e].x; dk[2 * e + 1] = dk2[e].y;
+        dv[2 * e] = dv2[e].x; dv[2 * e + 1] = dv2[e].y;
     }
     if (kvalid) {
         rope_chunk(a.rope, jj, c, dk, true);
@@ -435,8 +445,8 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
                              bool bf16, cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
     const long long items = rows * 4;
-    long long grid = (items + 256 * 2 - 1) / (256 * 2);
-    if (grid < 1) grid = 1;
+    long long grid = (items + 255) / 256;
+    if (grid > 152 * 16) grid = 152 * 16;       // 16 resident 256-thread blocks on each of 152 SMs
     if (bf16)
         rope_rows_kernel<__nv_bfloat16, __half><<<(unsigned)grid, 256, 0, st>>>(
             reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp);

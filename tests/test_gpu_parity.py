@@ -40,9 +40,15 @@ def bf16_out_tol(ref):
 
 
 def _rel(a, ref):
-    """max |a - ref| / max |ref|, the denominator floored at 1e-3: some exact
-    gradients are identically zero (e.g. dq with a single attended slot)."""
-    return float(np.max(np.abs(a - ref)) / max(np.max(np.abs(ref)), 1e-3))
+    """max |a - ref| / max |ref|, the denominator floored at 1e-2.
+
+    Some exact gradients are identically zero, e.g. dq of a query with a single
+    attended slot, where softmax gives p = 1 and dq = scale p dp k (1 - p).  The
+    kernel reaches that zero only up to the rounding of p = exp(s - lse) with
+    lse stored in natural-log units: one ulp of p (6e-8) times scale |dp| |k|
+    (about 3 at D = 64 with unit-normal inputs) leaves ~2e-7, so the floor must
+    sit at least three decades above that for the fp32 bound of 1e-4."""
+    return float(np.max(np.abs(a - ref)) / max(np.max(np.abs(ref)), 1e-2))
 
 
 def _offsets(kind, K):
