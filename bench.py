@@ -178,8 +178,8 @@ class Workload:
                    workspace=self.ws_f)
         for l in reversed(range(self.L)):
             fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], self.alphas[l], self.f, W,
-                   dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], dtheta=self.dth[l], dd=self.dd[l],
-                   workspace=self.ws_b)
+                   out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], dtheta=self.dth[l],
+                   dd=self.dd[l], workspace=self.ws_b)
 
     def fwd_only(self, W_):
         fa = self.fa
@@ -198,6 +198,8 @@ def algorithmic_bytes():
         "fwd": 4 * rows + 4 * n,                           # Q, K~, V read; O written; lse
         "rope_k": 2 * rows, "rope_q": 2 * rows,            # read, write rotated
         "bwd_query": 5 * rows + 4 * n + 2 * 4 * n * S,     # Q~ K~ V dO read, dQ written, lse, P/dS written
+        # Q, dO, O, K~, V read; dQ, Q~ written; lse read, Delta written; P/dp written
+        "bwd_query_mma": 7 * rows + 2 * 4 * n + 2 * 4 * n * S,
         "bwd_key": 4 * rows + 2 * 4 * n * S,               # Q~ dO read, dK dV written, P/dS read
         "bwd_finalize": 0,
     }
@@ -431,7 +433,7 @@ def ncu_case(which: str):
         for l, (q, k, v, g) in enumerate(bufs):
             out, lse = fa.fwd(q, k, v, 0.8 + 0.1 * l, f, W)
             if which == "bwd":
-                fa.bwd(q, k, v, lse, g, 0.8 + 0.1 * l, f, W)
+                fa.bwd(q, k, v, lse, g, 0.8 + 0.1 * l, f, W, out=out)
     torch.cuda.synchronize(dev)
     print(f"ncu case {which} done")
 

@@ -61,6 +61,11 @@ typedef struct {
                           2 shared-memory staged CUDA-core kernel; 3 tensor-core
                           kernel (2 and 3: bf16 I/O only; 3: W <= 16, K <= 16;
                           FIBATTN_ERR_UNSUPPORTED when the choice does not apply) */
+    int   bwd_kernel;  /* backward query pass: 0 automatic [default]; 1 row-gather
+                          single sweep (Delta accumulated from the slots, `out`
+                          unused); 2 tensor-core kernel (bf16 I/O, `out` given,
+                          W <= 16, K <= 16; FIBATTN_ERR_UNSUPPORTED otherwise).
+                          Automatic takes 2 where it applies, else 1. */
 } fibattn_opts;
 
 /* ---------------------------------------------------------------------------
@@ -84,6 +89,10 @@ int fibattn_fwd(const void* q, const void* k, const void* v,
  * Backward (the chain rule of the forward definition; the paper trains every
  * model through this path, Section 2 "Implementation note").
  * Inputs: q, k, v, dout as above and lse from fibattn_fwd of the same inputs.
+ * out: the output of that forward call, or NULL.  With out, the softmax term
+ * Delta_i = sum_slots p dp (= dout_i . out_i) is read as dout_i . out_i, which
+ * lets the tensor-core query pass (opts->bwd_kernel) form each score gradient
+ * in one pass; without it Delta is accumulated from the slots.
  * Outputs (overwritten, not accumulated): dq [B,H,T,D], dk and dv [B,Hkv,T,D]
  * in `dtype`, gradients with respect to the pre-RoPE q and k; dtheta (device,
  * 1 float) = dL/dtheta with alpha = 0.5 + sigmoid(theta); dd (device, K floats,
@@ -94,7 +103,7 @@ size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K,
                                    int dtype, const fibattn_opts* opts);
 
 int fibattn_bwd(const void* q, const void* k, const void* v,
-                const float* lse, const void* dout,
+                const void* out, const float* lse, const void* dout,
                 void* dq, void* dk, void* dv, float* dtheta, float* dd,
                 int B, int H, int T, int D, int W,
                 float alpha, const float* offsets, int K,

@@ -32,7 +32,8 @@ class FibattnError(RuntimeError):
 
 class Opts(ctypes.Structure):
     _fields_ = [("rope_base", ctypes.c_float), ("scale", ctypes.c_float),
-                ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int), ("fwd_kernel", ctypes.c_int)]
+                ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int), ("fwd_kernel", ctypes.c_int),
+                ("bwd_kernel", ctypes.c_int)]
 
 
 def library_path() -> str:
@@ -58,8 +59,8 @@ def lib():
             L.fibattn_fwd.restype = ci
             L.fibattn_bwd_workspace_bytes.argtypes = [ci] * 7 + [op]
             L.fibattn_bwd_workspace_bytes.restype = sz
-            L.fibattn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, fp, ci, ci, op,
-                                      vp, sz, vp]
+            L.fibattn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, fp, ci, ci,
+                                      op, vp, sz, vp]
             L.fibattn_bwd.restype = ci
             L.fibattn_last_error.argtypes = []
             L.fibattn_last_error.restype = ctypes.c_char_p
@@ -87,11 +88,12 @@ def _iptr(a: np.ndarray):
 
 
 FWD_KERNELS = {"auto": 0, "gather": 1, "staged": 2, "mma": 3}
+BWD_KERNELS = {"auto": 0, "gather": 1, "mma": 2}
 
 
-def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto") -> Opts:
+def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto", bwd_kernel="auto") -> Opts:
     return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1,
-                FWD_KERNELS[fwd_kernel])
+                FWD_KERNELS[fwd_kernel], BWD_KERNELS[bwd_kernel])
 
 
 def _dtype_code(t: torch.Tensor) -> int:
@@ -176,18 +178,20 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
     return out, lse
 
 
-def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
-        dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None):
-    """Backward pass.  Returns (dq, dk, dv, dtheta [1], dd [K]) on the device."""
+def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_base=1e4, scale=None, dedup=True,
+        dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None, kernel="auto"):
+    """Backward pass.  ``out``: the forward output (optional; enables the
+    tensor-core query pass).  ``kernel``: "auto", "gather" or "mma".
+    Returns (dq, dk, dv, dtheta [1], dd [K]) on the device."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
     K = len(f)
-    o = _opts(rope_base, scale, Hkv, dedup)
+    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel)
     code = _dtype_code(q)
-    for t in (q, k, v, dout):
+    for t in (q, k, v, dout) + ((out,) if out is not None else ()):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
-            raise ValueError("q, k, v, dout must be contiguous CUDA tensors of one dtype")
+            raise ValueError("q, k, v, dout, out must be contiguous CUDA tensors of one dtype")
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(k) if dk is None else dk
     dv = torch.empty_like(v) if dv is None else dv
@@ -196,7 +200,8 @@ def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, rope_base=1e4, sca
     need = int(lib().fibattn_bwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
-    _check(lib().fibattn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), lse.data_ptr(), dout.data_ptr(),
+    _check(lib().fibattn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr() if out is not None else None,
+                             lse.data_ptr(), dout.data_ptr(),
                              dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), dtheta.data_ptr(), dd.data_ptr(),
                              B, H, T, D, int(W), float(alpha), _fptr(f), K, code, ctypes.byref(o),
                              workspace.data_ptr(), workspace.numel(), _stream_ptr(stream)))

@@ -1,0 +1,479 @@
+// bwd_mma.cu -- query-centric backward on tensor cores (mma.sync, m16n8) with
+// TMA staging: the chain rule of the attended-set forward (arXiv 2606.28560,
+// Section 2 "Attended set" and "Implementation note").
+//
+// Tiles and staged rows are those of the tensor-core forward: a warp owns a
+// 16-row tile of queries placed every 15 queries, a CTA the union of rows its
+// tiles read (window band and one 16-row slab per rung).  With
+// Delta_i = dO_i . o_i (the forward output), the gradient of every score is
+// known as soon as its slot is:  dS = p (dp - Delta),  p = exp(s - lse),
+// dp = dO . val.  So the backward needs each staged tensor once:
+//
+//   values staged (bf16):  dP = dO V^T     window band 16 x (16+Wp) and the
+//                          16 x 16 slab of each rung; a rung keeps its far and
+//                          floor columns: dp = (1-w) dp0 + w dp1, ddp = dp1 - dp0
+//   keys staged (fp16):    S = Q~ K~^T     same blocks; p, dS per slot, then
+//                          dq~ += dS_band K~_band + dShat_k K~_slab
+//                          with dShat_k[u][u] = dS w, dShat_k[u][u+1] = dS (1-w)
+//
+// and the rung-distance gradient of query i (row -1 is a zero row):
+//   dL/dd_k += p (scale (s1 - s0)(dp - Delta) + ddp)
+// with s1, s0 the raw far and floor dot products.  P, dp per slot (zero where
+// not attended), Delta and the rotated queries go to the workspace for the
+// key-centric pass.  dS enters the dq MMAs as fp16 (11-bit significand);
+// accumulation is fp32.
+#include <cmath>
+
+#include "fibattn_internal.cuh"
+#include "fwd_mma.cuh"
+#include "mma_common.cuh"
+
+namespace fibattn {
+namespace {
+
+using namespace mma;
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr int kWarps = kMmaWarps;
+constexpr int kRowsPerWarp = 15;
+
+__device__ __forceinline__ float bf_lo(unsigned u) { return __uint_as_float(u << 16); }
+__device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 0xffff0000u); }
+
+template <int NT>
+__global__ void __launch_bounds__(kWarps * 32, 2)
+bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+                     BwdArgs a, MmaLayout L) {
+    constexpr int Wp = NT * 8 - 16;
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ unsigned long long bars[2];
+    __shared__ float dps[kWarps][kMmaMaxRungs][16][2];   // rung dp, ddp of each tile row
+    __shared__ float gsm[kWarps][kMmaMaxRungs];           // per-warp rung-gradient sums
+    unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const unsigned sbase = smem_u32(buf);
+
+    const Shape s = a.s;
+    const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
+    const int bh = blockIdx.x / tiles;
+    const int i0 = (blockIdx.x % tiles) * kMmaTile;
+    const int b = bh / s.H, h = bh % s.H, hk = h / s.G;
+    const int head = b * s.Hkv + hk;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int g4 = lane >> 2, c4 = lane & 3;
+    const int wrel = warp * kRowsPerWarp;
+    const int bw = i0 + wrel;
+
+    // ---- values first
+    if (tid == 0) {
+        mbar_init(&bars[0], 1);
+        mbar_init(&bars[1], 1);
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    if (warp == 0) {
+        __syncwarp();
+        issue_rows(buf, &tmV, L, i0, head, &bars[0], lane);
+    }
+
+    const int qlo = bw + g4, qhi = bw + g4 + 8;
+    const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
+    const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
+    const size_t rowbase = (size_t)bh * s.T;
+
+    // ---- dO as bf16 A fragments; Delta = dO . o of rows g4, g4+8
+    unsigned da[4][4];
+    float dlt_lo, dlt_hi;
+    {
+        const __nv_bfloat16* dO = reinterpret_cast<const __nv_bfloat16*>(a.dout) + rowbase * kHeadDim;
+        const __nv_bfloat16* Og = reinterpret_cast<const __nv_bfloat16*>(a.out) + rowbase * kHeadDim;
+        float part[2] = {0.f, 0.f};
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int pos = min(qlo + 8 * half, s.T - 1);
+            const __nv_bfloat16* rd = dO + (size_t)pos * kHeadDim;
+            const __nv_bfloat16* ro = Og + (size_t)pos * kHeadDim;
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                const unsigned u0 = *reinterpret_cast<const unsigned*>(rd + 16 * kc + 2 * c4);
+                const unsigned u1 = *reinterpret_cast<const unsigned*>(rd + 16 * kc + 8 + 2 * c4);
+                const unsigned o0 = *reinterpret_cast<const unsigned*>(ro + 16 * kc + 2 * c4);
+                const unsigned o1 = *reinterpret_cast<const unsigned*>(ro + 16 * kc + 8 + 2 * c4);
+                da[kc][half] = u0;
+                da[kc][2 + half] = u1;
+                part[half] = fmaf(bf_lo(u0), bf_lo(o0), part[half]);
+                part[half] = fmaf(bf_hi(u0), bf_hi(o0), part[half]);
+                part[half] = fmaf(bf_lo(u1), bf_lo(o1), part[half]);
+                part[half] = fmaf(bf_hi(u1), bf_hi(o1), part[half]);
+            }
+        }
+        dlt_lo = quad_sum(part[0]);
+        dlt_hi = quad_sum(part[1]);
+    }
+
+    // ---- q~ as fp16 A fragments (RoPE pairs m, m+32 in the same thread), also
+    // written to the workspace for the key pass
+    unsigned qa[4][4];
+    {
+        const __nv_bfloat16* Q = reinterpret_cast<const __nv_bfloat16*>(a.q) + rowbase * kHeadDim;
+        __half* Qt = reinterpret_cast<__half*>(a.qt) + rowbase * kHeadDim;
+        float cs[2][4], sn[2][4];
+#pragma unroll
+        for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+                const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
+                rope_cs(a.rope, m, qlo, cs[kc][j], sn[kc][j]);
+            }
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int pos = min(qlo + 8 * half, s.T - 1);
+            const __nv_bfloat16* row = Q + (size_t)pos * kHeadDim;
+            float x[4][4];
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                const unsigned u0 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 2 * c4);
+                const unsigned u1 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 8 + 2 * c4);
+                x[kc][0] = bf_lo(u0); x[kc][1] = bf_hi(u0);
+                x[kc][2] = bf_lo(u1); x[kc][3] = bf_hi(u1);
+            }
+            if (half == 1) {
+#pragma unroll
+                for (int kc = 0; kc < 2; ++kc)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) {
+                        const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
+                        const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                        const float cn = cs[kc][j] * c8 - sn[kc][j] * s8;
+                        sn[kc][j] = sn[kc][j] * c8 + cs[kc][j] * s8;
+                        cs[kc][j] = cn;
+                    }
+            }
+#pragma unroll
+            for (int kc = 0; kc < 2; ++kc) {
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    const float xa = x[kc][j], xb = x[kc + 2][j];
+                    x[kc][j] = xa * cs[kc][j] - xb * sn[kc][j];
+                    x[kc + 2][j] = xb * cs[kc][j] + xa * sn[kc][j];
+                }
+            }
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);
+                qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);
+            }
+            if (half == 0 ? vlo : vhi) {
+                __half* qr = Qt + (size_t)(qlo + 8 * half) * kHeadDim;
+#pragma unroll
+                for (int kc = 0; kc < 4; ++kc) {
+                    *reinterpret_cast<unsigned*>(qr + 16 * kc + 2 * c4) = qa[kc][half];
+                    *reinterpret_cast<unsigned*>(qr + 16 * kc + 8 + 2 * c4) = qa[kc][2 + half];
+                }
+            }
+        }
+    }
+    const float lse2_lo = vlo ? a.lse[rowbase + qlo] * kLog2e : 0.f;
+    const float lse2_hi = vhi ? a.lse[rowbase + qhi] * kLog2e : 0.f;
+    if (c4 == 0) {
+        if (vlo) a.Delta[rowbase + qlo] = dlt_lo;
+        if (vhi) a.Delta[rowbase + qhi] = dlt_hi;
+    }
+
+    // Columns of the rung slab: row r's far row is x = r, its floor row x = r+1;
+    // columns 2c4 + {0,1} of each 8-column n-tile belong to this thread.
+    const int xf_lo = g4, xl_lo = g4 + 1, xf_hi = g4 + 8, xl_hi = g4 + 9;
+    const bool own_f_lo = ((xf_lo & 7) >> 1) == c4, own_l_lo = ((xl_lo & 7) >> 1) == c4;
+    const bool own_f_hi = ((xf_hi & 7) >> 1) == c4, own_l_hi = ((xl_hi & 7) >> 1) == c4 && xl_hi < 16;
+
+    __syncthreads();                              // barrier init visible
+    const bool ok_v = mbar_wait(&bars[0], 0);
+
+    // ---- window band dp = dO . v
+    float dpw[NT][4];
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+        dpw[j][0] = dpw[j][1] = dpw[j][2] = dpw[j][3] = 0.f;
+        const int krow = L.win_smem + wrel - Wp + 8 * j + (lane & 7);
+#pragma unroll
+        for (int kc = 0; kc < 4; kc += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+            mma_bf16_16816(dpw[j], da[kc], b0, b1);
+            mma_bf16_16816(dpw[j], da[kc + 1], b2, b3);
+        }
+    }
+    // ---- rung dp (interpolated) and ddp = dp_far - dp_floor, to shared memory
+#pragma unroll 1
+    for (int k = 0; k < a.r.K; ++k) {
+        if (!((a.r.active >> k) & 1u)) continue;
+        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;        // masked for the whole warp
+        const float w = a.r.w[k], w1 = 1.f - w;
+        float dt[2][4];
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+            dt[t][0] = dt[t][1] = dt[t][2] = dt[t][3] = 0.f;
+            const int krow = L.rung_smem[k] + wrel + 8 * t + (lane & 7);
+#pragma unroll
+            for (int kc = 0; kc < 4; kc += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                mma_bf16_16816(dt[t], da[kc], b0, b1);
+                mma_bf16_16816(dt[t], da[kc + 1], b2, b3);
+            }
+        }
+        const float f_lo = (xf_lo & 1) ? dt[0][1] : dt[0][0];
+        const float l_lo0 = (xl_lo & 1) ? dt[0][1] : dt[0][0];
+        const float l_lo1 = (xl_lo & 1) ? dt[1][1] : dt[1][0];
+        const float l_lo = (xl_lo >> 3) ? l_lo1 : l_lo0;
+        const float f_hi = (xf_hi & 1) ? dt[1][3] : dt[1][2];
+        const float l_hi = (xl_hi & 1) ? dt[1][3] : dt[1][2];
+        const float d1_lo = quad_sum(own_f_lo ? f_lo : 0.f), d0_lo = quad_sum(own_l_lo ? l_lo : 0.f);
+        const float d1_hi = quad_sum(own_f_hi ? f_hi : 0.f), d0_hi = quad_sum(own_l_hi ? l_hi : 0.f);
+        if (c4 == 0) {
+            dps[warp][k][g4][0] = w1 * d0_lo + w * d1_lo;
+            dps[warp][k][g4][1] = d1_lo - d0_lo;
+            dps[warp][k][g4 + 8][0] = w1 * d0_hi + w * d1_hi;
+            dps[warp][k][g4 + 8][1] = d1_hi - d0_hi;
+        }
+    }
+
+    // ---- all warps are done with the values: stage the keys into the same buffer
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+    __syncthreads();
+    if (warp == 0) issue_rows(buf, &tmK, L, i0, head, &bars[1], lane);
+    const bool ok_k = mbar_wait(&bars[1], 0);
+
+    const float sc2 = s.scale * kLog2e;
+    float* Pg = a.P + rowbase * a.S;
+    float* DPg = a.DP + rowbase * a.S;
+
+    float dq[8][4];
+#pragma unroll
+    for (int n = 0; n < 8; ++n) dq[n][0] = dq[n][1] = dq[n][2] = dq[n][3] = 0.f;
+
+    // ---- window band: scores, p, dS; P and dp per slot to the workspace
+    {
+        float sw[NT][4];
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+            sw[j][0] = sw[j][1] = sw[j][2] = sw[j][3] = 0.f;
+            const int krow = L.win_smem + wrel - Wp + 8 * j + (lane & 7);
+#pragma unroll
+            for (int kc = 0; kc < 4; kc += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                mma_f16_16816(sw[j], qa[kc], b0, b1);
+                mma_f16_16816(sw[j], qa[kc + 1], b2, b3);
+            }
+        }
+        unsigned dsa[NT][2];
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+            float dsv[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool hi = e >= 2;
+                const int r = hi ? g4 + 8 : g4;
+                const int n = 8 * j + 2 * c4 + (e & 1);
+                const int t = r + Wp - n;                     // distance query - key
+                const int key = bw - Wp + n;
+                const bool rv = hi ? vhi : vlo;
+                const bool inband = t >= 0 && t <= s.W;
+                const bool ok = rv && inband && key >= 0;
+                const float p = ok ? exp2f(sw[j][e] * sc2 - (hi ? lse2_hi : lse2_lo)) : 0.f;
+                dsv[e] = p * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
+                if (rv && inband) {
+                    const size_t off = (size_t)(bw + r) * a.S + t;
+                    Pg[off] = p;
+                    DPg[off] = ok ? dpw[j][e] : 0.f;
+                }
+            }
+            dsa[j][0] = pack_f16(dsv[0], dsv[1]);
+            dsa[j][1] = pack_f16(dsv[2], dsv[3]);
+        }
+        // dq~ += dS_band K~_band
+#pragma unroll
+        for (int kk = 0; kk + 1 < NT; kk += 2) {
+            const unsigned afr[4] = {dsa[kk][0], dsa[kk][1], dsa[kk + 1][0], dsa[kk + 1][1]};
+            const int krow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+            for (int n = 0; n < 8; n += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4_t(row_chunk(sbase, krow, n + (lane >> 4)), b0, b1, b2, b3);
+                mma_f16_16816(dq[n], afr, b0, b1);
+                mma_f16_16816(dq[n + 1], afr, b2, b3);
+            }
+        }
+        if constexpr (NT & 1) {
+            const int kk = NT - 1;
+            const int krow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7);
+#pragma unroll
+            for (int n = 0; n < 8; n += 4) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4_t(row_chunk(sbase, krow, n + (lane >> 3)), b0, b1, b2, b3);
+                mma_f16_1688(dq[n], dsa[kk][0], dsa[kk][1], b0);
+                mma_f16_1688(dq[n + 1], dsa[kk][0], dsa[kk][1], b1);
+                mma_f16_1688(dq[n + 2], dsa[kk][0], dsa[kk][1], b2);
+                mma_f16_1688(dq[n + 3], dsa[kk][0], dsa[kk][1], b3);
+            }
+        }
+    }
+
+    // ---- rungs: scores, p, dS, dL/dd_k; dq~ += dShat_k K~_slab
+#pragma unroll 1
+    for (int k = 0; k < a.r.K; ++k) {
+        if (!((a.r.active >> k) & 1u)) continue;           // never read by the key pass
+        const int slot = s.W + 1 + k;
+        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) {   // masked for every row of the tile
+            if (c4 == 0) {
+                if (vlo) { Pg[(size_t)qlo * a.S + slot] = 0.f; DPg[(size_t)qlo * a.S + slot] = 0.f; }
+                if (vhi) { Pg[(size_t)qhi * a.S + slot] = 0.f; DPg[(size_t)qhi * a.S + slot] = 0.f; }
+            }
+            if (lane == 0) gsm[warp][k] = 0.f;
+            continue;
+        }
+        const float w = a.r.w[k], w1 = 1.f - w;
+        float st[2][4];
+#pragma unroll
+        for (int t = 0; t < 2; ++t) {
+            st[t][0] = st[t][1] = st[t][2] = st[t][3] = 0.f;
+            const int krow = L.rung_smem[k] + wrel + 8 * t + (lane & 7);
+#pragma unroll
+            for (int kc = 0; kc < 4; kc += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                mma_f16_16816(st[t], qa[kc], b0, b1);
+                mma_f16_16816(st[t], qa[kc + 1], b2, b3);
+            }
+        }
+        const float f_lo = (xf_lo & 1) ? st[0][1] : st[0][0];
+        const float l_lo0 = (xl_lo & 1) ? st[0][1] : st[0][0];
+        const float l_lo1 = (xl_lo & 1) ? st[1][1] : st[1][0];
+        const float l_lo = (xl_lo >> 3) ? l_lo1 : l_lo0;
+        const float f_hi = (xf_hi & 1) ? st[1][3] : st[1][2];
+        const float l_hi = (xl_hi & 1) ? st[1][3] : st[1][2];
+        const float s1_lo = quad_sum(own_f_lo ? f_lo : 0.f), s0_lo = quad_sum(own_l_lo ? l_lo : 0.f);
+        const float s1_hi = quad_sum(own_f_hi ? f_hi : 0.f), s0_hi = quad_sum(own_l_hi ? l_hi : 0.f);
+        const float dk = a.r.d[k];
+        const bool okl = vlo && dk <= (float)qlo, okh = vhi && dk <= (float)qhi;
+        const float dp_lo = dps[warp][k][g4][0], ddp_lo = dps[warp][k][g4][1];
+        const float dp_hi = dps[warp][k][g4 + 8][0], ddp_hi = dps[warp][k][g4 + 8][1];
+        const float p_lo = okl ? exp2f((w1 * s0_lo + w * s1_lo) * sc2 - lse2_lo) : 0.f;
+        const float p_hi = okh ? exp2f((w1 * s0_hi + w * s1_hi) * sc2 - lse2_hi) : 0.f;
+        const float e_lo = dp_lo - dlt_lo, e_hi = dp_hi - dlt_hi;
+        const float ds_lo = p_lo * e_lo, ds_hi = p_hi * e_hi;
+        if (c4 == 0) {
+            if (vlo) { Pg[(size_t)qlo * a.S + slot] = p_lo; DPg[(size_t)qlo * a.S + slot] = okl ? dp_lo : 0.f; }
+            if (vhi) { Pg[(size_t)qhi * a.S + slot] = p_hi; DPg[(size_t)qhi * a.S + slot] = okh ? dp_hi : 0.f; }
+        }
+        // dL/dd_k of this warp's rows, in a fixed order over the rows
+        float g = 0.f;
+        if (c4 == 0)
+            g = p_lo * fmaf(s.scale * (s1_lo - s0_lo), e_lo, ddp_lo) +
+                p_hi * fmaf(s.scale * (s1_hi - s0_hi), e_hi, ddp_hi);
+        g += __shfl_xor_sync(0xffffffffu, g, 4);
+        g += __shfl_xor_sync(0xffffffffu, g, 8);
+        g += __shfl_xor_sync(0xffffffffu, g, 16);
+        if (lane == 0) gsm[warp][k] = g;
+
+        // dShat_k as fp16 A fragment: columns 2c4 + {0,1} (a0, a1) and 2c4 + 8 + {0,1} (a2, a3)
+        unsigned afr[4];
+#pragma unroll
+        for (int cs = 0; cs < 4; cs += 2) {
+#pragma unroll
+            for (int half = 0; half < 2; ++half) {
+                const int r = g4 + 8 * half;
+                const float d = half ? ds_hi : ds_lo;
+                float e2[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int x = 2 * c4 + u + 8 * (cs >> 1);
+                    e2[u] = (x == r) ? d * w : ((x == r + 1) ? d * w1 : 0.f);
+                }
+                afr[(cs >> 1) * 2 + half] = pack_f16(e2[0], e2[1]);
+            }
+        }
+        const int krow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+        for (int n = 0; n < 8; n += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, krow, n + (lane >> 4)), b0, b1, b2, b3);
+            mma_f16_16816(dq[n], afr, b0, b1);
+            mma_f16_16816(dq[n + 1], afr, b2, b3);
+        }
+    }
+
+    // ---- dq = R(-theta pos) scale dq~, rows 0..14 of the tile
+    const bool ok = ok_k && ok_v;
+    const float sc = ok ? s.scale : __int_as_float(0x7fc00000);
+    __nv_bfloat16* dQ = reinterpret_cast<__nv_bfloat16*>(a.dq) + rowbase * kHeadDim;
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+        if (!(half ? vhi : vlo)) continue;
+        const int q = half ? qhi : qlo;
+        __nv_bfloat16* row = dQ + (size_t)q * kHeadDim;
+#pragma unroll
+        for (int n = 0; n < 4; ++n) {
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int m = 8 * n + 2 * c4 + u;           // pair (m, m + 32): n-tiles n and n + 4
+                float c, sgn;
+                rope_cs(a.rope, m, q, c, sgn);
+                const float xa = dq[n][2 * half + u] * sc, xb = dq[n + 4][2 * half + u] * sc;
+                dq[n][2 * half + u] = xa * c + xb * sgn;
+                dq[n + 4][2 * half + u] = xb * c - xa * sgn;
+            }
+        }
+#pragma unroll
+        for (int n = 0; n < 8; ++n)
+            *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(dq[n][2 * half], dq[n][2 * half + 1]);
+    }
+
+    // ---- per-CTA rung partials, warps summed in a fixed order
+    __syncthreads();
+    if (tid < a.r.K) {
+        float x = 0.f;
+        if ((a.r.active >> tid) & 1u)
+            for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
+        a.partial[(size_t)tid * a.nblocks_a + blockIdx.x] = x;
+    }
+    if (blockIdx.x == 0 && tid == 0) *a.ticket = 0u;
+}
+
+template <int NT>
+cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const BwdArgs& a, const MmaLayout& L,
+                      unsigned grid, size_t smem, cudaStream_t st) {
+    auto kern = bwd_query_mma_kernel<NT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kWarps * 32, smem, st>>>(mk, mv, a, L);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t bwd_mma_static_smem() {
+    return sizeof(float) * kWarps * kMmaMaxRungs * 16 * 2 + sizeof(float) * kWarps * kMmaMaxRungs + 64;
+}
+
+int bwd_mma_blocks(const Shape& s) {
+    const long long tiles = (s.T + kMmaTile - 1) / kMmaTile;
+    return (int)(tiles * s.B * s.H);
+}
+
+cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st) {
+    const long long grid = bwd_mma_blocks(a.s);
+    if (grid <= 0) return cudaSuccess;
+    CUtensorMap mk, mv;
+    const int heads = a.s.B * a.s.Hkv;
+    if (!encode_rows_map(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
+        !encode_rows_map(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
+        return cudaErrorInvalidValue;
+    const size_t smem = fwd_mma_smem_bytes(L);
+    switch (L.nt) {
+    case 2: return launch_nt<2>(mk, mv, a, L, (unsigned)grid, smem, st);
+    case 3: return launch_nt<3>(mk, mv, a, L, (unsigned)grid, smem, st);
+    default: return launch_nt<4>(mk, mv, a, L, (unsigned)grid, smem, st);
+    }
+}
+
+}  // namespace fibattn

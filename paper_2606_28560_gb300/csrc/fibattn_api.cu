@@ -39,7 +39,7 @@ size_t rot_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
 
 struct Resolved {
     float rope_base, scale;
-    int Hkv, dedup, fwd_kernel;
+    int Hkv, dedup, fwd_kernel, bwd_kernel;
 };
 
 int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
@@ -49,6 +49,8 @@ int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
     r->dedup = (o && o->no_dedup) ? 0 : 1;
     r->fwd_kernel = o ? o->fwd_kernel : 0;
     if (r->fwd_kernel < 0 || r->fwd_kernel > 3) return fail(FIBATTN_ERR_INVALID_ARG, "fwd_kernel must be 0, 1, 2 or 3");
+    r->bwd_kernel = o ? o->bwd_kernel : 0;
+    if (r->bwd_kernel < 0 || r->bwd_kernel > 2) return fail(FIBATTN_ERR_INVALID_ARG, "bwd_kernel must be 0, 1 or 2");
     if (!(r->rope_base > 1.f) || !std::isfinite(r->rope_base))
         return fail(FIBATTN_ERR_INVALID_ARG, "rope_base must be finite and > 1 (got %g)", (double)r->rope_base);
     if (!std::isfinite(r->scale)) return fail(FIBATTN_ERR_INVALID_ARG, "scale must be finite");
@@ -122,7 +124,8 @@ BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype) {
     size_t es = rot_size(dtype);
     size_t S = (size_t)W + 1 + K;
     Shape s; s.B = B; s.H = H; s.Hkv = Hkv; s.T = T; s.W = W; s.G = H / Hkv; s.scale = 1.f;
-    L.nblocks = bwd_simple_blocks(s);
+    L.nblocks = bwd_simple_blocks(s);               // rows of partial: the larger of the two query passes
+    if (bwd_mma_blocks(s) > L.nblocks) L.nblocks = bwd_mma_blocks(s);
     size_t off = 0;
     L.qt = off; off += align256((size_t)B * H * T * kHeadDim * es);
     L.kt = off; off += align256((size_t)B * Hkv * T * kHeadDim * es);
@@ -351,7 +354,7 @@ size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K, int
     return bwd_layout(B, H, o.Hkv, T, W, K, dtype).total;
 }
 
-int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, const void* dout,
+int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, const float* lse, const void* dout,
                 void* dq, void* dk, void* dv, float* dtheta, float* dd,
                 int B, int H, int T, int D, int W, float alpha, const float* offsets, int K,
                 int dtype, const fibattn_opts* opts, void* workspace, size_t workspace_bytes, void* stream) {
@@ -367,14 +370,15 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, c
     if (B > 0 && (!q || !k || !v || !lse || !dout || !dq || !dk || !dv))
         return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor pointer");
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(lse) || !aligned16(dout) || !aligned16(dq) ||
-        !aligned16(dk) || !aligned16(dv) || !aligned16(workspace) || ((uintptr_t)dtheta & 3u) || ((uintptr_t)dd & 3u))
+        !aligned16(dk) || !aligned16(dv) || !aligned16(workspace) || !aligned16(out) || ((uintptr_t)dtheta & 3u) ||
+        ((uintptr_t)dd & 3u))
         return fail(FIBATTN_ERR_INVALID_ARG, "pointers must be 16-byte aligned (dtheta, dd: 4-byte)");
     BwdLayout L = bwd_layout(B, H, o.Hkv, T, W, K, dtype);
     if (workspace_bytes < L.total) return fail(FIBATTN_ERR_INVALID_ARG, "workspace too small: %zu < %zu", workspace_bytes, L.total);
     prep_rope(o.rope_base, &a.rope);
     a.s = make_shape(B, H, T, W, o);
     char* ws = reinterpret_cast<char*>(workspace);
-    a.q = q; a.k = k; a.v = v; a.lse = lse; a.dout = dout; a.dq = dq; a.dk = dk; a.dv = dv;
+    a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.dout = dout; a.dq = dq; a.dk = dk; a.dv = dv;
     a.dtheta = dtheta; a.dd = dd;
     a.qt = ws + L.qt; a.kt = ws + L.kt;
     a.P = reinterpret_cast<float*>(ws + L.P); a.DP = reinterpret_cast<float*>(ws + L.DP);
@@ -387,19 +391,30 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const float* lse, c
     a.alpha = alpha;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool bf16 = dtype == FIBATTN_BF16;
+    MmaLayout ML;
+    const size_t smem_limit = 227 * 1024 - bwd_mma_static_smem();
+    const bool mma_ok = bf16 && out && (o.bwd_kernel == 0 || o.bwd_kernel == 2) &&
+                        build_mma_layout(a.s, a.r, o.rope_base, smem_limit, &ML);
+    if (o.bwd_kernel == 2 && !mma_ok)
+        return fail(FIBATTN_ERR_UNSUPPORTED, "tensor-core backward needs bf16, out, W <= 16, K <= 16 and a staged row "
+                                             "union that fits shared memory");
+    if (mma_ok) a.nblocks_a = B > 0 ? bwd_mma_blocks(a.s) : 0;
     cudaError_t e;
     if (B > 0) {
-        {
+        if (!mma_ok) {
             ProfScope p("rope_q", st);
             e = launch_rope_rows(q, a.qt, (long long)B * H * T, T, a.rope, bf16, st);
+            if (e != cudaSuccess) return cuda_fail(e, "rope prologue (q) launch");
         }
-        if (e != cudaSuccess) return cuda_fail(e, "rope prologue (q) launch");
         {
             ProfScope p("rope_k", st);
             e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
         }
         if (e != cudaSuccess) return cuda_fail(e, "rope prologue (k) launch");
-        {
+        if (mma_ok) {
+            ProfScope p("bwd_query_mma", st);
+            e = launch_bwd_query_mma(a, ML, st);
+        } else {
             ProfScope p("bwd_query", st);
             e = launch_bwd_query(a, bf16, st);
         }

@@ -57,6 +57,7 @@ struct BwdArgs {
     const void* v;
     const float* lse;         // [B,H,T]
     const void* dout;         // [B,H,T,D]
+    const void* out;          // forward output [B,H,T,D] or nullptr
     void* dq;                 // [B,H,T,D]
     void* dk;                 // [B,Hkv,T,D]
     void* dv;

@@ -33,114 +33,17 @@
 
 #include "fibattn_internal.cuh"
 #include "fwd_mma.cuh"
+#include "mma_common.cuh"
 
 namespace fibattn {
 namespace {
+
+using namespace mma;
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kWarps = kMmaWarps;
 constexpr int kRowsPerWarp = 15;                 // useful query rows of a 16-row tile
-constexpr unsigned kWaitLimit = 1u << 26;        // mbarrier polls before giving up
-
-// ------------------------------------------------------------------ PTX ----
-
-__device__ __forceinline__ unsigned smem_u32(const void* p) { return (unsigned)__cvta_generic_to_shared(p); }
-
-__device__ __forceinline__ void mbar_init(unsigned long long* bar, unsigned count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" :: "r"(smem_u32(bar)), "r"(count));
-}
-__device__ __forceinline__ void mbar_expect_tx(unsigned long long* bar, unsigned bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" :: "r"(smem_u32(bar)), "r"(bytes));
-}
-// Bounded wait on phase `parity`; returns false after kWaitLimit polls.
-__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity) {
-    const unsigned a = smem_u32(bar);
-    for (unsigned it = 0; it < kWaitLimit; ++it) {
-        unsigned done;
-        asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-                     " selp.u32 %0, 1, 0, p;\n}\n" : "=r"(done) : "r"(a), "r"(parity) : "memory");
-        if (done) return true;
-    }
-    return false;
-}
-__device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
-                                            unsigned long long* bar) {
-    asm volatile("cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes"
-                 " [%0], [%1, {%2, %3, %4}], [%5];\n"
-                 :: "r"(smem_u32(dst)), "l"(map), "r"(x), "r"(y), "r"(z), "r"(smem_u32(bar)) : "memory");
-}
-
-__device__ __forceinline__ void ldsm_x4(unsigned addr, unsigned& r0, unsigned& r1, unsigned& r2, unsigned& r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-__device__ __forceinline__ void ldsm_x4_t(unsigned addr, unsigned& r0, unsigned& r1, unsigned& r2, unsigned& r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];\n"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3) : "r"(addr));
-}
-
-__device__ __forceinline__ void mma_f16_16816(float* d, const unsigned* a, unsigned b0, unsigned b1) {
-    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-                 "{%0,%1,%2,%3};\n"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void mma_bf16_16816(float* d, const unsigned* a, unsigned b0, unsigned b1) {
-    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
-                 "{%0,%1,%2,%3};\n"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
-}
-__device__ __forceinline__ void mma_bf16_1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
-    asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, "
-                 "{%0,%1,%2,%3};\n"
-                 : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3]) : "r"(a0), "r"(a1), "r"(b0));
-}
-
-__device__ __forceinline__ unsigned pack_f16(float lo, float hi) {
-    __half2 h = __floats2half2_rn(lo, hi);
-    return *reinterpret_cast<unsigned*>(&h);
-}
-__device__ __forceinline__ unsigned pack_bf16(float lo, float hi) {
-    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<unsigned*>(&h);
-}
-__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
-
-__device__ __forceinline__ float quad_sum(float x) {
-    x += __shfl_xor_sync(0xffffffffu, x, 1);
-    x += __shfl_xor_sync(0xffffffffu, x, 2);
-    return x;
-}
-__device__ __forceinline__ float quad_max(float x) {
-    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 1));
-    x = fmaxf(x, __shfl_xor_sync(0xffffffffu, x, 2));
-    return x;
-}
-
-// Shared-memory byte address of 16-byte chunk `ch` of staged row `row` under the
-// 128-byte swizzle (chunk index XOR row % 8), buffer base 1024-byte aligned.
-__device__ __forceinline__ unsigned row_chunk(unsigned base, int row, int ch) {
-    return base + (unsigned)row * 128u + (unsigned)((ch ^ (row & 7)) << 4);
-}
-
-// Warp 0 issues the copies of one staged tensor: box b fills shared rows
-// [8b, 8b+8) from the interval that contains them.  Lane 0 announces the byte
-// count first; the boxes are then spread over the 32 lanes.
-__device__ __forceinline__ void issue_rows(unsigned char* dst, const CUtensorMap* map, const MmaLayout& L,
-                                           int i0, int head, unsigned long long* bar, int lane) {
-    if (lane == 0) mbar_expect_tx(bar, (unsigned)L.rows * 128u);
-    __syncwarp();
-    const int nbox = L.rows >> 3;
-    for (int bx = lane; bx < nbox; bx += 32) {
-        const int srow = bx * 8;
-        int iv = 0;
-        while (iv + 1 < L.n_iv && srow >= L.iv_smem[iv + 1]) ++iv;
-        const int rel = L.iv_start[iv] + (srow - L.iv_smem[iv]);
-        tma_load_3d(dst + (size_t)srow * 128, map, 0, i0 + rel, head, bar);
-    }
-}
 
 template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
@@ -440,7 +343,19 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
 
 // ------------------------------------------------------------ host side ----
 
-PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
+template <int NT>
+cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const FwdArgs& a, const MmaLayout& L,
+                      unsigned grid, size_t smem, cudaStream_t st) {
+    auto kern = fwd_mma_kernel<NT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kWarps * 32, smem, st>>>(mk, mv, a, L);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+static PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
         void* p = nullptr;
@@ -464,18 +379,6 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
-
-template <int NT>
-cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const FwdArgs& a, const MmaLayout& L,
-                      unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = fwd_mma_kernel<NT>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    kern<<<grid, kWarps * 32, smem, st>>>(mk, mv, a, L);
-    return cudaGetLastError();
-}
-
-}  // namespace
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.rows * 128 + 1024; }
 

@@ -1,5 +1,7 @@
 // fwd_mma.cuh -- host/device interface of the tensor-core forward kernel.
 #pragma once
+#include <cuda.h>
+
 #include "fibattn_internal.cuh"
 
 namespace fibattn {
@@ -26,6 +28,17 @@ struct MmaLayout {
 
 bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
 size_t fwd_mma_smem_bytes(const MmaLayout& L);
+// 3-D tensor map [heads][T][64] of 2-byte rows, 8-row boxes, 128-byte swizzle;
+// rows outside [0, T) read as zero.
+bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads);
 cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st);
+
+// Tensor-core query-centric backward over the same staged rows (bf16 I/O;
+// needs the forward output for Delta).  Its CTAs write rung partials as rows
+// [0, bwd_mma_blocks) of BwdArgs::partial; static shared memory is
+// bwd_mma_static_smem() bytes on top of fwd_mma_smem_bytes(L).
+size_t bwd_mma_static_smem();
+int bwd_mma_blocks(const Shape& s);
+cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st);
 
 }  // namespace fibattn

@@ -71,7 +71,7 @@ def _call_fwd(**kw):
                 K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0)
     args.update(kw)
     f = np.array([1, 2, 3] + [5] * 40, dtype=np.float32)
-    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, 0)
+    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, 0, 0)
     rc = lib.fibattn_fwd(args["q"], args["k"], args["v"], args["out"], args["lse"], args["B"], args["H"],
                          args["T"], args["D"], args["W"], args["alpha"], B._fptr(f), args["K"], args["dtype"],
                          ctypes.byref(o), args["ws"], args["wsb"], None)
@@ -94,17 +94,31 @@ def test_fwd_rejects_bad_arguments(kw, code):
 def test_bwd_rejects_bad_arguments():
     lib = B.lib()
     f = np.array([1, 2, 3], dtype=np.float32)
-    o = B.Opts(0.0, 0.0, 0, 0, 0)
+    o = B.Opts(0.0, 0.0, 0, 0, 0, 0)
     ok_ptr = 16
-    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None, None,
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, None, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None, None,
                          1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
     assert rc == 1 and "dtheta" in lib.fibattn_last_error().decode()
-    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, 18, None,
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, None, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, 18, None,
                          1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
     assert rc == 1
-    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None,
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, None, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None,
                          1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 8, None)
     assert rc == 1 and "workspace" in lib.fibattn_last_error().decode()
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, 24, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None,
+                         1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
+    assert rc == 1 and "aligned" in lib.fibattn_last_error().decode()       # misaligned out
+    for kern, code in ((3, 1), (-1, 1)):
+        o2 = B.Opts(0.0, 0.0, 0, 0, 0, kern)
+        rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None,
+                             1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o2), ok_ptr, 1 << 30, None)
+        assert rc == code and "bwd_kernel" in lib.fibattn_last_error().decode()
+    # the tensor-core query pass needs the forward output and bf16 I/O
+    for out_ptr, dt in ((None, 1), (ok_ptr, 0)):
+        o2 = B.Opts(0.0, 0.0, 0, 0, 0, 2)
+        rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, out_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None,
+                             1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, dt, ctypes.byref(o2), ok_ptr, 1 << 30, None)
+        assert rc == 2, lib.fibattn_last_error().decode()
 
 
 def test_workspace_queries():

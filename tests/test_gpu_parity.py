@@ -4,7 +4,7 @@ the same seeded inputs, element by element.
 Tolerances: fp32 I/O max abs error <= 1e-4 on out/lse and <= 1e-4 relative
 to the largest reference magnitude on gradients; bf16 I/O (fp32 accumulate)
 max abs error <= 1e-2 on out and <= 3e-2 relative (max |g - ref| / max |ref|,
-denominator floored at 1e-3) on gradients; dtheta |d - ref| / |ref|.
+denominator floored at 1e-2) on gradients; dtheta |d - ref| / |ref|.
 """
 from __future__ import annotations
 
@@ -83,10 +83,12 @@ def check_fwd(q, k, v, alpha, f, W, dedup=True, kernel="auto"):
     return out, lse
 
 
-def check_bwd(q, k, v, dout, alpha, f, W, dedup=True):
+def check_bwd(q, k, v, dout, alpha, f, W, dedup=True, kernel="auto"):
+    """kernel: backward query pass ("gather" runs without the forward output)."""
     qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), dout.cuda()
     out, lse = fa.fwd(qc, kc, vc, alpha, f, W, dedup=dedup)
-    dq, dk, dv, dth, dd = fa.bwd(qc, kc, vc, lse, gc, alpha, f, W, dedup=dedup)
+    dq, dk, dv, dth, dd = fa.bwd(qc, kc, vc, lse, gc, alpha, f, W, dedup=dedup, kernel=kernel,
+                                 out=None if kernel == "gather" else out)
     torch.cuda.synchronize()
     a32 = float(np.float32(alpha))
     d = O.offsets_fp32(a32, f.astype(np.float64))
@@ -140,14 +142,22 @@ def test_forward_small(case, dtype, kernel):
         raise
 
 
-@pytest.mark.parametrize("dtype", [torch.float32, torch.bfloat16], ids=["f32", "bf16"])
+BWD_KERNELS = [(torch.float32, "gather"), (torch.bfloat16, "gather"), (torch.bfloat16, "mma")]
+
+
+@pytest.mark.parametrize("dtype,kernel", BWD_KERNELS, ids=["f32", "bf16-gather", "bf16-mma"])
 @pytest.mark.parametrize("case", SMALL, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]}{c[6]}{c[7]}d{int(c[8])}"
                                               for c in SMALL])
-def test_backward_small(case, dtype):
+def test_backward_small(case, dtype, kernel):
     Bn, H, Hkv, T, W, alpha, base, K, dedup = case
     q, k, v = inputs.qkv(Bn, H, T, seed=T + W + 1, dtype=dtype, Hkv=Hkv)
     g = inputs.dout(Bn, H, T, seed=T + W + 2, dtype=dtype)
-    check_bwd(q, k, v, g, alpha, _offsets(base, K), W, dedup)
+    try:
+        check_bwd(q, k, v, g, alpha, _offsets(base, K), W, dedup, kernel)
+    except fa.FibattnError as e:
+        if e.status == 2:                        # kernel does not apply to this shape
+            pytest.skip(str(e))
+        raise
 
 
 def test_empty_batch():
@@ -164,12 +174,15 @@ def test_outputs_finite_and_deterministic():
     g = inputs.dout(2, 4, 700, seed=6, dtype=torch.bfloat16)
     qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), g.cuda()
     f = _offsets("fib", 15)
-    r1 = fa.bwd(qc, kc, vc, fa.fwd(qc, kc, vc, 0.77, f, 8)[1], gc, 0.77, f, 8)
-    r2 = fa.bwd(qc, kc, vc, fa.fwd(qc, kc, vc, 0.77, f, 8)[1], gc, 0.77, f, 8)
-    torch.cuda.synchronize()
-    for a, b in zip(r1, r2):
-        assert torch.equal(a, b)
-        assert torch.isfinite(a.float()).all()
+    for kernel in ("gather", "mma"):
+        o1, l1 = fa.fwd(qc, kc, vc, 0.77, f, 8)
+        r1 = fa.bwd(qc, kc, vc, l1, gc, 0.77, f, 8, out=o1, kernel=kernel)
+        o2, l2 = fa.fwd(qc, kc, vc, 0.77, f, 8)
+        r2 = fa.bwd(qc, kc, vc, l2, gc, 0.77, f, 8, out=o2, kernel=kernel)
+        torch.cuda.synchronize()
+        for a, b in zip(r1, r2):
+            assert torch.equal(a, b)
+            assert torch.isfinite(a.float()).all()
 
 
 # --------------------------------------------- full-size workload configs --
@@ -211,7 +224,9 @@ def test_config4_bf16_backward_learned_alpha():
         s = inputs.layer_seed(3, layer)
         q, k, v = inputs.qkv(16, 8, 1024, seed=s, dtype=torch.bfloat16)
         g = inputs.dout(16, 8, 1024, seed=s, dtype=torch.bfloat16)
-        check_bwd(q, k, v, g, float(alphas[layer]), f, 8)
+        check_bwd(q, k, v, g, float(alphas[layer]), f, 8, kernel="mma")
+        if layer == 0:
+            check_bwd(q, k, v, g, float(alphas[layer]), f, 8, kernel="gather")
 
 
 @pytest.mark.parametrize("base,K", [("fib", 15), ("pow2", 10)])

@@ -31,7 +31,7 @@ def _noalloc(q, k, v, alpha, f, W, out, lse):
                                       ctypes.POINTER(ctypes.c_float), ci, ci, ctypes.POINTER(B.Opts), vp]
     L.fibattn_fwd_noalloc.restype = ci
     f32 = np.ascontiguousarray(np.asarray(f, dtype=np.float32))
-    o = B.Opts(1e4, 0.0, k.shape[1], 0, 0)
+    o = B.Opts(1e4, 0.0, k.shape[1], 0, 0, 0)
     Bn, H, T, D = q.shape
     code = 1 if q.dtype == torch.bfloat16 else 0
     return L.fibattn_fwd_noalloc(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), lse.data_ptr(),
