@@ -1,0 +1,269 @@
+// bwd_key_mma.cu -- key-centric backward on tensor cores (mma.sync, m16n8)
+// with TMA staging (arXiv 2606.28560, Section 2 "Attended set"; the chain
+// rule of the forward).
+//
+// Key row j receives, from each query head of its group, the slots that read
+// it: window slot t of query j + t (weight 1), rung k of query j + s0_k (its
+// floor row, weight 1 - w_k) and of query j + s0_k + 1 (its far row, weight w_k):
+//   dv_j  = sum c p dO_i,        dk~_j = scale sum c dS q~_i,
+// with p and dS = p (dp - Delta) per (query, slot) from the tensor-core query
+// pass (slot-major arrays, read as runs of consecutive queries).  A warp owns 16 keys (tiles every 15 keys, the 16th row discarded);
+// with the keys as MMA rows and the queries as the reduction index both sums
+// are products of a banded matrix with staged query rows:
+//   window band  acc += P_band^T  X[b, b+16+Wp)       P_band^T[r][x] = p(b+x, t = x-r)
+//   rung k       acc += Phat_k^T  X[b+s0, b+s0+16)    Phat_k^T[r][r] = (1-w) p, [r][r+1] = w p
+// with X = dO rows (bf16, pass 1: dv) and then X = q~ rows (fp16, pass 2:
+// dk~, dS in place of p).  The CTA stages the union of the query rows its
+// warps read, one tensor (and query head) at a time, in one buffer.
+// A-operand values: p as bf16, dS as fp16; accumulation fp32.
+#include <cmath>
+
+#include "fibattn_internal.cuh"
+#include "fwd_mma.cuh"
+#include "mma_common.cuh"
+
+namespace fibattn {
+namespace {
+
+using namespace mma;
+
+constexpr int kWarps = kMmaWarps;
+constexpr int kRowsPerWarp = 15;
+
+template <bool F16>
+__device__ __forceinline__ unsigned pack2(float lo, float hi) {
+    return F16 ? pack_f16(lo, hi) : pack_bf16(lo, hi);
+}
+template <bool F16>
+__device__ __forceinline__ void mma16816(float* d, const unsigned* a, unsigned b0, unsigned b1) {
+    if constexpr (F16) mma_f16_16816(d, a, b0, b1); else mma_bf16_16816(d, a, b0, b1);
+}
+template <bool F16>
+__device__ __forceinline__ void mma1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
+    if constexpr (F16) mma_f16_1688(d, a0, a1, b0); else mma_bf16_1688(d, a0, a1, b0);
+}
+
+// One staged tensor of one query head: accumulate banded A x staged rows.
+// X: p or dS of this query head, slot-major [S][T]; F16: the operand type.
+template <int NT, bool F16>
+__device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, const BwdArgs& a, const MmaLayout& L,
+                                         unsigned sbase, int bw, int wrel, int g4, int c4, int lane, bool vlo,
+                                         bool vhi, unsigned long long* bar, unsigned parity, bool& ok,
+                                         float (*rv)[16]) {
+    const Shape& s = a.s;
+    // ---- rung values of the warp's 16 slab columns, all rungs at once (the
+    // loads are independent, so their latencies overlap): rv[k][x] = p or dS of
+    // query bw + s0_k + x, rung slot k (0 past the end of the sequence)
+#pragma unroll
+    for (int i = 0; i < kMmaMaxRungs * 16 / 32; ++i) {
+        const int u = lane + 32 * i;
+        const int k = u >> 4, x = u & 15;
+        const int q = bw + a.r.s0[k] + x;
+        const bool use = k < a.r.K && ((a.r.active >> k) & 1u) && q < s.T;
+        rv[k][x] = use ? X[(size_t)(s.W + 1 + k) * s.T + q] : 0.f;
+    }
+    __syncwarp();
+    // ---- window band values (loaded while the copies are in flight)
+    unsigned band[NT][2];
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+        float v[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const bool hi = e >= 2;
+            const int r = hi ? g4 + 8 : g4;
+            const int x = 8 * j + 2 * c4 + (e & 1);
+            const int t = x - r;                              // query - key
+            const int q = bw + x;
+            const bool use = (hi ? vhi : vlo) && t >= 0 && t <= s.W && q < s.T;
+            v[e] = use ? X[(size_t)t * s.T + q] : 0.f;
+        }
+        band[j][0] = pack2<F16>(v[0], v[1]);
+        band[j][1] = pack2<F16>(v[2], v[3]);
+    }
+    ok = mbar_wait(bar, parity) && ok;
+
+#pragma unroll
+    for (int kk = 0; kk + 1 < NT; kk += 2) {
+        const unsigned afr[4] = {band[kk][0], band[kk][1], band[kk + 1][0], band[kk + 1][1]};
+        const int xrow = L.win_smem + wrel + 8 * kk + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+        for (int n = 0; n < 8; n += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
+            mma16816<F16>(acc[n], afr, b0, b1);
+            mma16816<F16>(acc[n + 1], afr, b2, b3);
+        }
+    }
+    if constexpr (NT & 1) {
+        const int kk = NT - 1;
+        const int xrow = L.win_smem + wrel + 8 * kk + (lane & 7);
+#pragma unroll
+        for (int n = 0; n < 8; n += 4) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 3)), b0, b1, b2, b3);
+            mma1688<F16>(acc[n], band[kk][0], band[kk][1], b0);
+            mma1688<F16>(acc[n + 1], band[kk][0], band[kk][1], b1);
+            mma1688<F16>(acc[n + 2], band[kk][0], band[kk][1], b2);
+            mma1688<F16>(acc[n + 3], band[kk][0], band[kk][1], b3);
+        }
+    }
+
+    // ---- rungs: slab column x is query bw + s0 + x; row r takes x = r (floor
+    // side, weight 1-w) and x = r+1 (far side, weight w)
+#pragma unroll 1
+    for (int k = 0; k < a.r.K; ++k) {
+        if (!((a.r.active >> k) & 1u)) continue;
+        const int s0 = a.r.s0[k];
+        if (bw + s0 >= s.T) continue;                      // every query of the slab is past the end
+        const float w = a.r.w[k], w1 = 1.f - w;
+        float v[2][4];                                     // [row half][column slot]
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const int r = g4 + 8 * half;
+#pragma unroll
+            for (int cs = 0; cs < 4; ++cs) {
+                const int x = 2 * c4 + (cs & 1) + 8 * (cs >> 1);
+                const float c = (x == r) ? w1 : ((x == r + 1) ? w : 0.f);
+                const bool use = c != 0.f && (half ? vhi : vlo);
+                v[half][cs] = use ? c * rv[k][x] : 0.f;
+            }
+        }
+        const unsigned afr[4] = {pack2<F16>(v[0][0], v[0][1]), pack2<F16>(v[1][0], v[1][1]),
+                                 pack2<F16>(v[0][2], v[0][3]), pack2<F16>(v[1][2], v[1][3])};
+        const int xrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+        for (int n = 0; n < 8; n += 2) {
+            unsigned b0, b1, b2, b3;
+            ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
+            mma16816<F16>(acc[n], afr, b0, b1);
+            mma16816<F16>(acc[n + 1], afr, b2, b3);
+        }
+    }
+}
+
+template <int NT>
+__global__ void __launch_bounds__(kWarps * 32, 2)
+bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ RowMaps tmG, BwdArgs a,
+                   MmaLayout L) {
+    extern __shared__ unsigned char smem_raw[];
+    __shared__ unsigned long long bar;
+    __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
+    unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
+    const unsigned sbase = smem_u32(buf);
+
+    const Shape s = a.s;
+    const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
+    const int bhk = blockIdx.x / tiles;                   // b * Hkv + hk
+    const int j0 = (blockIdx.x % tiles) * kMmaTile;
+    const int b = bhk / s.Hkv, hk = bhk % s.Hkv;
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int g4 = lane >> 2, c4 = lane & 3;
+    const int wrel = warp * kRowsPerWarp;
+    const int bw = j0 + wrel;
+    const int klo = bw + g4, khi = bw + g4 + 8;
+    const bool vlo = klo < s.T && g4 < kRowsPerWarp;
+    const bool vhi = khi < s.T && g4 + 8 < kRowsPerWarp;
+
+    if (tid == 0) {
+        mbar_init(&bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    __syncthreads();
+
+    unsigned parity = 0;
+    bool ok = true;
+    const size_t krow0 = (size_t)bhk * s.T;
+#pragma unroll 1
+    for (int pass = 0; pass < 2; ++pass) {                // 0: dv from dO rows; 1: dk~ from q~ rows
+        float acc[8][4];
+#pragma unroll
+        for (int n = 0; n < 8; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;
+#pragma unroll 1
+        for (int g = 0; g < s.G; ++g) {
+            const int qhead = b * s.H + hk * s.G + g;
+            const float* X = (pass ? a.DSs : a.Ps) + (size_t)qhead * a.S * s.T;
+            if (warp == 0) {
+                const RowMaps& m = pass ? tmQ : tmG;
+                issue_rows(buf, &m.m64, &m.m8, L, j0, qhead, &bar, lane);
+            }
+            if (pass == 0)
+                key_pass<NT, false>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
+                                       rvals[warp]);
+            else
+                key_pass<NT, true>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
+                                      rvals[warp]);
+            parity ^= 1u;
+            // every warp is done with the staged rows before the buffer is refilled
+            asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+            __syncthreads();
+        }
+        const float sc = ok ? (pass ? s.scale : 1.f) : __int_as_float(0x7fc00000);
+        __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(pass ? a.dk : a.dv) + krow0 * kHeadDim;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            if (!(half ? vhi : vlo)) continue;
+            const int key = half ? khi : klo;
+#pragma unroll
+            for (int n = 0; n < 8; ++n) {
+                acc[n][2 * half] *= sc;
+                acc[n][2 * half + 1] *= sc;
+            }
+            if (pass) {                                   // dk = R(-theta key) dk~
+#pragma unroll
+                for (int n = 0; n < 4; ++n) {
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const int m = 8 * n + 2 * c4 + u;     // pair (m, m + 32): n-tiles n and n + 4
+                        float c, sn;
+                        rope_cs(a.rope, m, key, c, sn);
+                        const float xa = acc[n][2 * half + u], xb = acc[n + 4][2 * half + u];
+                        acc[n][2 * half + u] = xa * c + xb * sn;
+                        acc[n + 4][2 * half + u] = xb * c - xa * sn;
+                    }
+                }
+            }
+            __nv_bfloat16* row = dst + (size_t)key * kHeadDim;
+#pragma unroll
+            for (int n = 0; n < 8; ++n)
+                *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(acc[n][2 * half], acc[n][2 * half + 1]);
+        }
+    }
+}
+
+template <int NT>
+cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, const MmaLayout& L,
+                      unsigned grid, size_t smem, cudaStream_t st) {
+    auto kern = bwd_key_mma_kernel<NT>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    kern<<<grid, kWarps * 32, smem, st>>>(mq, mg, a, L);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+size_t bwd_key_mma_static_smem() { return sizeof(float) * kWarps * kMmaMaxRungs * 16 + 64; }
+
+int bwd_key_mma_blocks(const Shape& s) {
+    const long long tiles = (s.T + kMmaTile - 1) / kMmaTile;
+    return (int)(tiles * s.B * s.Hkv);
+}
+
+cudaError_t launch_bwd_key_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st) {
+    const long long grid = bwd_key_mma_blocks(a.s);
+    if (grid <= 0) return cudaSuccess;
+    RowMaps mq, mg;
+    const int heads = a.s.B * a.s.H;
+    if (!encode_row_maps(&mq, a.qt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
+        !encode_row_maps(&mg, a.dout, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
+        return cudaErrorInvalidValue;
+    const size_t smem = fwd_mma_smem_bytes(L);
+    switch (L.nt) {
+    case 2: return launch_nt<2>(mq, mg, a, L, (unsigned)grid, smem, st);
+    case 3: return launch_nt<3>(mq, mg, a, L, (unsigned)grid, smem, st);
+    default: return launch_nt<4>(mq, mg, a, L, (unsigned)grid, smem, st);
+    }
+}
+
+}  // namespace fibattn

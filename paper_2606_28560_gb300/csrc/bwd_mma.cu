@@ -18,9 +18,10 @@
 //
 // and the rung-distance gradient of query i (row -1 is a zero row):
 //   dL/dd_k += p (scale (s1 - s0)(dp - Delta) + ddp)
-// with s1, s0 the raw far and floor dot products.  P, dp per slot (zero where
-// not attended), Delta and the rotated queries go to the workspace for the
-// key-centric pass.  dS enters the dq MMAs as fp16 (11-bit significand);
+// with s1, s0 the raw far and floor dot products.  p and dS per slot (zero
+// where not attended; slot-major arrays [head][slot][T], so that the key pass
+// reads runs of consecutive queries), Delta and the rotated queries go to the
+// workspace for the key-centric pass.  dS enters the dq MMAs as fp16 (11-bit significand);
 // accumulation is fp32.
 #include <cmath>
 
@@ -42,7 +43,7 @@ __device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 
 
 template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
-bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                      BwdArgs a, MmaLayout L) {
     constexpr int Wp = NT * 8 - 16;
     extern __shared__ unsigned char smem_raw[];
@@ -71,7 +72,7 @@ bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
     }
     if (warp == 0) {
         __syncwarp();
-        issue_rows(buf, &tmV, L, i0, head, &bars[0], lane);
+        issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[0], lane);
     }
 
     const int qlo = bw + g4, qhi = bw + g4 + 8;
@@ -239,12 +240,12 @@ bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
     // ---- all warps are done with the values: stage the keys into the same buffer
     asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
     __syncthreads();
-    if (warp == 0) issue_rows(buf, &tmK, L, i0, head, &bars[1], lane);
+    if (warp == 0) issue_rows(buf, &tmK.m64, &tmK.m8, L, i0, head, &bars[1], lane);
     const bool ok_k = mbar_wait(&bars[1], 0);
 
     const float sc2 = s.scale * kLog2e;
-    float* Pg = a.P + rowbase * a.S;
-    float* DPg = a.DP + rowbase * a.S;
+    float* Pg = a.Ps + (size_t)bh * a.S * s.T;       // [slot][T] of this head
+    float* DSg = a.DSs + (size_t)bh * a.S * s.T;
 
     float dq[8][4];
 #pragma unroll
@@ -282,9 +283,8 @@ bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
                 const float p = ok ? exp2f(sw[j][e] * sc2 - (hi ? lse2_hi : lse2_lo)) : 0.f;
                 dsv[e] = p * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
                 if (rv && inband) {
-                    const size_t off = (size_t)(bw + r) * a.S + t;
-                    Pg[off] = p;
-                    DPg[off] = ok ? dpw[j][e] : 0.f;
+                    Pg[(size_t)t * s.T + bw + r] = p;
+                    DSg[(size_t)t * s.T + bw + r] = dsv[e];
                 }
             }
             dsa[j][0] = pack_f16(dsv[0], dsv[1]);
@@ -325,8 +325,8 @@ bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
         const int slot = s.W + 1 + k;
         if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) {   // masked for every row of the tile
             if (c4 == 0) {
-                if (vlo) { Pg[(size_t)qlo * a.S + slot] = 0.f; DPg[(size_t)qlo * a.S + slot] = 0.f; }
-                if (vhi) { Pg[(size_t)qhi * a.S + slot] = 0.f; DPg[(size_t)qhi * a.S + slot] = 0.f; }
+                if (vlo) { Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
+                if (vhi) { Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
             }
             if (lane == 0) gsm[warp][k] = 0.f;
             continue;
@@ -362,8 +362,8 @@ bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
         const float e_lo = dp_lo - dlt_lo, e_hi = dp_hi - dlt_hi;
         const float ds_lo = p_lo * e_lo, ds_hi = p_hi * e_hi;
         if (c4 == 0) {
-            if (vlo) { Pg[(size_t)qlo * a.S + slot] = p_lo; DPg[(size_t)qlo * a.S + slot] = okl ? dp_lo : 0.f; }
-            if (vhi) { Pg[(size_t)qhi * a.S + slot] = p_hi; DPg[(size_t)qhi * a.S + slot] = okh ? dp_hi : 0.f; }
+            if (vlo) { Pg[(size_t)slot * s.T + qlo] = p_lo; DSg[(size_t)slot * s.T + qlo] = ds_lo; }
+            if (vhi) { Pg[(size_t)slot * s.T + qhi] = p_hi; DSg[(size_t)slot * s.T + qhi] = ds_hi; }
         }
         // dL/dd_k of this warp's rows, in a fixed order over the rows
         float g = 0.f;
@@ -440,7 +440,7 @@ bwd_query_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_const
 }
 
 template <int NT>
-cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const BwdArgs& a, const MmaLayout& L,
+cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const BwdArgs& a, const MmaLayout& L,
                       unsigned grid, size_t smem, cudaStream_t st) {
     auto kern = bwd_query_mma_kernel<NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -463,10 +463,10 @@ int bwd_mma_blocks(const Shape& s) {
 cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st) {
     const long long grid = bwd_mma_blocks(a.s);
     if (grid <= 0) return cudaSuccess;
-    CUtensorMap mk, mv;
+    RowMaps mk, mv;
     const int heads = a.s.B * a.s.Hkv;
-    if (!encode_rows_map(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
-        !encode_rows_map(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
+    if (!encode_row_maps(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
+        !encode_row_maps(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
         return cudaErrorInvalidValue;
     const size_t smem = fwd_mma_smem_bytes(L);
     switch (L.nt) {

@@ -391,10 +391,13 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     a.alpha = alpha;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool bf16 = dtype == FIBATTN_BF16;
-    MmaLayout ML;
+    MmaLayout ML, KL;
     const size_t smem_limit = 227 * 1024 - bwd_mma_static_smem();
     const bool mma_ok = bf16 && out && (o.bwd_kernel == 0 || o.bwd_kernel == 2) &&
-                        build_mma_layout(a.s, a.r, o.rope_base, smem_limit, &ML);
+                        build_mma_layout(a.s, a.r, o.rope_base, smem_limit, &ML) &&
+                        build_key_layout(a.s, a.r, o.rope_base, 227 * 1024 - bwd_key_mma_static_smem(), &KL);
+    a.Ps = reinterpret_cast<float*>(ws + L.P);      // slot-major p and dS of the tensor-core passes
+    a.DSs = reinterpret_cast<float*>(ws + L.DP);
     if (o.bwd_kernel == 2 && !mma_ok)
         return fail(FIBATTN_ERR_UNSUPPORTED, "tensor-core backward needs bf16, out, W <= 16, K <= 16 and a staged row "
                                              "union that fits shared memory");
@@ -419,7 +422,10 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
             e = launch_bwd_query(a, bf16, st);
         }
         if (e != cudaSuccess) return cuda_fail(e, "backward query-pass launch");
-        {
+        if (mma_ok) {
+            ProfScope p("bwd_key_mma", st);
+            e = launch_bwd_key_mma(a, KL, st);
+        } else {
             ProfScope p("bwd_key", st);
             e = launch_bwd_key(a, bf16, st);
         }

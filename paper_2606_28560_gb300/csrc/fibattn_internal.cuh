@@ -69,6 +69,8 @@ struct BwdArgs {
     float* P;                 // softmax probabilities [B,H,T,S]
     float* DP;                // dL/dp = dO . val per slot [B,H,T,S]
     float* Delta;             // sum_slots p dL/dp per query [B,H,T]
+    float* Ps;                // tensor-core path, slot-major [B,H,S,T]: p      (P region)
+    float* DSs;               //                                      dS = p (dp - Delta)  (DP region)
     float* partial;           // per-block dL/dd_k partial sums [kMaxRungs][nblocks]
     double* colsum;           // dL/dd_k column sums [kMaxRungs]
     unsigned* ticket;         // finalize completion counter (reset by the query pass)

@@ -47,7 +47,7 @@ constexpr int kRowsPerWarp = 15;                 // useful query rows of a 16-ro
 
 template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
-fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ CUtensorMap tmV,
+fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                FwdArgs a, MmaLayout L) {
     constexpr int Wp = NT * 8 - 16;               // window rows before the tile
     extern __shared__ unsigned char smem_raw[];
@@ -74,7 +74,7 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
     }
     if (warp == 0) {
         __syncwarp();
-        issue_rows(buf, &tmK, L, i0, head, &bars[0], lane);
+        issue_rows(buf, &tmK.m64, &tmK.m8, L, i0, head, &bars[0], lane);
     }
 
     // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32)
@@ -224,7 +224,7 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
     // ---- all warps are done with the keys: stage the values into the same buffer
     asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
     __syncthreads();
-    if (warp == 0) issue_rows(buf, &tmV, L, i0, head, &bars[1], lane);
+    if (warp == 0) issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
 
     // ---- probabilities (unnormalised, row max -> exactly 1) while values arrive
     if (mlo == -INFINITY) mlo = 0.f;              // rows beyond T: keep arithmetic finite
@@ -344,7 +344,7 @@ fwd_mma_kernel(const __grid_constant__ CUtensorMap tmK, const __grid_constant__ 
 // ------------------------------------------------------------ host side ----
 
 template <int NT>
-cudaError_t launch_nt(const CUtensorMap& mk, const CUtensorMap& mv, const FwdArgs& a, const MmaLayout& L,
+cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const FwdArgs& a, const MmaLayout& L,
                       unsigned grid, size_t smem, cudaStream_t st) {
     auto kern = fwd_mma_kernel<NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -367,12 +367,12 @@ static PFN_cuTensorMapEncodeTiled_v12000 get_encode() {
     return fn;
 }
 
-bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads) {
+bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads, int box_rows) {
     auto fn = get_encode();
     if (!fn) return false;
     cuuint64_t dims[3] = {(cuuint64_t)kHeadDim, (cuuint64_t)T, (cuuint64_t)heads};
     cuuint64_t strides[2] = {(cuuint64_t)kHeadDim * 2, (cuuint64_t)T * kHeadDim * 2};
-    cuuint32_t box[3] = {(cuuint32_t)kHeadDim, 8, 1};
+    cuuint32_t box[3] = {(cuuint32_t)kHeadDim, (cuuint32_t)box_rows, 1};
     cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = fn(map, dt, 3, const_cast<void*>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                     CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -382,18 +382,13 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.rows * 128 + 1024; }
 
-bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L) {
-    if (s.W > 16 || r.K > kMmaMaxRungs) return false;
-    const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
-    const int Wp = NT * 8 - 16;
-    L->nt = NT;
-    // relative rows each warp tile reads; the tile spans rows [0, kMmaTile + 1)
-    struct Iv { int a, b; };
-    Iv iv[kMmaMaxRungs + 1];
-    int n = 0;
-    iv[n++] = {-Wp, kMmaTile + 1};
-    for (int k = 0; k < r.K; ++k)
-        if ((r.active >> k) & 1u) iv[n++] = {-r.s0[k] - 1, kMmaTile + 1 - r.s0[k]};
+namespace {
+
+struct Iv { int a, b; };
+
+// Merge relative row intervals (sorted by start), round each merged interval up
+// to whole 8-row TMA boxes and lay them out one after another in shared memory.
+void layout_intervals(Iv* iv, int n, MmaLayout* L) {
     for (int i = 1; i < n; ++i)                   // insertion sort by start
         for (int j = i; j > 0 && iv[j].a < iv[j - 1].a; --j) { Iv t = iv[j]; iv[j] = iv[j - 1]; iv[j - 1] = t; }
     int m = 0;
@@ -411,20 +406,63 @@ bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, siz
         rows += len;
     }
     L->rows = rows;
-    auto smem_row = [&](int rel) {
-        for (int i = 0; i < L->n_iv; ++i)
-            if (rel >= L->iv_start[i] && rel < L->iv_start[i] + L->iv_len[i]) return L->iv_smem[i] + (rel - L->iv_start[i]);
-        return -1;
-    };
-    L->win_smem = smem_row(0);
+}
+
+int smem_row_of(const MmaLayout& L, int rel) {
+    for (int i = 0; i < L.n_iv; ++i)
+        if (rel >= L.iv_start[i] && rel < L.iv_start[i] + L.iv_len[i]) return L.iv_smem[i] + (rel - L.iv_start[i]);
+    return -1;
+}
+
+void rope_steps(double rope_base, MmaLayout* L) {
     for (int m = 0; m < kHalf; ++m) {
         const double theta = std::pow(rope_base, -2.0 * m / (double)kHeadDim);
         L->rope_c8[m] = (float)std::cos(8.0 * theta);
         L->rope_s8[m] = (float)std::sin(8.0 * theta);
     }
+}
+
+}  // namespace
+
+bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L) {
+    if (s.W > 16 || r.K > kMmaMaxRungs) return false;
+    const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
+    const int Wp = NT * 8 - 16;
+    L->nt = NT;
+    // relative rows each warp tile reads; the tile spans rows [0, kMmaTile + 1)
+    Iv iv[kMmaMaxRungs + 1];
+    int n = 0;
+    iv[n++] = {-Wp, kMmaTile + 1};
+    for (int k = 0; k < r.K; ++k)
+        if ((r.active >> k) & 1u) iv[n++] = {-r.s0[k] - 1, kMmaTile + 1 - r.s0[k]};
+    layout_intervals(iv, n, L);
+    L->win_smem = smem_row_of(*L, 0);
+    rope_steps(rope_base, L);
     for (int k = 0; k < kMmaMaxRungs; ++k) L->rung_smem[k] = 0;
     for (int k = 0; k < r.K; ++k)
-        if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row(-r.s0[k] - 1);
+        if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row_of(*L, -r.s0[k] - 1);
+    return fwd_mma_smem_bytes(*L) <= smem_limit;
+}
+
+bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L) {
+    if (s.W > 16 || r.K > kMmaMaxRungs) return false;
+    const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
+    const int Wp = NT * 8 - 16;
+    L->nt = NT;
+    // query rows, relative to the first key of the tile, that a key tile's
+    // warps read: the band [0, kMmaTile + 1 + Wp) and per rung the slab
+    // [s0, s0 + kMmaTile + 1) (near query j + s0 and far query j + s0 + 1)
+    Iv iv[kMmaMaxRungs + 1];
+    int n = 0;
+    iv[n++] = {0, kMmaTile + 1 + Wp};
+    for (int k = 0; k < r.K; ++k)
+        if ((r.active >> k) & 1u) iv[n++] = {r.s0[k], r.s0[k] + kMmaTile + 1};
+    layout_intervals(iv, n, L);
+    L->win_smem = smem_row_of(*L, 0);
+    rope_steps(rope_base, L);
+    for (int k = 0; k < kMmaMaxRungs; ++k) L->rung_smem[k] = 0;
+    for (int k = 0; k < r.K; ++k)
+        if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row_of(*L, r.s0[k]);
     return fwd_mma_smem_bytes(*L) <= smem_limit;
 }
 
@@ -432,10 +470,10 @@ cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st
     const long long tiles = (a.s.T + kMmaTile - 1) / kMmaTile;
     const long long grid = tiles * a.s.B * a.s.H;
     if (grid <= 0) return cudaSuccess;
-    CUtensorMap mk, mv;
+    RowMaps mk, mv;
     const int heads = a.s.B * a.s.Hkv;
-    if (!encode_rows_map(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
-        !encode_rows_map(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
+    if (!encode_row_maps(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
+        !encode_row_maps(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
         return cudaErrorInvalidValue;
     const size_t smem = fwd_mma_smem_bytes(L);
     switch (L.nt) {

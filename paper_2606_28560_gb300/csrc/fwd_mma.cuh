@@ -27,10 +27,19 @@ struct MmaLayout {
 };
 
 bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
+// Key-centric counterpart: query rows [0, M+1+Wp) and [s0, s0+M+1) relative to
+// the first key of a tile (win_smem: relative row 0; rung_smem[k]: row s0_k).
+bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
 size_t fwd_mma_smem_bytes(const MmaLayout& L);
-// 3-D tensor map [heads][T][64] of 2-byte rows, 8-row boxes, 128-byte swizzle;
-// rows outside [0, T) read as zero.
-bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads);
+// 3-D tensor map [heads][T][64] of 2-byte rows, boxes of box_rows rows,
+// 128-byte swizzle; rows outside [0, T) read as zero.
+bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads, int box_rows);
+
+// A staged tensor: the same rows as 64-row and as 8-row boxes.
+struct RowMaps { CUtensorMap m64, m8; };
+inline bool encode_row_maps(RowMaps* m, const void* base, CUtensorMapDataType dt, int T, int heads) {
+    return encode_rows_map(&m->m64, base, dt, T, heads, 64) && encode_rows_map(&m->m8, base, dt, T, heads, 8);
+}
 cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st);
 
 // Tensor-core query-centric backward over the same staged rows (bf16 I/O;
@@ -40,5 +49,10 @@ cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st
 size_t bwd_mma_static_smem();
 int bwd_mma_blocks(const Shape& s);
 cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st);
+// Tensor-core key-centric backward: dv and dk from the {p, dS} pairs of the
+// tensor-core query pass, staging q~ and dO rows of the layout above.
+int bwd_key_mma_blocks(const Shape& s);
+size_t bwd_key_mma_static_smem();
+cudaError_t launch_bwd_key_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st);
 
 }  // namespace fibattn

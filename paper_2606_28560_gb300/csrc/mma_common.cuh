@@ -94,20 +94,20 @@ __device__ __forceinline__ unsigned row_chunk(unsigned base, int row, int ch) {
     return base + (unsigned)row * 128u + (unsigned)((ch ^ (row & 7)) << 4);
 }
 
-// Warp 0 issues the copies of one staged tensor: box b fills shared rows
-// [8b, 8b+8) from the interval that contains them.  Lane 0 announces the byte
-// count first; the boxes are then spread over the 32 lanes.
-__device__ __forceinline__ void issue_rows(unsigned char* dst, const CUtensorMap* map, const MmaLayout& L,
-                                           int i0, int head, unsigned long long* bar, int lane) {
+// Warp 0 issues the copies of one staged tensor.  Lane n copies merged
+// interval n: whole 64-row boxes (map64) first, then 8-row boxes (map8) for
+// the rest of it (interval lengths are multiples of 8 rows).  Large boxes move
+// the same rows at well over the rate of 8-row ones.  Lane 0 announces the
+// byte count before any copy is issued.
+__device__ __forceinline__ void issue_rows(unsigned char* dst, const CUtensorMap* map64, const CUtensorMap* map8,
+                                           const MmaLayout& L, int i0, int head, unsigned long long* bar, int lane) {
     if (lane == 0) mbar_expect_tx(bar, (unsigned)L.rows * 128u);
     __syncwarp();
-    const int nbox = L.rows >> 3;
-    for (int bx = lane; bx < nbox; bx += 32) {
-        const int srow = bx * 8;
-        int iv = 0;
-        while (iv + 1 < L.n_iv && srow >= L.iv_smem[iv + 1]) ++iv;
-        const int rel = L.iv_start[iv] + (srow - L.iv_smem[iv]);
-        tma_load_3d(dst + (size_t)srow * 128, map, 0, i0 + rel, head, bar);
+    for (int iv = lane; iv < L.n_iv; iv += 32) {
+        const int len = L.iv_len[iv], srow = L.iv_smem[iv], grow = i0 + L.iv_start[iv];
+        int r = 0;
+        for (; r + 64 <= len; r += 64) tma_load_3d(dst + (size_t)(srow + r) * 128, map64, 0, grow + r, head, bar);
+        for (; r < len; r += 8) tma_load_3d(dst + (size_t)(srow + r) * 128, map8, 0, grow + r, head, bar);
     }
 }
 
