@@ -110,27 +110,29 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
     }
 
     // ---- rungs: slab column x is query bw + s0 + x; row r takes x = r (floor
-    // side, weight 1-w) and x = r+1 (far side, weight w)
+    // side, weight 1-w) and x = r+1 (far side, weight w).  In this thread's A
+    // fragment (rows g4, g4+8; columns 2c4, 2c4+1, 2c4+8, 2c4+9) the nonzero
+    // pattern depends only on delta = 2c4 - g4: registers a0 (row g4, columns
+    // 2c4..) and a3 (row g4+8, columns 2c4+8..) share the coefficients
+    //   column x0:   1-w if delta = 0,  w if delta = 1
+    //   column x0+1: 1-w if delta = -1, w if delta = 0,
+    // a1 (row g4+8, columns 2c4..) is always zero and a2 (row g4, columns
+    // 2c4+8..) holds only w at column 8 of row 7 (lane g4 = 7, c4 = 0).
+    const int dl = 2 * c4 - g4;
+    const float alo = dl == 0 ? 1.f : 0.f, blo = dl == 0 ? -1.f : (dl == 1 ? 1.f : 0.f);
+    const float ahi = dl == -1 ? 1.f : 0.f, bhi = dl == -1 ? -1.f : (dl == 0 ? 1.f : 0.f);
+    const float m2 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
 #pragma unroll 1
     for (int k = 0; k < a.r.K; ++k) {
         if (!((a.r.active >> k) & 1u)) continue;
         const int s0 = a.r.s0[k];
         if (bw + s0 >= s.T) continue;                      // every query of the slab is past the end
-        const float w = a.r.w[k], w1 = 1.f - w;
-        float v[2][4];                                     // [row half][column slot]
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            const int r = g4 + 8 * half;
-#pragma unroll
-            for (int cs = 0; cs < 4; ++cs) {
-                const int x = 2 * c4 + (cs & 1) + 8 * (cs >> 1);
-                const float c = (x == r) ? w1 : ((x == r + 1) ? w : 0.f);
-                const bool use = c != 0.f && (half ? vhi : vlo);
-                v[half][cs] = use ? c * rv[k][x] : 0.f;
-            }
-        }
-        const unsigned afr[4] = {pack2<F16>(v[0][0], v[0][1]), pack2<F16>(v[1][0], v[1][1]),
-                                 pack2<F16>(v[0][2], v[0][3]), pack2<F16>(v[1][2], v[1][3])};
+        const float w = a.r.w[k];
+        const float clo = fmaf(blo, w, alo), chi = fmaf(bhi, w, ahi);
+        const float2 v0 = *reinterpret_cast<const float2*>(&rv[k][2 * c4]);
+        const float2 v8 = *reinterpret_cast<const float2*>(&rv[k][2 * c4 + 8]);
+        const unsigned afr[4] = {pack2<F16>(clo * v0.x, chi * v0.y), 0u,
+                                 pack2<F16>(m2 * w * v8.x, 0.f), pack2<F16>(clo * v8.x, chi * v8.y)};
         const int xrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {

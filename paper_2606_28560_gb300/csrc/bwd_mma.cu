@@ -179,11 +179,20 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         if (vhi) a.Delta[rowbase + qhi] = dlt_hi;
     }
 
-    // Columns of the rung slab: row r's far row is x = r, its floor row x = r+1;
-    // columns 2c4 + {0,1} of each 8-column n-tile belong to this thread.
-    const int xf_lo = g4, xl_lo = g4 + 1, xf_hi = g4 + 8, xl_hi = g4 + 9;
-    const bool own_f_lo = ((xf_lo & 7) >> 1) == c4, own_l_lo = ((xl_lo & 7) >> 1) == c4;
-    const bool own_f_hi = ((xf_hi & 7) >> 1) == c4, own_l_hi = ((xl_hi & 7) >> 1) == c4 && xl_hi < 16;
+    // Columns of a rung slab: row r's far row is x = r (weight w), its floor
+    // row x = r+1 (weight 1-w).  Of this thread's accumulator and A-fragment
+    // entries (rows g4, g4+8; columns 2c4, 2c4+1 and 2c4+8, 2c4+9) only those
+    // with x - r in {-1, 0, 1} can be either, a pattern fixed by
+    // delta = 2c4 - g4: entries (g4, 2c4 + u) and (g4+8, 2c4+8 + u) take the
+    // interpolation weights  u=0: w if delta = 0, 1-w if delta = 1;
+    //                        u=1: w if delta = -1, 1-w if delta = 0,
+    // each weight of the form A + B w; the far-minus-floor difference takes
+    // +1 / -1 at the same places.  Row g4 = 7 also has its floor at column 8.
+    const int dl = 2 * c4 - g4;
+    const float ia0 = dl == 1 ? 1.f : 0.f, ib0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f);
+    const float ia1 = dl == 0 ? 1.f : 0.f, ib1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
+    const float df0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f), df1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
+    const float m7 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
 
     __syncthreads();                              // barrier init visible
     const bool ok_v = mbar_wait(&bars[0], 0);
@@ -221,19 +230,14 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 mma_bf16_16816(dt[t], da[kc + 1], b2, b3);
             }
         }
-        const float f_lo = (xf_lo & 1) ? dt[0][1] : dt[0][0];
-        const float l_lo0 = (xl_lo & 1) ? dt[0][1] : dt[0][0];
-        const float l_lo1 = (xl_lo & 1) ? dt[1][1] : dt[1][0];
-        const float l_lo = (xl_lo >> 3) ? l_lo1 : l_lo0;
-        const float f_hi = (xf_hi & 1) ? dt[1][3] : dt[1][2];
-        const float l_hi = (xl_hi & 1) ? dt[1][3] : dt[1][2];
-        const float d1_lo = quad_sum(own_f_lo ? f_lo : 0.f), d0_lo = quad_sum(own_l_lo ? l_lo : 0.f);
-        const float d1_hi = quad_sum(own_f_hi ? f_hi : 0.f), d0_hi = quad_sum(own_l_hi ? l_hi : 0.f);
+        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+        const float dp_lo = quad_sum(fmaf(c0, dt[0][0], fmaf(c1, dt[0][1], c7 * dt[1][0])));
+        const float ddp_lo = quad_sum(fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0])));
+        const float dp_hi = quad_sum(fmaf(c0, dt[1][2], c1 * dt[1][3]));
+        const float ddp_hi = quad_sum(fmaf(df0, dt[1][2], df1 * dt[1][3]));
         if (c4 == 0) {
-            dps[warp][k][g4][0] = w1 * d0_lo + w * d1_lo;
-            dps[warp][k][g4][1] = d1_lo - d0_lo;
-            dps[warp][k][g4 + 8][0] = w1 * d0_hi + w * d1_hi;
-            dps[warp][k][g4 + 8][1] = d1_hi - d0_hi;
+            *reinterpret_cast<float2*>(dps[warp][k][g4]) = make_float2(dp_lo, ddp_lo);
+            *reinterpret_cast<float2*>(dps[warp][k][g4 + 8]) = make_float2(dp_hi, ddp_hi);
         }
     }
 
@@ -345,20 +349,19 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 mma_f16_16816(st[t], qa[kc + 1], b2, b3);
             }
         }
-        const float f_lo = (xf_lo & 1) ? st[0][1] : st[0][0];
-        const float l_lo0 = (xl_lo & 1) ? st[0][1] : st[0][0];
-        const float l_lo1 = (xl_lo & 1) ? st[1][1] : st[1][0];
-        const float l_lo = (xl_lo >> 3) ? l_lo1 : l_lo0;
-        const float f_hi = (xf_hi & 1) ? st[1][3] : st[1][2];
-        const float l_hi = (xl_hi & 1) ? st[1][3] : st[1][2];
-        const float s1_lo = quad_sum(own_f_lo ? f_lo : 0.f), s0_lo = quad_sum(own_l_lo ? l_lo : 0.f);
-        const float s1_hi = quad_sum(own_f_hi ? f_hi : 0.f), s0_hi = quad_sum(own_l_hi ? l_hi : 0.f);
+        // interpolated score and far-minus-floor raw score of rows g4, g4+8
+        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+        const float si_lo = quad_sum(fmaf(c0, st[0][0], fmaf(c1, st[0][1], c7 * st[1][0])));
+        const float sd_lo = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
+        const float si_hi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3]));
+        const float sd_hi = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
         const float dk = a.r.d[k];
         const bool okl = vlo && dk <= (float)qlo, okh = vhi && dk <= (float)qhi;
-        const float dp_lo = dps[warp][k][g4][0], ddp_lo = dps[warp][k][g4][1];
-        const float dp_hi = dps[warp][k][g4 + 8][0], ddp_hi = dps[warp][k][g4 + 8][1];
-        const float p_lo = okl ? exp2f((w1 * s0_lo + w * s1_lo) * sc2 - lse2_lo) : 0.f;
-        const float p_hi = okh ? exp2f((w1 * s0_hi + w * s1_hi) * sc2 - lse2_hi) : 0.f;
+        const float2 dpl = *reinterpret_cast<const float2*>(dps[warp][k][g4]);
+        const float2 dph = *reinterpret_cast<const float2*>(dps[warp][k][g4 + 8]);
+        const float dp_lo = dpl.x, ddp_lo = dpl.y, dp_hi = dph.x, ddp_hi = dph.y;
+        const float p_lo = okl ? exp2f(si_lo * sc2 - lse2_lo) : 0.f;
+        const float p_hi = okh ? exp2f(si_hi * sc2 - lse2_hi) : 0.f;
         const float e_lo = dp_lo - dlt_lo, e_hi = dp_hi - dlt_hi;
         const float ds_lo = p_lo * e_lo, ds_hi = p_hi * e_hi;
         if (c4 == 0) {
@@ -368,30 +371,15 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         // dL/dd_k of this warp's rows, in a fixed order over the rows
         float g = 0.f;
         if (c4 == 0)
-            g = p_lo * fmaf(s.scale * (s1_lo - s0_lo), e_lo, ddp_lo) +
-                p_hi * fmaf(s.scale * (s1_hi - s0_hi), e_hi, ddp_hi);
+            g = p_lo * fmaf(s.scale * sd_lo, e_lo, ddp_lo) + p_hi * fmaf(s.scale * sd_hi, e_hi, ddp_hi);
         g += __shfl_xor_sync(0xffffffffu, g, 4);
         g += __shfl_xor_sync(0xffffffffu, g, 8);
         g += __shfl_xor_sync(0xffffffffu, g, 16);
         if (lane == 0) gsm[warp][k] = g;
 
-        // dShat_k as fp16 A fragment: columns 2c4 + {0,1} (a0, a1) and 2c4 + 8 + {0,1} (a2, a3)
-        unsigned afr[4];
-#pragma unroll
-        for (int cs = 0; cs < 4; cs += 2) {
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                const int r = g4 + 8 * half;
-                const float d = half ? ds_hi : ds_lo;
-                float e2[2];
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    const int x = 2 * c4 + u + 8 * (cs >> 1);
-                    e2[u] = (x == r) ? d * w : ((x == r + 1) ? d * w1 : 0.f);
-                }
-                afr[(cs >> 1) * 2 + half] = pack_f16(e2[0], e2[1]);
-            }
-        }
+        // dShat_k as fp16 A fragment: the interpolation weights times dS of the row
+        const unsigned afr[4] = {pack_f16(c0 * ds_lo, c1 * ds_lo), 0u, pack_f16(c7 * ds_lo, 0.f),
+                                 pack_f16(c0 * ds_hi, c1 * ds_hi)};
         const int krow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {

@@ -173,11 +173,18 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     mhi = quad_max(mhi);
 
     // ---- rung scores: slab rows x = 0..15 at absolute bw - s0 - 1 + x.
-    // Row r's far score is column x = r, its floor score column x = r + 1.
-    // Columns 2c4 + {0,1} of n-tile t belong to this thread.
-    const int xf_lo = g4, xl_lo = g4 + 1, xf_hi = g4 + 8, xl_hi = g4 + 9;
-    const bool own_f_lo = ((xf_lo & 7) >> 1) == c4, own_l_lo = ((xl_lo & 7) >> 1) == c4;
-    const bool own_f_hi = ((xf_hi & 7) >> 1) == c4, own_l_hi = ((xl_hi & 7) >> 1) == c4 && xl_hi < 16;
+    // Row r's far score is column x = r (weight w), its floor score column
+    // x = r + 1 (weight 1-w).  Of this thread's entries (rows g4, g4+8; columns
+    // 2c4, 2c4+1 and 2c4+8, 2c4+9) only those with x - r in {-1, 0, 1} can be
+    // either, a pattern fixed by delta = 2c4 - g4: entries (g4, 2c4 + u) and
+    // (g4+8, 2c4+8 + u) take  u=0: w if delta = 0, 1-w if delta = 1;
+    //                         u=1: w if delta = -1, 1-w if delta = 0,
+    // each of the form A + B w; row g4 = 7 also has its floor at column 8.
+    // The same weights place p in the A fragment of the value product.
+    const int dl = 2 * c4 - g4;
+    const float ia0 = dl == 1 ? 1.f : 0.f, ib0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f);
+    const float ia1 = dl == 0 ? 1.f : 0.f, ib1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
+    const float m7 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
     float rs[kMmaMaxRungs][2];
 #pragma unroll
     for (int k = 0; k < kMmaMaxRungs; ++k) { rs[k][0] = -INFINITY; rs[k][1] = -INFINITY; }
@@ -199,21 +206,9 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
                 mma_f16_16816(st[t], qa[kc + 1], b2, b3);
             }
         }
-        // element of (row half, column x): n-tile x >> 3, register 2*half + (x & 1)
-        float plo = 0.f, phi = 0.f;
-        {
-            // row lo: far column g4 lies in n-tile 0; floor column g4+1 in n-tile (g4+1)>>3
-            const float f_lo = (xf_lo & 1) ? st[0][1] : st[0][0];
-            const float l_lo0 = (xl_lo & 1) ? st[0][1] : st[0][0];
-            const float l_lo1 = (xl_lo & 1) ? st[1][1] : st[1][0];
-            const float l_lo = (xl_lo >> 3) ? l_lo1 : l_lo0;
-            const float f_hi = (xf_hi & 1) ? st[1][3] : st[1][2];
-            const float l_hi = (xl_hi & 1) ? st[1][3] : st[1][2];
-            plo = (own_f_lo ? w * f_lo : 0.f) + (own_l_lo ? w1 * l_lo : 0.f);
-            phi = (own_f_hi ? w * f_hi : 0.f) + (own_l_hi ? w1 * l_hi : 0.f);
-        }
-        plo = quad_sum(plo) * sc2;
-        phi = quad_sum(phi) * sc2;
+        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+        const float plo = quad_sum(fmaf(c0, st[0][0], fmaf(c1, st[0][1], c7 * st[1][0]))) * sc2;
+        const float phi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3])) * sc2;
         const float dk = a.r.d[k];
         rs[k][0] = (vlo && dk <= (float)qlo) ? plo : -INFINITY;
         rs[k][1] = (vhi && dk <= (float)qhi) ? phi : -INFINITY;
@@ -286,28 +281,14 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         const float plo = exp2f(rs[k][0] - mlo), phi = exp2f(rs[k][1] - mhi);   // 0 when masked
         llo += plo;
         lhi += phi;
-        float ev[2][4];                           // [row half][column slot]
-#pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            const int r = g4 + 8 * half;
-            const float p = half ? phi : plo;
-#pragma unroll
-            for (int cs = 0; cs < 4; ++cs) {
-                const int x = 2 * c4 + (cs & 1) + 8 * (cs >> 1);
-                ev[half][cs] = (x == r) ? p * w : ((x == r + 1) ? p * w1 : 0.f);
-            }
-        }
-        unsigned ahi[4], alo[4];
-#pragma unroll
-        for (int cs = 0; cs < 4; cs += 2) {
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                const float e0 = ev[half][cs], e1 = ev[half][cs + 1];
-                const float h0 = bf16_round(e0), h1 = bf16_round(e1);
-                ahi[(cs >> 1) * 2 + half] = pack_bf16(h0, h1);
-                alo[(cs >> 1) * 2 + half] = pack_bf16(e0 - h0, e1 - h1);
-            }
-        }
+        // Phat as bf16 hi + lo A fragments (a1, row g4+8 at columns 2c4.., is zero)
+        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+        const float e00 = c0 * plo, e01 = c1 * plo, e20 = c7 * plo, e30 = c0 * phi, e31 = c1 * phi;
+        const float h00 = bf16_round(e00), h01 = bf16_round(e01), h20 = bf16_round(e20);
+        const float h30 = bf16_round(e30), h31 = bf16_round(e31);
+        const unsigned ahi[4] = {pack_bf16(h00, h01), 0u, pack_bf16(h20, 0.f), pack_bf16(h30, h31)};
+        const unsigned alo[4] = {pack_bf16(e00 - h00, e01 - h01), 0u, pack_bf16(e20 - h20, 0.f),
+                                 pack_bf16(e30 - h30, e31 - h31)};
         const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
