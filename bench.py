@@ -201,7 +201,6 @@ def algorithmic_bytes():
         # Q, dO, O, K~, V read; dQ, Q~ written; lse read, Delta written; P/dp written
         "bwd_query_mma": 7 * rows + 2 * 4 * n + 2 * 4 * n * S,
         "bwd_key": 4 * rows + 2 * 4 * n * S,               # Q~ dO read, dK dV written, P/dS read
-        "bwd_finalize": 0,
     }
 
 

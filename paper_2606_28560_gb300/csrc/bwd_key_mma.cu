@@ -51,16 +51,17 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
                                          bool vhi, unsigned long long* bar, unsigned parity, bool& ok,
                                          float (*rv)[16]) {
     const Shape& s = a.s;
-    // ---- rung values of the warp's 16 slab columns, all rungs at once (the
-    // loads are independent, so their latencies overlap): rv[k][x] = p or dS of
-    // query bw + s0_k + x, rung slot k (0 past the end of the sequence)
+    // ---- rung values of the warp's 16 slab columns, all active rungs at once
+    // (the loads are independent, so their latencies overlap): rv[i][x] = p or
+    // dS of query bw + s0 + x for active rung i in increasing d (0 past the end
+    // of the sequence and for the padding entries)
 #pragma unroll
-    for (int i = 0; i < kMmaMaxRungs * 16 / 32; ++i) {
-        const int u = lane + 32 * i;
-        const int k = u >> 4, x = u & 15;
-        const int q = bw + a.r.s0[k] + x;
-        const bool use = k < a.r.K && ((a.r.active >> k) & 1u) && q < s.T;
-        rv[k][x] = use ? X[(size_t)(s.W + 1 + k) * s.T + q] : 0.f;
+    for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
+        const int u = lane + 32 * j;
+        const int i = u >> 4, x = u & 15;
+        const int q = bw + L.act_s0[i] + x;
+        const bool use = i < L.n_act && q < s.T;
+        rv[i][x] = use ? X[(size_t)(s.W + 1 + L.act_k[i]) * s.T + q] : 0.f;
     }
     __syncwarp();
     // ---- window band values (loaded while the copies are in flight)
@@ -122,24 +123,30 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
     const float alo = dl == 0 ? 1.f : 0.f, blo = dl == 0 ? -1.f : (dl == 1 ? 1.f : 0.f);
     const float ahi = dl == -1 ? 1.f : 0.f, bhi = dl == -1 ? -1.f : (dl == 0 ? 1.f : 0.f);
     const float m2 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
+    // Rungs whose slab starts before the end of the sequence: a prefix of the
+    // list.  Two per iteration (independent work to overlap); an odd count
+    // runs one padding entry, whose values are zero.
+    int n_use = 0;
+    while (n_use < L.n_act && bw + L.act_s0[n_use] < s.T) ++n_use;
 #pragma unroll 1
-    for (int k = 0; k < a.r.K; ++k) {
-        if (!((a.r.active >> k) & 1u)) continue;
-        const int s0 = a.r.s0[k];
-        if (bw + s0 >= s.T) continue;                      // every query of the slab is past the end
-        const float w = a.r.w[k];
-        const float clo = fmaf(blo, w, alo), chi = fmaf(bhi, w, ahi);
-        const float2 v0 = *reinterpret_cast<const float2*>(&rv[k][2 * c4]);
-        const float2 v8 = *reinterpret_cast<const float2*>(&rv[k][2 * c4 + 8]);
-        const unsigned afr[4] = {pack2<F16>(clo * v0.x, chi * v0.y), 0u,
-                                 pack2<F16>(m2 * w * v8.x, 0.f), pack2<F16>(clo * v8.x, chi * v8.y)};
-        const int xrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+    for (int i = 0; i < n_use; i += 2) {
 #pragma unroll
-        for (int n = 0; n < 8; n += 2) {
-            unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
-            mma16816<F16>(acc[n], afr, b0, b1);
-            mma16816<F16>(acc[n + 1], afr, b2, b3);
+        for (int u = 0; u < 2; ++u) {
+            const int ii = i + u;
+            const float w = L.act_w[ii];
+            const float clo = fmaf(blo, w, alo), chi = fmaf(bhi, w, ahi);
+            const float2 v0 = *reinterpret_cast<const float2*>(&rv[ii][2 * c4]);
+            const float2 v8 = *reinterpret_cast<const float2*>(&rv[ii][2 * c4 + 8]);
+            const unsigned afr[4] = {pack2<F16>(clo * v0.x, chi * v0.y), 0u,
+                                     pack2<F16>(m2 * w * v8.x, 0.f), pack2<F16>(clo * v8.x, chi * v8.y)};
+            const int xrow = L.act_smem[ii] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+            for (int n = 0; n < 8; n += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
+                mma16816<F16>(acc[n], afr, b0, b1);
+                mma16816<F16>(acc[n + 1], afr, b2, b3);
+            }
         }
     }
 }
@@ -151,6 +158,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bar;
     __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
+    __shared__ float red[kMmaMaxRungs];                   // block 0: dL/dd_k
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const unsigned sbase = smem_u32(buf);
 
@@ -172,6 +180,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     __syncthreads();
+    if (blockIdx.x == 0) convert_rung_sums(a, red);
 
     unsigned parity = 0;
     bool ok = true;
@@ -245,7 +254,7 @@ cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, co
 
 }  // namespace
 
-size_t bwd_key_mma_static_smem() { return sizeof(float) * kWarps * kMmaMaxRungs * 16 + 64; }
+size_t bwd_key_mma_static_smem() { return sizeof(float) * (kWarps * kMmaMaxRungs * 16 + kMmaMaxRungs) + 64; }
 
 int bwd_key_mma_blocks(const Shape& s) {
     const long long tiles = (s.T + kMmaTile - 1) / kMmaTile;

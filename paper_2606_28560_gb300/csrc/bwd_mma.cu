@@ -418,13 +418,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 
     // ---- per-CTA rung partials, warps summed in a fixed order
     __syncthreads();
-    if (tid < a.r.K) {
-        float x = 0.f;
-        if ((a.r.active >> tid) & 1u)
-            for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
-        a.partial[(size_t)tid * a.nblocks_a + blockIdx.x] = x;
-    }
-    if (blockIdx.x == 0 && tid == 0) *a.ticket = 0u;
+    float x = 0.f;
+    if (tid < a.r.K && ((a.r.active >> tid) & 1u))
+        for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
+    add_rung_partials(a, x);
 }
 
 template <int NT>

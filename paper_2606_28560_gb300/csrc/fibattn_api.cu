@@ -115,26 +115,20 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
 }
 
 struct BwdLayout {
-    size_t qt, kt, P, DP, Delta, partial, colsum, ticket, total;
-    int nblocks;
+    size_t qt, kt, P, DP, Delta, racc, total;
 };
 
 BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype) {
     BwdLayout L;
     size_t es = rot_size(dtype);
     size_t S = (size_t)W + 1 + K;
-    Shape s; s.B = B; s.H = H; s.Hkv = Hkv; s.T = T; s.W = W; s.G = H / Hkv; s.scale = 1.f;
-    L.nblocks = bwd_simple_blocks(s);               // rows of partial: the larger of the two query passes
-    if (bwd_mma_blocks(s) > L.nblocks) L.nblocks = bwd_mma_blocks(s);
     size_t off = 0;
     L.qt = off; off += align256((size_t)B * H * T * kHeadDim * es);
     L.kt = off; off += align256((size_t)B * Hkv * T * kHeadDim * es);
     L.P = off; off += align256((size_t)B * H * T * S * 4);
     L.DP = off; off += align256((size_t)B * H * T * S * 4);
     L.Delta = off; off += align256((size_t)B * H * T * 4);
-    L.partial = off; off += align256((size_t)(L.nblocks > 0 ? L.nblocks : 1) * kMaxRungs * 4);
-    L.colsum = off; off += align256((size_t)kMaxRungs * 8);
-    L.ticket = off; off += 256;
+    L.racc = off; off += align256((size_t)kMaxRungs * 8);       // fixed-point rung sums
     L.total = off;
     return L;
 }
@@ -383,10 +377,7 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     a.qt = ws + L.qt; a.kt = ws + L.kt;
     a.P = reinterpret_cast<float*>(ws + L.P); a.DP = reinterpret_cast<float*>(ws + L.DP);
     a.Delta = reinterpret_cast<float*>(ws + L.Delta);
-    a.partial = reinterpret_cast<float*>(ws + L.partial);
-    a.colsum = reinterpret_cast<double*>(ws + L.colsum);
-    a.ticket = reinterpret_cast<unsigned*>(ws + L.ticket);
-    a.nblocks_a = B > 0 ? L.nblocks : 0;
+    a.racc = reinterpret_cast<unsigned long long*>(ws + L.racc);
     a.S = W + 1 + K;
     a.alpha = alpha;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -401,7 +392,6 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     if (o.bwd_kernel == 2 && !mma_ok)
         return fail(FIBATTN_ERR_UNSUPPORTED, "tensor-core backward needs bf16, out, W <= 16, K <= 16 and a staged row "
                                              "union that fits shared memory");
-    if (mma_ok) a.nblocks_a = B > 0 ? bwd_mma_blocks(a.s) : 0;
     cudaError_t e;
     if (B > 0) {
         if (!mma_ok) {
@@ -411,7 +401,8 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         }
         {
             ProfScope p("rope_k", st);
-            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st,
+                                 reinterpret_cast<unsigned*>(a.racc), 2 * kMaxRungs);
         }
         if (e != cudaSuccess) return cuda_fail(e, "rope prologue (k) launch");
         if (mma_ok) {
@@ -437,12 +428,7 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         if (e != cudaSuccess) return cuda_fail(e, "zero gradients for an empty batch");
         return FIBATTN_OK;
     }
-    {
-        ProfScope p("bwd_finalize", st);
-        e = launch_bwd_finalize(a, st);
-    }
-    if (e != cudaSuccess) return cuda_fail(e, "backward finalize launch");
-    return FIBATTN_OK;
+    return FIBATTN_OK;                           // dtheta and dd: written by block 0 of the key pass
 }
 
 }  // extern "C"

@@ -71,10 +71,8 @@ struct BwdArgs {
     float* Delta;             // sum_slots p dL/dp per query [B,H,T]
     float* Ps;                // tensor-core path, slot-major [B,H,S,T]: p      (P region)
     float* DSs;               //                                      dS = p (dp - Delta)  (DP region)
-    float* partial;           // per-block dL/dd_k partial sums [kMaxRungs][nblocks]
-    double* colsum;           // dL/dd_k column sums [kMaxRungs]
-    unsigned* ticket;         // finalize completion counter (reset by the query pass)
-    int nblocks_a;            // number of query-centric blocks (rows of partial)
+    unsigned long long* racc; // dL/dd_k as 2^-32 fixed point [kMaxRungs] (zeroed by the launch before
+                              // the query pass)
     int S;                    // slots per query = W + 1 + K
     float alpha;
     Shape s;
@@ -191,14 +189,47 @@ __device__ __forceinline__ void rope_chunk(const RopeParams& rp, int pos, int c,
     }
 }
 
+// ------------------------------------------------- rung-gradient reduction --
+
+// dL/dd_k accumulates the query blocks' partial sums as 64-bit fixed point
+// (2^-32 units): integer addition is exact and order-free, so the result does
+// not depend on which block finishes first.  The query pass adds each block's
+// partials (threads k < K hold rung k's; the accumulators are zeroed by the
+// launch before the pass); block 0 of the key pass, which starts after the
+// query pass has completed, converts them and applies the chain rule
+// dL/dalpha = sum_k f_k dL/dd_k, dL/dtheta = dL/dalpha (alpha - 0.5)(1.5 - alpha),
+// alpha = 0.5 + sigmoid(theta).
+__device__ __forceinline__ void add_rung_partials(const BwdArgs& a, float partial) {
+    if ((int)threadIdx.x < a.r.K)
+        atomicAdd(a.racc + threadIdx.x, (unsigned long long)__float2ll_rn(partial * 4294967296.0f));
+}
+
+// Called by every thread of block 0 of the key pass.  red: shared scratch of
+// at least K floats.
+__device__ __forceinline__ void convert_rung_sums(const BwdArgs& a, float* red) {
+    const int t = threadIdx.x;
+    if (t < a.r.K) {
+        const float v = (float)((double)(long long)__ldcg(a.racc + t) * 2.3283064365386962890625e-10);
+        red[t] = v;
+        if (a.dd) a.dd[t] = v;
+    }
+    __syncthreads();
+    if (t == 0) {
+        float da = 0.f;
+        for (int k = 0; k < a.r.K; ++k) da += a.r.f[k] * red[k];
+        *a.dtheta = da * (a.alpha - 0.5f) * (1.5f - a.alpha);
+    }
+}
+
 // ----------------------------------------------------------- launchers ----
 
+// zero / nzero (may be null / 0): device words the launch sets to 0 (the
+// rung accumulators of the query pass that follows it).
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
-                             bool bf16, cudaStream_t st);
+                             bool bf16, cudaStream_t st, unsigned* zero = nullptr, int nzero = 0);
 cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_query(const BwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st);
-cudaError_t launch_bwd_finalize(const BwdArgs& a, cudaStream_t st);
 int bwd_simple_blocks(const Shape& s);
 
 // Records a message for fibattn_last_error() and returns `code`.

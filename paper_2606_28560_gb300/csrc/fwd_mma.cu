@@ -395,6 +395,25 @@ int smem_row_of(const MmaLayout& L, int rel) {
     return -1;
 }
 
+// Active rungs sorted by d (ties by index), with their shared rows.
+void active_list(const RungParams& r, MmaLayout* L) {
+    L->n_act = 0;
+    for (int i = 0; i < kMmaMaxRungs; ++i) {
+        L->act_k[i] = 0; L->act_s0[i] = 0; L->act_smem[i] = 0; L->act_w[i] = 0.f; L->act_d[i] = 3.0e38f;
+    }
+    for (int k = 0; k < r.K; ++k) {
+        if (!((r.active >> k) & 1u)) continue;
+        int i = L->n_act++;
+        while (i > 0 && L->act_d[i - 1] > r.d[k]) {
+            L->act_k[i] = L->act_k[i - 1]; L->act_s0[i] = L->act_s0[i - 1]; L->act_smem[i] = L->act_smem[i - 1];
+            L->act_w[i] = L->act_w[i - 1]; L->act_d[i] = L->act_d[i - 1];
+            --i;
+        }
+        L->act_k[i] = k; L->act_s0[i] = r.s0[k]; L->act_smem[i] = L->rung_smem[k];
+        L->act_w[i] = r.w[k]; L->act_d[i] = r.d[k];
+    }
+}
+
 void rope_steps(double rope_base, MmaLayout* L) {
     for (int m = 0; m < kHalf; ++m) {
         const double theta = std::pow(rope_base, -2.0 * m / (double)kHeadDim);
@@ -422,6 +441,7 @@ bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, siz
     for (int k = 0; k < kMmaMaxRungs; ++k) L->rung_smem[k] = 0;
     for (int k = 0; k < r.K; ++k)
         if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row_of(*L, -r.s0[k] - 1);
+    active_list(r, L);
     return fwd_mma_smem_bytes(*L) <= smem_limit;
 }
 
@@ -444,6 +464,7 @@ bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, siz
     for (int k = 0; k < kMmaMaxRungs; ++k) L->rung_smem[k] = 0;
     for (int k = 0; k < r.K; ++k)
         if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row_of(*L, r.s0[k]);
+    active_list(r, L);
     return fwd_mma_smem_bytes(*L) <= smem_limit;
 }
 

@@ -24,6 +24,14 @@ struct MmaLayout {
     int rung_smem[kMmaMaxRungs];                  // shared row of relative row -s0_k - 1
     float rope_c8[kHalf];                         // cos, sin of 8 position steps of pair m
     float rope_s8[kHalf];
+    // The active rungs in increasing d (so the rungs a tile can use form a
+    // prefix); entries n_act.. pad the list with zero weight and shared row 0.
+    int n_act;
+    int act_k[kMmaMaxRungs];
+    int act_s0[kMmaMaxRungs];
+    int act_smem[kMmaMaxRungs];
+    float act_w[kMmaMaxRungs];
+    float act_d[kMmaMaxRungs];
 };
 
 bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);

@@ -53,7 +53,9 @@ __device__ __forceinline__ void axpy16x2(float a, const float2* x, float2* y) {
 
 template <typename T, typename R>
 __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ src, R* __restrict__ dst,
-                                                        long long rows, int T_, RopeParams rp) {
+                                                        long long rows, int T_, RopeParams rp, unsigned* zero,
+                                                        int nzero) {
+    if (blockIdx.x == 0 && (int)threadIdx.x < nzero) zero[threadIdx.x] = 0u;
     // One (row, 8-pair chunk) item per thread per pass; grid-stride over items.
     const long long n = rows * 4;
     for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
@@ -297,16 +299,15 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
     if (c == 0) dsm[qloc] = qvalid ? delta : 0.f;
     __syncthreads();
     // per-block rung partials sum_i (t1 - Delta_i t2), queries in a fixed order
-    if (threadIdx.x < kMaxRungs) {
+    float x = 0.f;
+    if (threadIdx.x < a.r.K) {
         const int k = threadIdx.x;
-        float x = 0.f;
         for (int u = 0; u < kRowsPerBlock; ++u) {
             const bool valid = (blockIdx.x % tiles) * kRowsPerBlock + u < s.T;
             if (valid) x += tsm[u][k][0] - dsm[u] * tsm[u][k][1];
         }
-        a.partial[(size_t)k * a.nblocks_a + blockIdx.x] = x;
     }
-    if (blockIdx.x == 0 && threadIdx.x == 0) *a.ticket = 0u;
+    add_rung_partials(a, x);
 }
 
 // Key-centric pass.  Key row j of kv head hk receives, from every query head
@@ -316,6 +317,8 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
 // dS = P (dp - Delta_i) from the query pass.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
+    __shared__ float red[kMaxRungs];
+    if (blockIdx.x == 0) convert_rung_sums(a, red);
     const Shape s = a.s;
     const int c = threadIdx.x & 3;
     const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
@@ -385,74 +388,21 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
     }
 }
 
-// Fixed-order sum of the per-block rung partials, then the chain rule
-// dL/dalpha = sum_k f_k dL/dd_k and dL/dtheta = dL/dalpha (alpha-0.5)(1.5-alpha).
-// Block k sums column k: thread t adds rows t, t+256, ... in order with
-// compensated (Kahan) fp32 sums, then a fixed shared-memory tree combines the
-// 256 (sum, compensation) pairs, so the result does not depend on scheduling.
-// (fp64 arithmetic is avoided: it runs on a slow pipe on this part.)  The last
-// block to finish (ticket counter, no waiting) forms dL/dalpha and dL/dtheta
-// from the K column sums and resets the ticket for the next call.
-constexpr int kFinThreads = 256;
-__global__ void __launch_bounds__(kFinThreads) bwd_finalize_kernel(BwdArgs a) {
-    __shared__ float red[kFinThreads], cmp[kFinThreads];
-    __shared__ bool last;
-    const int t = threadIdx.x, k = blockIdx.x;
-    const float* col = a.partial + (size_t)k * a.nblocks_a;
-    float sum = 0.f, c = 0.f;
-    for (int blk = t; blk < a.nblocks_a; blk += kFinThreads) {
-        const float y = col[blk] - c;
-        const float tt = sum + y;
-        c = (tt - sum) - y;
-        sum = tt;
-    }
-    red[t] = sum;
-    cmp[t] = c;
-    __syncthreads();
-    for (int w = kFinThreads / 2; w > 0; w >>= 1) {
-        if (t < w) {
-            const float y = red[t + w] - (cmp[t] + cmp[t + w]);
-            const float tt = red[t] + y;
-            cmp[t] = (tt - red[t]) - y;
-            red[t] = tt;
-        }
-        __syncthreads();
-    }
-    if (t == 0) {
-        a.colsum[k] = (double)red[0];
-        if (a.dd) a.dd[k] = red[0];
-        __threadfence();
-        last = atomicAdd(a.ticket, 1u) == (unsigned)(gridDim.x - 1);
-    }
-    __syncthreads();
-    if (last) {                                  // block-uniform
-        __threadfence();
-        // every column sum is now visible; load them in parallel, sum in order
-        if (t < a.r.K) red[t] = a.r.f[t] * (float)__ldcg(a.colsum + t);
-        __syncthreads();
-        if (t == 0) {
-            float da = 0.f;
-            for (int u = 0; u < a.r.K; ++u) da += red[u];
-            *a.dtheta = da * (a.alpha - 0.5f) * (1.5f - a.alpha);
-            *a.ticket = 0u;
-        }
-    }
-}
-
 }  // namespace
 
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
-                             bool bf16, cudaStream_t st) {
+                             bool bf16, cudaStream_t st, unsigned* zero, int nzero) {
+    if (nzero > 256) return cudaErrorInvalidValue;
     if (rows <= 0) return cudaSuccess;
     const long long items = rows * 4;
     long long grid = (items + 255) / 256;
     if (grid > 152 * 16) grid = 152 * 16;       // 16 resident 256-thread blocks on each of 152 SMs
     if (bf16)
         rope_rows_kernel<__nv_bfloat16, __half><<<(unsigned)grid, 256, 0, st>>>(
-            reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp);
+            reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp, zero, nzero);
     else
         rope_rows_kernel<float, float><<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const float*>(src),
-                                                              reinterpret_cast<float*>(dst), rows, T, rp);
+                                                              reinterpret_cast<float*>(dst), rows, T, rp, zero, nzero);
     return cudaGetLastError();
 }
 
@@ -485,15 +435,6 @@ cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st) {
     if (gk <= 0) return cudaSuccess;
     if (bf16) bwd_key_kernel<__nv_bfloat16><<<(unsigned)gk, kThreads, 0, st>>>(a);
     else bwd_key_kernel<float><<<(unsigned)gk, kThreads, 0, st>>>(a);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_bwd_finalize(const BwdArgs& a, cudaStream_t st) {
-    if (a.r.K == 0) {                            // no rungs: dL/dtheta = 0
-        cudaError_t e = cudaMemsetAsync(a.dtheta, 0, sizeof(float), st);
-        return e != cudaSuccess ? e : cudaGetLastError();
-    }
-    bwd_finalize_kernel<<<a.r.K, kFinThreads, 0, st>>>(a);
     return cudaGetLastError();
 }
 
