@@ -155,6 +155,7 @@ template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ RowMaps tmG, BwdArgs a,
                    MmaLayout L) {
+    grid_dependency_sync();
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bar;
     __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
@@ -248,8 +249,7 @@ cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, co
     auto kern = bwd_key_mma_kernel<NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kWarps * 32, smem, st>>>(mq, mg, a, L);
-    return cudaGetLastError();
+    return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mq, mg, a, L);
 }
 
 }  // namespace

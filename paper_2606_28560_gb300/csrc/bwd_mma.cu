@@ -45,6 +45,7 @@ template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                      BwdArgs a, MmaLayout L) {
+    grid_dependency_sync();
     constexpr int Wp = NT * 8 - 16;
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[2];
@@ -430,8 +431,7 @@ cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const BwdArgs& a, co
     auto kern = bwd_query_mma_kernel<NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<grid, kWarps * 32, smem, st>>>(mk, mv, a, L);
-    return cudaGetLastError();
+    return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mk, mv, a, L);
 }
 
 }  // namespace

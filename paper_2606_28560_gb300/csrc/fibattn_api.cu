@@ -4,6 +4,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <cstdint>
 #include <mutex>
@@ -16,6 +17,16 @@
 #include "fwd_mma.cuh"
 
 using namespace fibattn;
+
+namespace fibattn {
+bool pdl_enabled() {
+    static const bool on = [] {
+        const char* v = std::getenv("FIBATTN_PDL");
+        return !(v && v[0] == '0');
+    }();
+    return on;
+}
+}  // namespace fibattn
 
 namespace {
 

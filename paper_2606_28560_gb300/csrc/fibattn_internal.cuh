@@ -221,6 +221,39 @@ __device__ __forceinline__ void convert_rung_sums(const BwdArgs& a, float* red) 
     }
 }
 
+// ------------------------------------------- programmatic dependent launch --
+
+// Every kernel starts with this, before its first global-memory access: it
+// waits until the previous kernel in the stream has completed and its writes
+// are visible (a no-op when the launch carries no programmatic dependency),
+// then lets the next kernel be scheduled, so that its blocks can become
+// resident and run up to their own wait while this grid's last blocks run.
+__device__ __forceinline__ void grid_dependency_sync() {
+    asm volatile("griddepcontrol.wait;\n" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+
+// Host: whether launches carry the programmatic-serialisation attribute
+// (environment FIBATTN_PDL=0 turns it off).
+bool pdl_enabled();
+
+template <typename... KArgs, typename... Args>
+cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st,
+                          Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = pdl_enabled() ? 1 : 0;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, kern, args...);
+    return e != cudaSuccess ? e : cudaGetLastError();
+}
+
 // ----------------------------------------------------------- launchers ----
 
 // zero / nzero (may be null / 0): device words the launch sets to 0 (the

@@ -119,6 +119,7 @@ __device__ __forceinline__ float group_transpose_sum(float* v, int lane) {
 
 template <typename T, int R>
 __global__ void __launch_bounds__(8 * kStagedM / R) fwd_staged_kernel(FwdArgs a, StageLayout L) {
+    grid_dependency_sync();
     using RT = typename RotOf<T>::type;
     constexpr int M = kStagedM;
     constexpr int QPW = 4 * R;                   // queries per warp
@@ -328,8 +329,7 @@ cudaError_t launch_fwd_staged(const FwdArgs& a, const StageLayout& L, bool bf16,
     auto kern = fwd_staged_kernel<__nv_bfloat16, R>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    kern<<<(unsigned)grid, threads, smem, st>>>(a, L);
-    return cudaGetLastError();
+    return launch_kernel(kern, dim3((unsigned)grid), dim3(threads), smem, st, a, L);
 }
 
 }  // namespace fibattn

@@ -55,6 +55,7 @@ template <typename T, typename R>
 __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ src, R* __restrict__ dst,
                                                         long long rows, int T_, RopeParams rp, unsigned* zero,
                                                         int nzero) {
+    grid_dependency_sync();
     if (blockIdx.x == 0 && (int)threadIdx.x < nzero) zero[threadIdx.x] = 0u;
     // One (row, 8-pair chunk) item per thread per pass; grid-stride over items.
     const long long n = rows * 4;
@@ -73,6 +74,7 @@ __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ sr
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) fwd_simple_kernel(FwdArgs a) {
+    grid_dependency_sync();
     const Shape s = a.s;
     const int lane = threadIdx.x & 31, c = lane & 3;
     const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
@@ -193,6 +195,7 @@ __global__ void __launch_bounds__(kThreads) fwd_simple_kernel(FwdArgs a) {
 // pass, which forms dL/dscore = P (dp - Delta).
 template <typename T>
 __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
+    grid_dependency_sync();
     __shared__ float tsm[kRowsPerBlock][kMaxRungs][2];   // per-query t1, t2 of each rung
     __shared__ float dsm[kRowsPerBlock];                 // per-query Delta (0 when i >= T)
     const Shape s = a.s;
@@ -317,6 +320,7 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
 // dS = P (dp - Delta_i) from the query pass.
 template <typename T>
 __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
+    grid_dependency_sync();
     __shared__ float red[kMaxRungs];
     if (blockIdx.x == 0) convert_rung_sums(a, red);
     const Shape s = a.s;
@@ -398,21 +402,19 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
     long long grid = (items + 255) / 256;
     if (grid > 152 * 16) grid = 152 * 16;       // 16 resident 256-thread blocks on each of 152 SMs
     if (bf16)
-        rope_rows_kernel<__nv_bfloat16, __half><<<(unsigned)grid, 256, 0, st>>>(
-            reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp, zero, nzero);
-    else
-        rope_rows_kernel<float, float><<<(unsigned)grid, 256, 0, st>>>(reinterpret_cast<const float*>(src),
-                                                              reinterpret_cast<float*>(dst), rows, T, rp, zero, nzero);
-    return cudaGetLastError();
+        return launch_kernel(rope_rows_kernel<__nv_bfloat16, __half>, dim3((unsigned)grid), dim3(256), 0, st,
+                             reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp,
+                             zero, nzero);
+    return launch_kernel(rope_rows_kernel<float, float>, dim3((unsigned)grid), dim3(256), 0, st,
+                         reinterpret_cast<const float*>(src), reinterpret_cast<float*>(dst), rows, T, rp, zero, nzero);
 }
 
 cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st) {
     const long long tiles = (a.s.T + kRowsPerBlock - 1) / kRowsPerBlock;
     const long long grid = tiles * a.s.B * a.s.H;
     if (grid <= 0) return cudaSuccess;
-    if (bf16) fwd_simple_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, st>>>(a);
-    else fwd_simple_kernel<float><<<(unsigned)grid, kThreads, 0, st>>>(a);
-    return cudaGetLastError();
+    if (bf16) return launch_kernel(fwd_simple_kernel<__nv_bfloat16>, dim3((unsigned)grid), dim3(kThreads), 0, st, a);
+    return launch_kernel(fwd_simple_kernel<float>, dim3((unsigned)grid), dim3(kThreads), 0, st, a);
 }
 
 int bwd_simple_blocks(const Shape& s) {
@@ -424,18 +426,16 @@ cudaError_t launch_bwd_query(const BwdArgs& a, bool bf16, cudaStream_t st) {
     const long long tiles = (a.s.T + kRowsPerBlock - 1) / kRowsPerBlock;
     const long long gq = tiles * a.s.B * a.s.H;
     if (gq <= 0) return cudaSuccess;
-    if (bf16) bwd_query_kernel<__nv_bfloat16><<<(unsigned)gq, kThreads, 0, st>>>(a);
-    else bwd_query_kernel<float><<<(unsigned)gq, kThreads, 0, st>>>(a);
-    return cudaGetLastError();
+    if (bf16) return launch_kernel(bwd_query_kernel<__nv_bfloat16>, dim3((unsigned)gq), dim3(kThreads), 0, st, a);
+    return launch_kernel(bwd_query_kernel<float>, dim3((unsigned)gq), dim3(kThreads), 0, st, a);
 }
 
 cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st) {
     const long long tiles = (a.s.T + kRowsPerBlock - 1) / kRowsPerBlock;
     const long long gk = tiles * a.s.B * a.s.Hkv;
     if (gk <= 0) return cudaSuccess;
-    if (bf16) bwd_key_kernel<__nv_bfloat16><<<(unsigned)gk, kThreads, 0, st>>>(a);
-    else bwd_key_kernel<float><<<(unsigned)gk, kThreads, 0, st>>>(a);
-    return cudaGetLastError();
+    if (bf16) return launch_kernel(bwd_key_kernel<__nv_bfloat16>, dim3((unsigned)gk), dim3(kThreads), 0, st, a);
+    return launch_kernel(bwd_key_kernel<float>, dim3((unsigned)gk), dim3(kThreads), 0, st, a);
 }
 
 }  // namespace fibattn
