@@ -212,8 +212,29 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
         }
         const float sc = ok ? (pass ? s.scale : 1.f) : __int_as_float(0x7fc00000);
         __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(pass ? a.dk : a.dv) + krow0 * kHeadDim;
+        // dk = R(-theta key) dk~: cos, sin of pair m = 8n + 2c4 + u (m + 32 in
+        // n-tile n + 4) at klo, advanced by 8 positions for khi
+        float ec[4][2], es[4][2];
+        if (pass) {
+#pragma unroll
+            for (int n = 0; n < 4; ++n)
+#pragma unroll
+                for (int u = 0; u < 2; ++u) rope_cs(a.rope, 8 * n + 2 * c4 + u, klo, ec[n][u], es[n][u]);
+        }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
+            if (pass && half == 1) {
+#pragma unroll
+                for (int n = 0; n < 4; ++n)
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const int m = 8 * n + 2 * c4 + u;
+                        const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                        const float cn = ec[n][u] * c8 - es[n][u] * s8;
+                        es[n][u] = es[n][u] * c8 + ec[n][u] * s8;
+                        ec[n][u] = cn;
+                    }
+            }
             if (!(half ? vhi : vlo)) continue;
             const int key = half ? khi : klo;
 #pragma unroll
@@ -221,17 +242,14 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
                 acc[n][2 * half] *= sc;
                 acc[n][2 * half + 1] *= sc;
             }
-            if (pass) {                                   // dk = R(-theta key) dk~
+            if (pass) {
 #pragma unroll
                 for (int n = 0; n < 4; ++n) {
 #pragma unroll
                     for (int u = 0; u < 2; ++u) {
-                        const int m = 8 * n + 2 * c4 + u;     // pair (m, m + 32): n-tiles n and n + 4
-                        float c, sn;
-                        rope_cs(a.rope, m, key, c, sn);
                         const float xa = acc[n][2 * half + u], xb = acc[n + 4][2 * half + u];
-                        acc[n][2 * half + u] = xa * c + xb * sn;
-                        acc[n + 4][2 * half + u] = xb * c - xa * sn;
+                        acc[n][2 * half + u] = xa * ec[n][u] + xb * es[n][u];
+                        acc[n + 4][2 * half + u] = xb * ec[n][u] - xa * es[n][u];
                     }
                 }
             }

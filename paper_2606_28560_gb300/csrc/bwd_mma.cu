@@ -395,8 +395,27 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     const bool ok = ok_k && ok_v;
     const float sc = ok ? s.scale : __int_as_float(0x7fc00000);
     __nv_bfloat16* dQ = reinterpret_cast<__nv_bfloat16*>(a.dq) + rowbase * kHeadDim;
+    // cos, sin of pair m = 8n + 2c4 + u (m + 32 sits in n-tile n + 4) at qlo,
+    // then advanced by 8 positions for qhi with the host's cos, sin(8 theta_m)
+    float ec[4][2], es[4][2];
+#pragma unroll
+    for (int n = 0; n < 4; ++n)
+#pragma unroll
+        for (int u = 0; u < 2; ++u) rope_cs(a.rope, 8 * n + 2 * c4 + u, qlo, ec[n][u], es[n][u]);
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
+        if (half == 1) {
+#pragma unroll
+            for (int n = 0; n < 4; ++n)
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int m = 8 * n + 2 * c4 + u;
+                    const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                    const float cn = ec[n][u] * c8 - es[n][u] * s8;
+                    es[n][u] = es[n][u] * c8 + ec[n][u] * s8;
+                    ec[n][u] = cn;
+                }
+        }
         if (!(half ? vhi : vlo)) continue;
         const int q = half ? qhi : qlo;
         __nv_bfloat16* row = dQ + (size_t)q * kHeadDim;
@@ -404,12 +423,9 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         for (int n = 0; n < 4; ++n) {
 #pragma unroll
             for (int u = 0; u < 2; ++u) {
-                const int m = 8 * n + 2 * c4 + u;           // pair (m, m + 32): n-tiles n and n + 4
-                float c, sgn;
-                rope_cs(a.rope, m, q, c, sgn);
                 const float xa = dq[n][2 * half + u] * sc, xb = dq[n + 4][2 * half + u] * sc;
-                dq[n][2 * half + u] = xa * c + xb * sgn;
-                dq[n + 4][2 * half + u] = xb * c - xa * sgn;
+                dq[n][2 * half + u] = xa * ec[n][u] + xb * es[n][u];
+                dq[n + 4][2 * half + u] = xb * ec[n][u] - xa * es[n][u];
             }
         }
 #pragma unroll
