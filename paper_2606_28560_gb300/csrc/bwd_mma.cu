@@ -44,11 +44,11 @@ __device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 
 template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
-                     BwdArgs a, MmaLayout L) {
+                     const __grid_constant__ QTileMaps tm, BwdArgs a, MmaLayout L) {
     grid_dependency_sync();
     constexpr int Wp = NT * 8 - 16;
     extern __shared__ unsigned char smem_raw[];
-    __shared__ unsigned long long bars[2];
+    __shared__ unsigned long long bars[4];        // V (first batch), K~, V (second batch), tile rows
     __shared__ float dps[kWarps][kMmaMaxRungs][16][2];   // rung dp, ddp of each tile row
     __shared__ float gsm[kWarps][kMmaMaxRungs];           // per-warp rung-gradient sums
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -65,15 +65,24 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     const int wrel = warp * kRowsPerWarp;
     const int bw = i0 + wrel;
 
-    // ---- values first
+    // ---- the tile's q, dO, o rows (two 64-row boxes each) to buffer rows
+    // [0, 384), and the value rows that do not overlap them
     if (tid == 0) {
-        mbar_init(&bars[0], 1);
-        mbar_init(&bars[1], 1);
+        for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 0) {
         __syncwarp();
-        issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[0], lane);
+        if (lane == 0) {
+            mbar_expect_tx(&bars[3], 3u * 128u * 128u);
+            const CUtensorMap* maps[3] = {&tm.q, &tm.g, &tm.o};
+#pragma unroll
+            for (int t = 0; t < 3; ++t)
+#pragma unroll
+                for (int hb = 0; hb < 2; ++hb)
+                    tma_load_3d(buf + (size_t)(128 * t + 64 * hb) * 128, maps[t], 0, i0 + 64 * hb, bh, &bars[3]);
+        }
+        if (L.bytes_lo) issue_rows_batch(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[0], lane, false);
     }
 
     const int qlo = bw + g4, qhi = bw + g4 + 8;
@@ -81,42 +90,43 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
     const size_t rowbase = (size_t)bh * s.T;
 
+    __syncthreads();                              // barrier init visible
+    bool ok_v = mbar_wait(&bars[3], 0);
+
+    // A fragments of this warp's 16 tile rows from a staged region: for
+    // k-chunk kc, registers (row g4, dims 16kc + 2c4..), (row g4+8, same),
+    // (row g4, dims 16kc + 8 + 2c4..), (row g4+8, same)
+    auto tile_frags = [&](int region, unsigned (&f)[4][4]) {
+        const int row = 128 * region + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+        for (int kc = 0; kc < 4; ++kc)
+            ldsm_x4(row_chunk(sbase, row, 2 * kc + (lane >> 4)), f[kc][0], f[kc][1], f[kc][2], f[kc][3]);
+    };
+
     // ---- dO as bf16 A fragments; Delta = dO . o of rows g4, g4+8
     unsigned da[4][4];
     float dlt_lo, dlt_hi;
     {
-        const __nv_bfloat16* dO = reinterpret_cast<const __nv_bfloat16*>(a.dout) + rowbase * kHeadDim;
-        const __nv_bfloat16* Og = reinterpret_cast<const __nv_bfloat16*>(a.out) + rowbase * kHeadDim;
+        unsigned oa[4][4];
+        tile_frags(1, da);
+        tile_frags(2, oa);
         float part[2] = {0.f, 0.f};
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-            const int pos = min(qlo + 8 * half, s.T - 1);
-            const __nv_bfloat16* rd = dO + (size_t)pos * kHeadDim;
-            const __nv_bfloat16* ro = Og + (size_t)pos * kHeadDim;
+        for (int kc = 0; kc < 4; ++kc)
 #pragma unroll
-            for (int kc = 0; kc < 4; ++kc) {
-                const unsigned u0 = *reinterpret_cast<const unsigned*>(rd + 16 * kc + 2 * c4);
-                const unsigned u1 = *reinterpret_cast<const unsigned*>(rd + 16 * kc + 8 + 2 * c4);
-                const unsigned o0 = *reinterpret_cast<const unsigned*>(ro + 16 * kc + 2 * c4);
-                const unsigned o1 = *reinterpret_cast<const unsigned*>(ro + 16 * kc + 8 + 2 * c4);
-                da[kc][half] = u0;
-                da[kc][2 + half] = u1;
-                part[half] = fmaf(bf_lo(u0), bf_lo(o0), part[half]);
-                part[half] = fmaf(bf_hi(u0), bf_hi(o0), part[half]);
-                part[half] = fmaf(bf_lo(u1), bf_lo(o1), part[half]);
-                part[half] = fmaf(bf_hi(u1), bf_hi(o1), part[half]);
+            for (int j = 0; j < 4; ++j) {
+                part[j & 1] = fmaf(bf_lo(da[kc][j]), bf_lo(oa[kc][j]), part[j & 1]);
+                part[j & 1] = fmaf(bf_hi(da[kc][j]), bf_hi(oa[kc][j]), part[j & 1]);
             }
-        }
         dlt_lo = quad_sum(part[0]);
         dlt_hi = quad_sum(part[1]);
     }
 
-    // ---- q~ as fp16 A fragments (RoPE pairs m, m+32 in the same thread), also
-    // written to the workspace for the key pass
+    // ---- q~ as fp16 A fragments (RoPE pairs m, m+32 in the same thread)
     unsigned qa[4][4];
     {
-        const __nv_bfloat16* Q = reinterpret_cast<const __nv_bfloat16*>(a.q) + rowbase * kHeadDim;
-        __half* Qt = reinterpret_cast<__half*>(a.qt) + rowbase * kHeadDim;
+        unsigned qr[4][4];
+        tile_frags(0, qr);
         float cs[2][4], sn[2][4];
 #pragma unroll
         for (int kc = 0; kc < 2; ++kc)
@@ -127,13 +137,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-            const int pos = min(qlo + 8 * half, s.T - 1);
-            const __nv_bfloat16* row = Q + (size_t)pos * kHeadDim;
             float x[4][4];
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
-                const unsigned u0 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 2 * c4);
-                const unsigned u1 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 8 + 2 * c4);
+                const unsigned u0 = qr[kc][half], u1 = qr[kc][2 + half];
                 x[kc][0] = bf_lo(u0); x[kc][1] = bf_hi(u0);
                 x[kc][2] = bf_lo(u1); x[kc][3] = bf_hi(u1);
             }
@@ -163,15 +170,37 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);
                 qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);
             }
-            if (half == 0 ? vlo : vhi) {
-                __half* qr = Qt + (size_t)(qlo + 8 * half) * kHeadDim;
-#pragma unroll
-                for (int kc = 0; kc < 4; ++kc) {
-                    *reinterpret_cast<unsigned*>(qr + 16 * kc + 2 * c4) = qa[kc][half];
-                    *reinterpret_cast<unsigned*>(qr + 16 * kc + 8 + 2 * c4) = qa[kc][2 + half];
-                }
-            }
         }
+    }
+    // ---- q~ rows to the workspace (for the key pass): written in place of the
+    // staged q rows, then stored by TMA (rows past T are clipped); the value
+    // rows of the second batch follow once the store has read them
+    __syncthreads();                              // every warp has read the tile rows
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+        if (g4 + 8 * half >= kRowsPerWarp) continue;
+        const int row = wrel + g4 + 8 * half;
+#pragma unroll
+        for (int kc = 0; kc < 4; ++kc) {
+            asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc) + 4 * c4), "r"(qa[kc][half]));
+            asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc + 1) + 4 * c4),
+                         "r"(qa[kc][2 + half]));
+        }
+    }
+    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+    __syncthreads();
+    if (warp == 0) {
+        if (lane == 0) {
+#pragma unroll
+            for (int t = 0; t < 3; ++t)                // 3 boxes of 40 rows: the tile's 120 queries
+                asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];\n"
+                             :: "l"(&tm.qt), "r"(0), "r"(i0 + 40 * t), "r"(bh),
+                                "r"(sbase + (unsigned)(40 * t * 128)) : "memory");
+            asm volatile("cp.async.bulk.commit_group;\n" ::: "memory");
+            asm volatile("cp.async.bulk.wait_group.read 0;\n" ::: "memory");
+        }
+        __syncwarp();
+        issue_rows_batch(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[2], lane, true);
     }
     const float lse2_lo = vlo ? a.lse[rowbase + qlo] * kLog2e : 0.f;
     const float lse2_hi = vhi ? a.lse[rowbase + qhi] * kLog2e : 0.f;
@@ -195,8 +224,17 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     const float df0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f), df1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
     const float m7 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
 
-    __syncthreads();                              // barrier init visible
-    const bool ok_v = mbar_wait(&bars[0], 0);
+    // Value rows: the first batch (rows from L.lo_start on) now, the second
+    // before the first use of a row below L.lo_start.
+    if (L.bytes_lo) ok_v = mbar_wait(&bars[0], 0) && ok_v;
+    bool hi_done = false;
+    auto need_rows = [&](int row) {
+        if (!hi_done && row < L.lo_start) {
+            ok_v = mbar_wait(&bars[2], 0) && ok_v;
+            hi_done = true;
+        }
+    };
+    need_rows(L.win_smem + wrel - Wp);
 
     // ---- window band dp = dO . v
     float dpw[NT][4];
@@ -218,6 +256,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         if (!((a.r.active >> k) & 1u)) continue;
         if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;        // masked for the whole warp
         const float w = a.r.w[k], w1 = 1.f - w;
+        need_rows(L.rung_smem[k] + wrel);
         float dt[2][4];
 #pragma unroll
         for (int t = 0; t < 2; ++t) {
@@ -241,6 +280,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             *reinterpret_cast<float2*>(dps[warp][k][g4 + 8]) = make_float2(dp_hi, ddp_hi);
         }
     }
+
+    need_rows(-1);                                // every copy has landed before the buffer is refilled
 
     // ---- all warps are done with the values: stage the keys into the same buffer
     asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
@@ -442,12 +483,12 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 }
 
 template <int NT>
-cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const BwdArgs& a, const MmaLayout& L,
-                      unsigned grid, size_t smem, cudaStream_t st) {
+cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const QTileMaps& mt, const BwdArgs& a,
+                      const MmaLayout& L, unsigned grid, size_t smem, cudaStream_t st) {
     auto kern = bwd_query_mma_kernel<NT>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mk, mv, a, L);
+    return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mk, mv, mt, a, L);
 }
 
 }  // namespace
@@ -465,15 +506,20 @@ cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStrea
     const long long grid = bwd_mma_blocks(a.s);
     if (grid <= 0) return cudaSuccess;
     RowMaps mk, mv;
-    const int heads = a.s.B * a.s.Hkv;
+    QTileMaps mt;
+    const int heads = a.s.B * a.s.Hkv, qheads = a.s.B * a.s.H;
     if (!encode_row_maps(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
-        !encode_row_maps(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
+        !encode_row_maps(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads) ||
+        !encode_rows_map(&mt.q, a.q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 64) ||
+        !encode_rows_map(&mt.g, a.dout, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 64) ||
+        !encode_rows_map(&mt.o, a.out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 64) ||
+        !encode_rows_map(&mt.qt, a.qt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, qheads, 40))
         return cudaErrorInvalidValue;
     const size_t smem = fwd_mma_smem_bytes(L);
     switch (L.nt) {
-    case 2: return launch_nt<2>(mk, mv, a, L, (unsigned)grid, smem, st);
-    case 3: return launch_nt<3>(mk, mv, a, L, (unsigned)grid, smem, st);
-    default: return launch_nt<4>(mk, mv, a, L, (unsigned)grid, smem, st);
+    case 2: return launch_nt<2>(mk, mv, mt, a, L, (unsigned)grid, smem, st);
+    case 3: return launch_nt<3>(mk, mv, mt, a, L, (unsigned)grid, smem, st);
+    default: return launch_nt<4>(mk, mv, mt, a, L, (unsigned)grid, smem, st);
     }
 }
 

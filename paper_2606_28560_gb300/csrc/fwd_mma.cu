@@ -361,7 +361,7 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
     return r == CUDA_SUCCESS;
 }
 
-size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.rows * 128 + 1024; }
+size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.buf_rows * 128 + 1024; }
 
 namespace {
 
@@ -424,7 +424,30 @@ void rope_steps(double rope_base, MmaLayout* L) {
 
 }  // namespace
 
-bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L) {
+// Copy boxes in issue order (per interval: 64-row boxes, then 8-row boxes);
+// split them at the first box that starts at or after the tile regions.
+void plan_tile_regions(MmaLayout* L) {
+    L->buf_rows = L->rows > kTileRegionRows ? L->rows : kTileRegionRows;
+    L->lo_start = L->rows;
+    L->bytes_lo = 0;
+    L->bytes_hi = 0;
+    for (int iv = 0; iv < L->n_iv; ++iv) {
+        int r = 0;
+        auto box = [&](int srow, int h) {
+            if (srow >= kTileRegionRows) {
+                if (srow < L->lo_start) L->lo_start = srow;
+                L->bytes_lo += (unsigned)h * 128u;
+            } else {
+                L->bytes_hi += (unsigned)h * 128u;
+            }
+        };
+        for (; r + 64 <= L->iv_len[iv]; r += 64) box(L->iv_smem[iv] + r, 64);
+        for (; r < L->iv_len[iv]; r += 8) box(L->iv_smem[iv] + r, 8);
+    }
+}
+
+bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L,
+                      bool reserve_tiles) {
     if (s.W > 16 || r.K > kMmaMaxRungs) return false;
     const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
     const int Wp = NT * 8 - 16;
@@ -442,6 +465,11 @@ bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, siz
     for (int k = 0; k < r.K; ++k)
         if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row_of(*L, -r.s0[k] - 1);
     active_list(r, L);
+    L->buf_rows = L->rows;
+    L->lo_start = 0;
+    L->bytes_lo = (unsigned)L->rows * 128u;
+    L->bytes_hi = 0;
+    if (reserve_tiles) plan_tile_regions(L);
     return fwd_mma_smem_bytes(*L) <= smem_limit;
 }
 
@@ -465,6 +493,10 @@ bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, siz
     for (int k = 0; k < r.K; ++k)
         if ((r.active >> k) & 1u) L->rung_smem[k] = smem_row_of(*L, r.s0[k]);
     active_list(r, L);
+    L->buf_rows = L->rows;
+    L->lo_start = 0;
+    L->bytes_lo = (unsigned)L->rows * 128u;
+    L->bytes_hi = 0;
     return fwd_mma_smem_bytes(*L) <= smem_limit;
 }
 

@@ -32,9 +32,20 @@ struct MmaLayout {
     int act_smem[kMmaMaxRungs];
     float act_w[kMmaMaxRungs];
     float act_d[kMmaMaxRungs];
+    // Staging buffer rows (>= rows).  The query backward first copies its
+    // tile's q, dO, o rows to buffer rows [0, kTileRegionRows); copy boxes that
+    // start at or after lo_start (bytes_lo) are issued at once, the others
+    // (bytes_hi) once the tile rows have been read.
+    int buf_rows;
+    int lo_start;
+    unsigned bytes_lo, bytes_hi;
 };
 
-bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
+constexpr int kTileRegionRows = 3 * 128;          // q, dO, o: 128 rows (two 64-row boxes) each
+
+// reserve_tiles: plan the query backward's tile regions (see MmaLayout).
+bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L,
+                      bool reserve_tiles = false);
 // Key-centric counterpart: query rows [0, M+1+Wp) and [s0, s0+M+1) relative to
 // the first key of a tile (win_smem: relative row 0; rung_smem[k]: row s0_k).
 bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
@@ -48,6 +59,9 @@ struct RowMaps { CUtensorMap m64, m8; };
 inline bool encode_row_maps(RowMaps* m, const void* base, CUtensorMapDataType dt, int T, int heads) {
     return encode_rows_map(&m->m64, base, dt, T, heads, 64) && encode_rows_map(&m->m8, base, dt, T, heads, 8);
 }
+// The query backward's tile rows: q, dO, o (64-row loads) and the rotated q
+// it writes back (40-row stores).
+struct QTileMaps { CUtensorMap q, g, o, qt; };
 cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st);
 
 // Tensor-core query-centric backward over the same staged rows (bf16 I/O;

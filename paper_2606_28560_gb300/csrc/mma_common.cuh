@@ -111,6 +111,24 @@ __device__ __forceinline__ void issue_rows(unsigned char* dst, const CUtensorMap
     }
 }
 
+// One batch of the copies issue_rows makes: boxes that start at or after
+// L.lo_start (hi_batch false) or before it (hi_batch true); the barrier
+// expects that batch's bytes.  Boxes are the same as issue_rows's.
+__device__ __forceinline__ void issue_rows_batch(unsigned char* dst, const CUtensorMap* map64, const CUtensorMap* map8,
+                                                 const MmaLayout& L, int i0, int head, unsigned long long* bar,
+                                                 int lane, bool hi_batch) {
+    if (lane == 0) mbar_expect_tx(bar, hi_batch ? L.bytes_hi : L.bytes_lo);
+    __syncwarp();
+    for (int iv = lane; iv < L.n_iv; iv += 32) {
+        const int len = L.iv_len[iv], srow = L.iv_smem[iv], grow = i0 + L.iv_start[iv];
+        int r = 0;
+        for (; r + 64 <= len; r += 64)
+            if ((srow + r < L.lo_start) == hi_batch) tma_load_3d(dst + (size_t)(srow + r) * 128, map64, 0, grow + r, head, bar);
+        for (; r < len; r += 8)
+            if ((srow + r < L.lo_start) == hi_batch) tma_load_3d(dst + (size_t)(srow + r) * 128, map8, 0, grow + r, head, bar);
+    }
+}
+
 __device__ __forceinline__ void mma_f16_1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
     asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, "
                  "{%0,%1,%2,%3};\n"
