@@ -70,6 +70,59 @@ __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ sr
     }
 }
 
+// bf16 rows in, fp16 rotated rows out.  Thread item = (group of kRopeHeads
+// heads, position, chunk): the 8 angles of the chunk's pairs are evaluated
+// once and applied to that position's row in each head of the group; the
+// rows' loads are all issued before any arithmetic.  A warp covers 8
+// consecutive positions x 4 chunks of one head per access: 1 KB contiguous.
+constexpr int kRopeHeads = 4;
+__global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16* __restrict__ src,
+                                                             __half* __restrict__ dst, int heads, int T_,
+                                                             RopeParams rp, unsigned* zero, int nzero) {
+    grid_dependency_sync();
+    if (blockIdx.x == 0 && (int)threadIdx.x < nzero) zero[threadIdx.x] = 0u;
+    const int groups = (heads + kRopeHeads - 1) / kRopeHeads;
+    const long long n = (long long)groups * T_ * 4;
+    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
+         g += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(g & 3);
+        const long long pg = g >> 2;
+        const int p = (int)(pg % T_), h0 = (int)(pg / T_) * kRopeHeads;
+        uint4 raw[kRopeHeads][2];
+#pragma unroll
+        for (int u = 0; u < kRopeHeads; ++u) {
+            if (h0 + u < heads) {
+                const __nv_bfloat16* row = src + ((size_t)(h0 + u) * T_ + p) * kHeadDim;
+                raw[u][0] = *reinterpret_cast<const uint4*>(row + 8 * c);
+                raw[u][1] = *reinterpret_cast<const uint4*>(row + kHalf + 8 * c);
+            }
+        }
+        float cs[8], sn[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) rope_cs(rp, 8 * c + e, p, cs[e], sn[e]);
+#pragma unroll
+        for (int u = 0; u < kRopeHeads; ++u) {
+            if (h0 + u >= heads) break;
+            const unsigned* wa = reinterpret_cast<const unsigned*>(&raw[u][0]);
+            const unsigned* wb = reinterpret_cast<const unsigned*>(&raw[u][1]);
+            unsigned oa[4], ob[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const float a0 = __uint_as_float(wa[e] << 16), a1 = __uint_as_float(wa[e] & 0xffff0000u);
+                const float b0 = __uint_as_float(wb[e] << 16), b1 = __uint_as_float(wb[e] & 0xffff0000u);
+                const int m0 = 2 * e, m1 = 2 * e + 1;        // pairs (8c + m, 32 + 8c + m)
+                __half2 ra = __floats2half2_rn(a0 * cs[m0] - b0 * sn[m0], a1 * cs[m1] - b1 * sn[m1]);
+                __half2 rb = __floats2half2_rn(b0 * cs[m0] + a0 * sn[m0], b1 * cs[m1] + a1 * sn[m1]);
+                oa[e] = *reinterpret_cast<unsigned*>(&ra);
+                ob[e] = *reinterpret_cast<unsigned*>(&rb);
+            }
+            __half* row = dst + ((size_t)(h0 + u) * T_ + p) * kHeadDim;
+            *reinterpret_cast<uint4*>(row + 8 * c) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
+            *reinterpret_cast<uint4*>(row + kHalf + 8 * c) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
+        }
+    }
+}
+
 // ------------------------------------------------------------- forward ----
 
 template <typename T>
@@ -401,10 +454,15 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
     const long long items = rows * 4;
     long long grid = (items + 255) / 256;
     if (grid > 152 * 16) grid = 152 * 16;       // 16 resident 256-thread blocks on each of 152 SMs
-    if (bf16)
-        return launch_kernel(rope_rows_kernel<__nv_bfloat16, __half>, dim3((unsigned)grid), dim3(256), 0, st,
-                             reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), rows, T, rp,
-                             zero, nzero);
+    if (bf16) {
+        const int heads = (int)(rows / T);
+        const long long gitems = (long long)((heads + kRopeHeads - 1) / kRopeHeads) * T * 4;
+        long long g2 = (gitems + 255) / 256;
+        if (g2 > 152 * 8) g2 = 152 * 8;
+        return launch_kernel(rope_rows_bf16_kernel, dim3((unsigned)g2), dim3(256), 0, st,
+                             reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), heads, T,
+                             rp, zero, nzero);
+    }
     return launch_kernel(rope_rows_kernel<float, float>, dim3((unsigned)grid), dim3(256), 0, st,
                          reinterpret_cast<const float*>(src), reinterpret_cast<float*>(dst), rows, T, rp, zero, nzero);
 }
