@@ -396,7 +396,7 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     MmaLayout ML, KL;
     const size_t smem_limit = 227 * 1024 - bwd_mma_static_smem();
     const bool mma_ok = bf16 && out && (o.bwd_kernel == 0 || o.bwd_kernel == 2) &&
-                        build_mma_layout(a.s, a.r, o.rope_base, smem_limit, &ML, true) &&
+                        build_mma_layout(a.s, a.r, o.rope_base, smem_limit, &ML, 3 * kTileRows) &&
                         build_key_layout(a.s, a.r, o.rope_base, 227 * 1024 - bwd_key_mma_static_smem(), &KL);
     a.Ps = reinterpret_cast<float*>(ws + L.P);      // slot-major p and dS of the tensor-core passes
     a.DSs = reinterpret_cast<float*>(ws + L.DP);

@@ -426,15 +426,15 @@ void rope_steps(double rope_base, MmaLayout* L) {
 
 // Copy boxes in issue order (per interval: 64-row boxes, then 8-row boxes);
 // split them at the first box that starts at or after the tile regions.
-void plan_tile_regions(MmaLayout* L) {
-    L->buf_rows = L->rows > kTileRegionRows ? L->rows : kTileRegionRows;
+void plan_tile_regions(MmaLayout* L, int reserve_rows) {
+    L->buf_rows = L->rows > reserve_rows ? L->rows : reserve_rows;
     L->lo_start = L->rows;
     L->bytes_lo = 0;
     L->bytes_hi = 0;
     for (int iv = 0; iv < L->n_iv; ++iv) {
         int r = 0;
         auto box = [&](int srow, int h) {
-            if (srow >= kTileRegionRows) {
+            if (srow >= reserve_rows) {
                 if (srow < L->lo_start) L->lo_start = srow;
                 L->bytes_lo += (unsigned)h * 128u;
             } else {
@@ -447,7 +447,7 @@ void plan_tile_regions(MmaLayout* L) {
 }
 
 bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L,
-                      bool reserve_tiles) {
+                      int reserve_rows) {
     if (s.W > 16 || r.K > kMmaMaxRungs) return false;
     const int NT = s.W == 0 ? 2 : (s.W <= 8 ? 3 : 4);
     const int Wp = NT * 8 - 16;
@@ -469,7 +469,7 @@ bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, siz
     L->lo_start = 0;
     L->bytes_lo = (unsigned)L->rows * 128u;
     L->bytes_hi = 0;
-    if (reserve_tiles) plan_tile_regions(L);
+    if (reserve_rows > 0) plan_tile_regions(L, reserve_rows);
     return fwd_mma_smem_bytes(*L) <= smem_limit;
 }
 

@@ -32,20 +32,22 @@ struct MmaLayout {
     int act_smem[kMmaMaxRungs];
     float act_w[kMmaMaxRungs];
     float act_d[kMmaMaxRungs];
-    // Staging buffer rows (>= rows).  The query backward first copies its
-    // tile's q, dO, o rows to buffer rows [0, kTileRegionRows); copy boxes that
-    // start at or after lo_start (bytes_lo) are issued at once, the others
-    // (bytes_hi) once the tile rows have been read.
+    // Staging buffer rows (>= rows).  A kernel that first copies its tile's own
+    // rows (128 per tensor: q in the forward; q, dO, o in the query backward)
+    // to buffer rows [0, reserved rows) issues the copy boxes that start at or
+    // after lo_start (bytes_lo) at once and the others (bytes_hi) once the tile
+    // rows have been read.  Without reserved rows, lo_start = 0.
     int buf_rows;
     int lo_start;
     unsigned bytes_lo, bytes_hi;
 };
 
-constexpr int kTileRegionRows = 3 * 128;          // q, dO, o: 128 rows (two 64-row boxes) each
+constexpr int kTileRows = 128;                    // a tile's own rows of one tensor (two 64-row boxes)
 
-// reserve_tiles: plan the query backward's tile regions (see MmaLayout).
+// reserve_rows: buffer rows [0, reserve_rows) hold the tile's own rows first
+// (a multiple of kTileRows; see MmaLayout).
 bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L,
-                      bool reserve_tiles = false);
+                      int reserve_rows = 0);
 // Key-centric counterpart: query rows [0, M+1+Wp) and [s0, s0+M+1) relative to
 // the first key of a tile (win_smem: relative row 0; rung_smem[k]: row s0_k).
 bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
