@@ -63,7 +63,7 @@ def job_throughput(world: int, steps: int, ms_max: float) -> float:
 def workload_config():
     return {"workload": "fwd+bwd, 16 layers, learned alpha (theta_l ~ N(0,0.5)), Fibonacci K=15",
             "B": B, "H": H, "Hkv": H, "T": T, "D": D, "W": W, "layers": L, "K": K, "seed": SEED,
-            "io": "bf16, fp32 accumulate",
+            "io": "bf16, fp32 accumulate; each layer's RoPE-rotated keys kept from its forward for its backward",
             "l2": "inputs larger than L2: distinct per-layer buffers, 1.07 GB of inputs per step"}
 
 
@@ -162,6 +162,8 @@ class Workload:
                 inputs.device_normal_(t, s * 10 + j)
             self.q.append(ts[0]); self.k.append(ts[1]); self.v.append(ts[2]); self.g.append(ts[3])
         self.out = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
+        # rotated keys of each layer, written by its forward and read by its backward
+        self.rk = [torch.empty(shp, dtype=torch.float16, device=device) for _ in range(layers)]
         self.lse = [torch.empty((B, H, T), dtype=torch.float32, device=device) for _ in range(layers)]
         self.dq = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
         self.dk = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
@@ -175,17 +177,17 @@ class Workload:
         fa = self.fa
         for l in range(self.L):
             fa.fwd(self.q[l], self.k[l], self.v[l], self.alphas[l], self.f, W, out=self.out[l], lse=self.lse[l],
-                   workspace=self.ws_f)
+                   workspace=self.ws_f, rotated_k=self.rk[l])
         for l in reversed(range(self.L)):
             fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], self.alphas[l], self.f, W,
                    out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], dtheta=self.dth[l],
-                   dd=self.dd[l], workspace=self.ws_b)
+                   dd=self.dd[l], workspace=self.ws_b, rotated_k=self.rk[l])
 
     def fwd_only(self, W_):
         fa = self.fa
         for l in range(self.L):
             fa.fwd(self.q[l], self.k[l], self.v[l], self.alphas[l], self.f, W_, out=self.out[l], lse=self.lse[l],
-                   workspace=self.ws_f)
+                   workspace=self.ws_f, rotated_k=self.rk[l])
 
 
 def algorithmic_bytes():

@@ -66,6 +66,13 @@ typedef struct {
                           unused); 2 tensor-core kernel (bf16 I/O, `out` given,
                           W <= 16, K <= 16; FIBATTN_ERR_UNSUPPORTED otherwise).
                           Automatic takes 2 where it applies, else 1. */
+    void* rotated_k;   /* optional device buffer of B*Hkv*T*D elements (fp16 for bf16
+                          I/O, fp32 for fp32 I/O), 16-byte aligned [NULL].  Given
+                          it, fibattn_fwd writes the RoPE-rotated keys there
+                          instead of into its workspace, and fibattn_bwd reads
+                          them from there instead of rotating k again (k may then
+                          be NULL): a caller that keeps this buffer from the
+                          forward to the backward keeps it in place of k. */
 } fibattn_opts;
 
 /* ---------------------------------------------------------------------------

@@ -33,7 +33,7 @@ class FibattnError(RuntimeError):
 class Opts(ctypes.Structure):
     _fields_ = [("rope_base", ctypes.c_float), ("scale", ctypes.c_float),
                 ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int), ("fwd_kernel", ctypes.c_int),
-                ("bwd_kernel", ctypes.c_int)]
+                ("bwd_kernel", ctypes.c_int), ("rotated_k", ctypes.c_void_p)]
 
 
 def library_path() -> str:
@@ -91,9 +91,25 @@ FWD_KERNELS = {"auto": 0, "gather": 1, "staged": 2, "mma": 3}
 BWD_KERNELS = {"auto": 0, "gather": 1, "mma": 2}
 
 
-def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto", bwd_kernel="auto") -> Opts:
+def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto", bwd_kernel="auto",
+          rotated_k=None) -> Opts:
     return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1,
-                FWD_KERNELS[fwd_kernel], BWD_KERNELS[bwd_kernel])
+                FWD_KERNELS[fwd_kernel], BWD_KERNELS[bwd_kernel],
+                rotated_k.data_ptr() if rotated_k is not None else None)
+
+
+def rotated_k_like(k: torch.Tensor) -> torch.Tensor:
+    """A buffer for the rotated keys (``rotated_k=``): fp16 for bf16 k, fp32 for fp32 k."""
+    return torch.empty(k.shape, dtype=torch.float16 if k.dtype == torch.bfloat16 else torch.float32,
+                       device=k.device)
+
+
+def _check_rotated(rk, k):
+    if rk is None:
+        return
+    want = torch.float16 if k.dtype == torch.bfloat16 else torch.float32
+    if not (rk.is_cuda and rk.is_contiguous() and rk.dtype == want and rk.shape == k.shape):
+        raise ValueError(f"rotated_k must be a contiguous CUDA {want} tensor of k's shape")
 
 
 def _dtype_code(t: torch.Tensor) -> int:
@@ -154,13 +170,16 @@ def bwd_workspace_bytes(B, H, T, W, K, dtype, Hkv=None, D=64) -> int:
 
 
 def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
-        out=None, lse=None, workspace=None, stream=None, kernel="auto"):
+        out=None, lse=None, workspace=None, stream=None, kernel="auto", rotated_k=None):
     """Forward pass.  q [B,H,T,64]; k, v [B,Hkv,T,64] (fp32 or bf16, CUDA,
-    contiguous).  ``kernel``: "auto", "gather", "staged" or "mma".  Returns (out, lse)."""
+    contiguous).  ``kernel``: "auto", "gather", "staged" or "mma".
+    ``rotated_k``: optional buffer (``rotated_k_like(k)``) that receives the
+    rotated keys for a later ``bwd(..., rotated_k=...)``.  Returns (out, lse)."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
-    o = _opts(rope_base, scale, Hkv, dedup, kernel)
+    _check_rotated(rotated_k, k)
+    o = _opts(rope_base, scale, Hkv, dedup, kernel, rotated_k=rotated_k)
     code = _dtype_code(q)
     for t in (q, k, v):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
@@ -179,15 +198,18 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
 
 
 def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_base=1e4, scale=None, dedup=True,
-        dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None, kernel="auto"):
+        dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None, kernel="auto",
+        rotated_k=None):
     """Backward pass.  ``out``: the forward output (optional; enables the
     tensor-core query pass).  ``kernel``: "auto", "gather" or "mma".
-    Returns (dq, dk, dv, dtheta [1], dd [K]) on the device."""
+    ``rotated_k``: the buffer the forward of the same k filled (skips rotating
+    k again).  Returns (dq, dk, dv, dtheta [1], dd [K]) on the device."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
     K = len(f)
-    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel)
+    _check_rotated(rotated_k, k)
+    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel, rotated_k=rotated_k)
     code = _dtype_code(q)
     for t in (q, k, v, dout) + ((out,) if out is not None else ()):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):

@@ -160,6 +160,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     __shared__ unsigned long long bar;
     __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
     __shared__ float red[kMmaMaxRungs];                   // block 0: dL/dd_k
+    __shared__ long long red64[kWarps * kMmaMaxRungs];
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const unsigned sbase = smem_u32(buf);
 
@@ -181,7 +182,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     __syncthreads();
-    if (blockIdx.x == 0) convert_rung_sums(a, red);
+    if (blockIdx.x == 0) convert_rung_sums(a, red, red64);
 
     unsigned parity = 0;
     bool ok = true;
@@ -272,7 +273,9 @@ cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, co
 
 }  // namespace
 
-size_t bwd_key_mma_static_smem() { return sizeof(float) * (kWarps * kMmaMaxRungs * 16 + kMmaMaxRungs) + 64; }
+size_t bwd_key_mma_static_smem() {
+    return sizeof(float) * (kWarps * kMmaMaxRungs * 16 + kMmaMaxRungs) + sizeof(long long) * kWarps * kMmaMaxRungs + 64;
+}
 
 int bwd_key_mma_blocks(const Shape& s) {
     const long long tiles = (s.T + kMmaTile - 1) / kMmaTile;

@@ -479,7 +479,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     float x = 0.f;
     if (tid < a.r.K && ((a.r.active >> tid) & 1u))
         for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
-    add_rung_partials(a, x);
+    write_rung_partials(a, x);
 }
 
 template <int NT>

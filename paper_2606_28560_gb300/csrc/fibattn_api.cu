@@ -1,6 +1,7 @@
 // fibattn_api.cu -- the C ABI declared in include/fibattn.h: argument checks,
 // host-side parameter prep (rung distances, RoPE phase increments),
 // workspace layout, and the launches.  arXiv 2606.28560, Section 2.
+#include <algorithm>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -51,6 +52,7 @@ size_t rot_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
 struct Resolved {
     float rope_base, scale;
     int Hkv, dedup, fwd_kernel, bwd_kernel;
+    void* rotated_k;
 };
 
 int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
@@ -61,6 +63,8 @@ int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
     r->fwd_kernel = o ? o->fwd_kernel : 0;
     if (r->fwd_kernel < 0 || r->fwd_kernel > 3) return fail(FIBATTN_ERR_INVALID_ARG, "fwd_kernel must be 0, 1, 2 or 3");
     r->bwd_kernel = o ? o->bwd_kernel : 0;
+    r->rotated_k = o ? o->rotated_k : nullptr;
+    if ((uintptr_t)r->rotated_k & 15u) return fail(FIBATTN_ERR_INVALID_ARG, "rotated_k must be 16-byte aligned");
     if (r->bwd_kernel < 0 || r->bwd_kernel > 2) return fail(FIBATTN_ERR_INVALID_ARG, "bwd_kernel must be 0, 1 or 2");
     if (!(r->rope_base > 1.f) || !std::isfinite(r->rope_base))
         return fail(FIBATTN_ERR_INVALID_ARG, "rope_base must be finite and > 1 (got %g)", (double)r->rope_base);
@@ -126,20 +130,25 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
 }
 
 struct BwdLayout {
-    size_t qt, kt, P, DP, Delta, racc, total;
+    size_t qt, kt, P, DP, Delta, rpart, total;
 };
 
-BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype) {
+BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype, bool own_kt) {
     BwdLayout L;
     size_t es = rot_size(dtype);
     size_t S = (size_t)W + 1 + K;
     size_t off = 0;
     L.qt = off; off += align256((size_t)B * H * T * kHeadDim * es);
-    L.kt = off; off += align256((size_t)B * Hkv * T * kHeadDim * es);
+    L.kt = off;
+    if (own_kt) off += align256((size_t)B * Hkv * T * kHeadDim * es);   // else the caller's rotated_k
     L.P = off; off += align256((size_t)B * H * T * S * 4);
     L.DP = off; off += align256((size_t)B * H * T * S * 4);
     L.Delta = off; off += align256((size_t)B * H * T * 4);
-    L.racc = off; off += align256((size_t)kMaxRungs * 8);       // fixed-point rung sums
+    L.rpart = off;                                  // fixed-point rung partials, one per query block
+    Shape s;
+    std::memset(&s, 0, sizeof(s));
+    s.B = B; s.H = H; s.Hkv = Hkv; s.T = T; s.W = W; s.G = H / Hkv;
+    off += align256((size_t)kMaxRungs * 8 * std::max(bwd_simple_blocks(s), bwd_mma_blocks(s)));
     L.total = off;
     return L;
 }
@@ -297,6 +306,7 @@ int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, floa
 size_t fibattn_fwd_workspace_bytes(int B, int H, int T, int D, int W, int K, int dtype, const fibattn_opts* opts) {
     Resolved o;
     if (check_shape(B, H, T, D, W, K, dtype) || resolve_opts(opts, H, D, &o)) return 0;
+    if (o.rotated_k) return 0;                   // the rotated keys go to the caller's buffer
     return align256((size_t)B * o.Hkv * T * kHeadDim * rot_size(dtype));
 }
 
@@ -311,20 +321,22 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     std::memset(&a, 0, sizeof(a));
     if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
     if (B == 0) return FIBATTN_OK;
-    if (!q || !k || !v || !out || !lse || !workspace) return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor or workspace pointer");
+    if (!q || !k || !v || !out || !lse || (!workspace && !o.rotated_k))
+        return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor or workspace pointer");
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(out) || !aligned16(lse) || !aligned16(workspace))
         return fail(FIBATTN_ERR_INVALID_ARG, "tensor pointers must be 16-byte aligned");
     size_t need = fibattn_fwd_workspace_bytes(B, H, T, D, W, K, dtype, opts);
     if (workspace_bytes < need) return fail(FIBATTN_ERR_INVALID_ARG, "workspace too small: %zu < %zu", workspace_bytes, need);
     prep_rope(o.rope_base, &a.rope);
     a.s = make_shape(B, H, T, W, o);
-    a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.kt = workspace;
+    void* kt = o.rotated_k ? o.rotated_k : workspace;
+    a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.kt = kt;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool bf16 = dtype == FIBATTN_BF16;
     cudaError_t e;
     {
         ProfScope p("rope_k", st);
-        e = launch_rope_rows(k, workspace, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+        e = launch_rope_rows(k, kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
     }
     if (e != cudaSuccess) return cuda_fail(e, "rope prologue launch");
     // bf16 I/O: the tensor-core kernel when its layout applies (W <= 16,
@@ -356,7 +368,7 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
 size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K, int dtype, const fibattn_opts* opts) {
     Resolved o;
     if (check_shape(B, H, T, D, W, K, dtype) || resolve_opts(opts, H, D, &o)) return 0;
-    return bwd_layout(B, H, o.Hkv, T, W, K, dtype).total;
+    return bwd_layout(B, H, o.Hkv, T, W, K, dtype, !o.rotated_k).total;
 }
 
 int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, const float* lse, const void* dout,
@@ -372,23 +384,24 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
     if (!dtheta) return fail(FIBATTN_ERR_INVALID_ARG, "dtheta is NULL");
     if (!workspace) return fail(FIBATTN_ERR_INVALID_ARG, "workspace is NULL");
-    if (B > 0 && (!q || !k || !v || !lse || !dout || !dq || !dk || !dv))
+    if (B > 0 && (!q || (!k && !o.rotated_k) || !v || !lse || !dout || !dq || !dk || !dv))
         return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor pointer");
     if (!aligned16(q) || !aligned16(k) || !aligned16(v) || !aligned16(lse) || !aligned16(dout) || !aligned16(dq) ||
         !aligned16(dk) || !aligned16(dv) || !aligned16(workspace) || !aligned16(out) || ((uintptr_t)dtheta & 3u) ||
         ((uintptr_t)dd & 3u))
         return fail(FIBATTN_ERR_INVALID_ARG, "pointers must be 16-byte aligned (dtheta, dd: 4-byte)");
-    BwdLayout L = bwd_layout(B, H, o.Hkv, T, W, K, dtype);
+    BwdLayout L = bwd_layout(B, H, o.Hkv, T, W, K, dtype, !o.rotated_k);
     if (workspace_bytes < L.total) return fail(FIBATTN_ERR_INVALID_ARG, "workspace too small: %zu < %zu", workspace_bytes, L.total);
     prep_rope(o.rope_base, &a.rope);
     a.s = make_shape(B, H, T, W, o);
     char* ws = reinterpret_cast<char*>(workspace);
     a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.dout = dout; a.dq = dq; a.dk = dk; a.dv = dv;
     a.dtheta = dtheta; a.dd = dd;
-    a.qt = ws + L.qt; a.kt = ws + L.kt;
+    a.qt = ws + L.qt; a.kt = o.rotated_k ? o.rotated_k : ws + L.kt;
     a.P = reinterpret_cast<float*>(ws + L.P); a.DP = reinterpret_cast<float*>(ws + L.DP);
     a.Delta = reinterpret_cast<float*>(ws + L.Delta);
-    a.racc = reinterpret_cast<unsigned long long*>(ws + L.racc);
+    a.rpart = reinterpret_cast<long long*>(ws + L.rpart);
+    a.nblk_q = bwd_simple_blocks(a.s);
     a.S = W + 1 + K;
     a.alpha = alpha;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
@@ -403,6 +416,7 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     if (o.bwd_kernel == 2 && !mma_ok)
         return fail(FIBATTN_ERR_UNSUPPORTED, "tensor-core backward needs bf16, out, W <= 16, K <= 16 and a staged row "
                                              "union that fits shared memory");
+    if (mma_ok) a.nblk_q = bwd_mma_blocks(a.s);
     cudaError_t e;
     if (B > 0) {
         if (!mma_ok) {
@@ -410,12 +424,11 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
             e = launch_rope_rows(q, a.qt, (long long)B * H * T, T, a.rope, bf16, st);
             if (e != cudaSuccess) return cuda_fail(e, "rope prologue (q) launch");
         }
-        {
+        if (!o.rotated_k) {                      // else the rotated keys come from the forward
             ProfScope p("rope_k", st);
-            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st,
-                                 reinterpret_cast<unsigned*>(a.racc), 2 * kMaxRungs);
+            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+            if (e != cudaSuccess) return cuda_fail(e, "rope prologue (k) launch");
         }
-        if (e != cudaSuccess) return cuda_fail(e, "rope prologue (k) launch");
         if (mma_ok) {
             ProfScope p("bwd_query_mma", st);
             e = launch_bwd_query_mma(a, ML, st);

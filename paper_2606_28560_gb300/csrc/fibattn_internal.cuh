@@ -71,8 +71,8 @@ struct BwdArgs {
     float* Delta;             // sum_slots p dL/dp per query [B,H,T]
     float* Ps;                // tensor-core path, slot-major [B,H,S,T]: p      (P region)
     float* DSs;               //                                      dS = p (dp - Delta)  (DP region)
-    unsigned long long* racc; // dL/dd_k as 2^-32 fixed point [kMaxRungs] (zeroed by the launch before
-                              // the query pass)
+    long long* rpart;         // per query-pass block dL/dd_k partials, 2^-32 fixed point [kMaxRungs][nblk_q]
+    int nblk_q;               // query-pass blocks
     int S;                    // slots per query = W + 1 + K
     float alpha;
     Shape s;
@@ -191,25 +191,36 @@ __device__ __forceinline__ void rope_chunk(const RopeParams& rp, int pos, int c,
 
 // ------------------------------------------------- rung-gradient reduction --
 
-// dL/dd_k accumulates the query blocks' partial sums as 64-bit fixed point
-// (2^-32 units): integer addition is exact and order-free, so the result does
-// not depend on which block finishes first.  The query pass adds each block's
-// partials (threads k < K hold rung k's; the accumulators are zeroed by the
-// launch before the pass); block 0 of the key pass, which starts after the
-// query pass has completed, converts them and applies the chain rule
+// dL/dd_k is the sum of the query blocks' partials.  Each block writes its
+// partials as 64-bit fixed point (2^-32 units; threads k < K hold rung k's);
+// block 0 of the key pass, which starts after the query pass has completed,
+// adds them up -- integer addition is exact and order-free, so the result
+// does not depend on scheduling -- and applies the chain rule
 // dL/dalpha = sum_k f_k dL/dd_k, dL/dtheta = dL/dalpha (alpha - 0.5)(1.5 - alpha),
 // alpha = 0.5 + sigmoid(theta).
-__device__ __forceinline__ void add_rung_partials(const BwdArgs& a, float partial) {
+__device__ __forceinline__ void write_rung_partials(const BwdArgs& a, float partial) {
     if ((int)threadIdx.x < a.r.K)
-        atomicAdd(a.racc + threadIdx.x, (unsigned long long)__float2ll_rn(partial * 4294967296.0f));
+        a.rpart[(size_t)threadIdx.x * a.nblk_q + blockIdx.x] = __float2ll_rn(partial * 4294967296.0f);
 }
 
-// Called by every thread of block 0 of the key pass.  red: shared scratch of
-// at least K floats.
-__device__ __forceinline__ void convert_rung_sums(const BwdArgs& a, float* red) {
-    const int t = threadIdx.x;
+// Called by every thread of block 0 of the key pass (blockDim a multiple of
+// 32, at most 32 warps).  red: shared scratch of at least K floats; red64:
+// shared scratch of at least (blockDim / 32) * K 64-bit words.
+__device__ __forceinline__ void convert_rung_sums(const BwdArgs& a, float* red, long long* red64) {
+    const int t = threadIdx.x, lane = t & 31, warp = t >> 5, nw = blockDim.x >> 5;
+    for (int k = 0; k < a.r.K; ++k) {
+        const long long* col = a.rpart + (size_t)k * a.nblk_q;
+        long long v = 0;
+        for (int blk = t; blk < a.nblk_q; blk += blockDim.x) v += __ldcg(col + blk);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+        if (lane == 0) red64[warp * a.r.K + k] = v;
+    }
+    __syncthreads();
     if (t < a.r.K) {
-        const float v = (float)((double)(long long)__ldcg(a.racc + t) * 2.3283064365386962890625e-10);
+        long long tot = 0;
+        for (int w = 0; w < nw; ++w) tot += red64[w * a.r.K + t];
+        const float v = (float)((double)tot * 2.3283064365386962890625e-10);
         red[t] = v;
         if (a.dd) a.dd[t] = v;
     }
@@ -256,10 +267,8 @@ cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t 
 
 // ----------------------------------------------------------- launchers ----
 
-// zero / nzero (may be null / 0): device words the launch sets to 0 (the
-// rung accumulators of the query pass that follows it).
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
-                             bool bf16, cudaStream_t st, unsigned* zero = nullptr, int nzero = 0);
+                             bool bf16, cudaStream_t st);
 cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_query(const BwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st);

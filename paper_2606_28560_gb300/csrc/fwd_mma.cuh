@@ -67,8 +67,8 @@ struct QTileMaps { CUtensorMap q, g, o, qt; };
 cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st);
 
 // Tensor-core query-centric backward over the same staged rows (bf16 I/O;
-// needs the forward output for Delta).  Its CTAs write rung partials as rows
-// [0, bwd_mma_blocks) of BwdArgs::partial; static shared memory is
+// needs the forward output for Delta).  Its CTAs write rung partials as
+// columns [0, bwd_mma_blocks) of BwdArgs::rpart; static shared memory is
 // bwd_mma_static_smem() bytes on top of fwd_mma_smem_bytes(L).
 size_t bwd_mma_static_smem();
 int bwd_mma_blocks(const Shape& s);

@@ -53,10 +53,8 @@ __device__ __forceinline__ void axpy16x2(float a, const float2* x, float2* y) {
 
 template <typename T, typename R>
 __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ src, R* __restrict__ dst,
-                                                        long long rows, int T_, RopeParams rp, unsigned* zero,
-                                                        int nzero) {
+                                                        long long rows, int T_, RopeParams rp) {
     grid_dependency_sync();
-    if (blockIdx.x == 0 && (int)threadIdx.x < nzero) zero[threadIdx.x] = 0u;
     // One (row, 8-pair chunk) item per thread per pass; grid-stride over items.
     const long long n = rows * 4;
     for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
@@ -78,9 +76,8 @@ __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ sr
 constexpr int kRopeHeads = 4;
 __global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16* __restrict__ src,
                                                              __half* __restrict__ dst, int heads, int T_,
-                                                             RopeParams rp, unsigned* zero, int nzero) {
+                                                             RopeParams rp) {
     grid_dependency_sync();
-    if (blockIdx.x == 0 && (int)threadIdx.x < nzero) zero[threadIdx.x] = 0u;
     const int groups = (heads + kRopeHeads - 1) / kRopeHeads;
     const long long n = (long long)groups * T_ * 4;
     for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
@@ -363,7 +360,7 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
             if (valid) x += tsm[u][k][0] - dsm[u] * tsm[u][k][1];
         }
     }
-    add_rung_partials(a, x);
+    write_rung_partials(a, x);
 }
 
 // Key-centric pass.  Key row j of kv head hk receives, from every query head
@@ -375,7 +372,8 @@ template <typename T>
 __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
     grid_dependency_sync();
     __shared__ float red[kMaxRungs];
-    if (blockIdx.x == 0) convert_rung_sums(a, red);
+    __shared__ long long red64[(kThreads / 32) * kMaxRungs];
+    if (blockIdx.x == 0) convert_rung_sums(a, red, red64);
     const Shape s = a.s;
     const int c = threadIdx.x & 3;
     const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;
@@ -448,8 +446,7 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
 }  // namespace
 
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
-                             bool bf16, cudaStream_t st, unsigned* zero, int nzero) {
-    if (nzero > 256) return cudaErrorInvalidValue;
+                             bool bf16, cudaStream_t st) {
     if (rows <= 0) return cudaSuccess;
     const long long items = rows * 4;
     long long grid = (items + 255) / 256;
@@ -461,10 +458,10 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
         if (g2 > 152 * 8) g2 = 152 * 8;
         return launch_kernel(rope_rows_bf16_kernel, dim3((unsigned)g2), dim3(256), 0, st,
                              reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), heads, T,
-                             rp, zero, nzero);
+                             rp);
     }
     return launch_kernel(rope_rows_kernel<float, float>, dim3((unsigned)grid), dim3(256), 0, st,
-                         reinterpret_cast<const float*>(src), reinterpret_cast<float*>(dst), rows, T, rp, zero, nzero);
+                         reinterpret_cast<const float*>(src), reinterpret_cast<float*>(dst), rows, T, rp);
 }
 
 cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st) {

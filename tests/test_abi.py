@@ -68,10 +68,10 @@ def test_rung_params_match_oracle(alpha, W):
 def _call_fwd(**kw):
     lib = B.lib()
     args = dict(q=16, k=16, v=16, out=16, lse=16, B=1, H=2, T=8, D=64, W=2, alpha=1.0,
-                K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0)
+                K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0, rk=None)
     args.update(kw)
     f = np.array([1, 2, 3] + [5] * 40, dtype=np.float32)
-    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, 0, 0)
+    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, 0, 0, args["rk"])
     rc = lib.fibattn_fwd(args["q"], args["k"], args["v"], args["out"], args["lse"], args["B"], args["H"],
                          args["T"], args["D"], args["W"], args["alpha"], B._fptr(f), args["K"], args["dtype"],
                          ctypes.byref(o), args["ws"], args["wsb"], None)
@@ -84,6 +84,7 @@ def _call_fwd(**kw):
     (dict(D=128), 2), (dict(D=32), 2), (dict(T=0), 1), (dict(H=0), 1), (dict(dtype=7), 1),
     (dict(Hkv=3), 1), (dict(q=0), 1), (dict(lse=0), 1), (dict(ws=0), 1),
     (dict(q=17), 1), (dict(out=24), 1), (dict(wsb=10), 1), (dict(rope_base=-2.0), 1),
+    (dict(rk=24), 1),
 ])
 def test_fwd_rejects_bad_arguments(kw, code):
     rc, msg = _call_fwd(**kw)
@@ -123,6 +124,13 @@ def test_bwd_rejects_bad_arguments():
 
 def test_workspace_queries():
     import torch
+    lib = B.lib()
+    code = 1
+    with_rk = B.Opts(0.0, 0.0, 0, 0, 0, 0, 256)            # any aligned address: only the size is queried
+    assert lib.fibattn_fwd_workspace_bytes(16, 8, 1024, 64, 8, 15, code, ctypes.byref(with_rk)) == 0
+    plain = lib.fibattn_bwd_workspace_bytes(16, 8, 1024, 64, 8, 15, code, None)
+    assert plain - lib.fibattn_bwd_workspace_bytes(16, 8, 1024, 64, 8, 15, code, ctypes.byref(with_rk)) == \
+        16 * 8 * 1024 * 64 * 2                               # no rotated-key region of its own
     assert fa.fwd_workspace_bytes(16, 8, 1024, 8, 15, torch.bfloat16) >= 16 * 8 * 1024 * 64 * 2
     assert fa.bwd_workspace_bytes(16, 8, 1024, 8, 15, torch.bfloat16) > fa.fwd_workspace_bytes(16, 8, 1024, 8, 15,
                                                                                                  torch.bfloat16)

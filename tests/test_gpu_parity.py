@@ -160,6 +160,25 @@ def test_backward_small(case, dtype, kernel):
         raise
 
 
+@pytest.mark.parametrize("dtype", [torch.bfloat16, torch.float32], ids=["bf16", "f32"])
+def test_rotated_keys_from_the_forward(dtype):
+    """The backward given the forward's rotated keys equals the backward that
+    rotates k itself, bit for bit (same rotation, same kernels)."""
+    q, k, v = inputs.qkv(2, 4, 333, seed=41, dtype=dtype, Hkv=2)
+    g = inputs.dout(2, 4, 333, seed=42, dtype=dtype)
+    qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), g.cuda()
+    f = _offsets("fib", 15)
+    rk = fa.binding.rotated_k_like(kc)
+    out, lse = fa.fwd(qc, kc, vc, 0.9, f, 8, rotated_k=rk)
+    out2, lse2 = fa.fwd(qc, kc, vc, 0.9, f, 8)
+    r1 = fa.bwd(qc, kc, vc, lse, gc, 0.9, f, 8, out=out, rotated_k=rk)
+    r2 = fa.bwd(qc, kc, vc, lse, gc, 0.9, f, 8, out=out)
+    torch.cuda.synchronize()
+    assert torch.equal(out, out2) and torch.equal(lse, lse2)
+    for a, b in zip(r1, r2):
+        assert torch.equal(a, b)
+
+
 def test_empty_batch():
     q = torch.zeros((0, 2, 16, 64), device="cuda")
     out, lse = fa.fwd(q, q, q, 1.0, _offsets("fib", 15), 4)
