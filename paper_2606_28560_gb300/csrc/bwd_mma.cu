@@ -51,6 +51,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     __shared__ unsigned long long bars[4];        // V (first batch), K~, V (second batch), tile rows
     __shared__ float dps[kWarps][kMmaMaxRungs][16][2];   // rung dp, ddp of each tile row
     __shared__ float gsm[kWarps][kMmaMaxRungs];           // per-warp rung-gradient sums
+    __shared__ unsigned long long kbar[kMmaMaxRungs + 1]; // key rows of each merged interval
+    __shared__ unsigned rel_cnt[kMmaMaxRungs + 1];        // warps done with an interval's value rows
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const unsigned sbase = smem_u32(buf);
 
@@ -69,6 +71,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     // [0, 384), and the value rows that do not overlap them
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
+        for (int j = 0; j < L.n_iv; ++j) {
+            mbar_init(&kbar[j], 1);
+            rel_cnt[j] = 0u;
+        }
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     if (warp == 0) {
@@ -250,18 +256,39 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             mma_bf16_16816(dpw[j], da[kc + 1], b2, b3);
         }
     }
+    // Rungs in increasing d; those masked for every row of the warp's tile
+    // (d > bw + 14) form the tail of the list.
+    int n_use = 0;
+    while (n_use < L.n_act && L.act_d[n_use] <= (float)(bw + kRowsPerWarp - 1)) ++n_use;
+
+    // Key rows replace the value rows interval by interval.  A warp visits
+    // intervals in decreasing order (the band's is the last; a rung with larger
+    // d sits lower) and releases each one as it moves below it; the last of the
+    // kWarps warps to release an interval issues its key copies.
+    int rel = L.n_iv;                             // intervals >= rel are released
+    auto release_above = [&](int iv) {
+        while (rel - 1 > iv) {
+            const int j = --rel;
+            if (L.iv_smem[j] < L.lo_start) need_rows(-1);   // second value batch landed first
+            asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+            __syncwarp();
+            if (lane == 0 && atom_add_acq_rel(&rel_cnt[j], 1u) == kWarps - 1)
+                issue_interval(buf, &tmK.m64, &tmK.m8, L, j, i0, head, &kbar[j]);
+            __syncwarp();
+        }
+    };
+
     // ---- rung dp (interpolated) and ddp = dp_far - dp_floor, to shared memory
 #pragma unroll 1
-    for (int k = 0; k < a.r.K; ++k) {
-        if (!((a.r.active >> k) & 1u)) continue;
-        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;        // masked for the whole warp
-        const float w = a.r.w[k], w1 = 1.f - w;
-        need_rows(L.rung_smem[k] + wrel);
+    for (int i = 0; i < n_use; ++i) {
+        release_above(L.act_iv[i]);
+        const float w = L.act_w[i], w1 = 1.f - w;
+        need_rows(L.act_smem[i] + wrel);
         float dt[2][4];
 #pragma unroll
         for (int t = 0; t < 2; ++t) {
             dt[t][0] = dt[t][1] = dt[t][2] = dt[t][3] = 0.f;
-            const int krow = L.rung_smem[k] + wrel + 8 * t + (lane & 7);
+            const int krow = L.act_smem[i] + wrel + 8 * t + (lane & 7);
 #pragma unroll
             for (int kc = 0; kc < 4; kc += 2) {
                 unsigned b0, b1, b2, b3;
@@ -276,18 +303,21 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         const float dp_hi = quad_sum(fmaf(c0, dt[1][2], c1 * dt[1][3]));
         const float ddp_hi = quad_sum(fmaf(df0, dt[1][2], df1 * dt[1][3]));
         if (c4 == 0) {
-            *reinterpret_cast<float2*>(dps[warp][k][g4]) = make_float2(dp_lo, ddp_lo);
-            *reinterpret_cast<float2*>(dps[warp][k][g4 + 8]) = make_float2(dp_hi, ddp_hi);
+            *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
+            *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
         }
     }
+    release_above(-1);
 
-    need_rows(-1);                                // every copy has landed before the buffer is refilled
-
-    // ---- all warps are done with the values: stage the keys into the same buffer
-    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-    __syncthreads();
-    if (warp == 0) issue_rows(buf, &tmK.m64, &tmK.m8, L, i0, head, &bars[1], lane);
-    const bool ok_k = mbar_wait(&bars[1], 0);
+    // key rows of an interval: waited for before its first use
+    bool ok_k = true;
+    unsigned waited = 0u;
+    auto need_keys = [&](int iv) {
+        if (!((waited >> iv) & 1u)) {
+            ok_k = mbar_wait(&kbar[iv], 0) && ok_k;
+            waited |= 1u << iv;
+        }
+    };
 
     const float sc2 = s.scale * kLog2e;
     float* Pg = a.Ps + (size_t)bh * a.S * s.T;       // [slot][T] of this head
@@ -298,6 +328,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     for (int n = 0; n < 8; ++n) dq[n][0] = dq[n][1] = dq[n][2] = dq[n][3] = 0.f;
 
     // ---- window band: scores, p, dS; P and dp per slot to the workspace
+    need_keys(L.win_iv);
     {
         float sw[NT][4];
 #pragma unroll
@@ -364,25 +395,27 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         }
     }
 
+    // ---- rungs that no row of the tile attends: zero slots for the key pass
+    for (int i = n_use; i < L.n_act; ++i) {
+        const int slot = s.W + 1 + L.act_k[i];
+        if (c4 == 0) {
+            if (vlo) { Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
+            if (vhi) { Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
+        }
+        if (lane == 0) gsm[warp][L.act_k[i]] = 0.f;
+    }
     // ---- rungs: scores, p, dS, dL/dd_k; dq~ += dShat_k K~_slab
 #pragma unroll 1
-    for (int k = 0; k < a.r.K; ++k) {
-        if (!((a.r.active >> k) & 1u)) continue;           // never read by the key pass
+    for (int i = 0; i < n_use; ++i) {
+        need_keys(L.act_iv[i]);
+        const int k = L.act_k[i];
         const int slot = s.W + 1 + k;
-        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) {   // masked for every row of the tile
-            if (c4 == 0) {
-                if (vlo) { Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
-                if (vhi) { Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
-            }
-            if (lane == 0) gsm[warp][k] = 0.f;
-            continue;
-        }
-        const float w = a.r.w[k], w1 = 1.f - w;
+        const float w = L.act_w[i], w1 = 1.f - w;
         float st[2][4];
 #pragma unroll
         for (int t = 0; t < 2; ++t) {
             st[t][0] = st[t][1] = st[t][2] = st[t][3] = 0.f;
-            const int krow = L.rung_smem[k] + wrel + 8 * t + (lane & 7);
+            const int krow = L.act_smem[i] + wrel + 8 * t + (lane & 7);
 #pragma unroll
             for (int kc = 0; kc < 4; kc += 2) {
                 unsigned b0, b1, b2, b3;
@@ -397,10 +430,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         const float sd_lo = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
         const float si_hi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3]));
         const float sd_hi = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
-        const float dk = a.r.d[k];
+        const float dk = L.act_d[i];
         const bool okl = vlo && dk <= (float)qlo, okh = vhi && dk <= (float)qhi;
-        const float2 dpl = *reinterpret_cast<const float2*>(dps[warp][k][g4]);
-        const float2 dph = *reinterpret_cast<const float2*>(dps[warp][k][g4 + 8]);
+        const float2 dpl = *reinterpret_cast<const float2*>(dps[warp][i][g4]);
+        const float2 dph = *reinterpret_cast<const float2*>(dps[warp][i][g4 + 8]);
         const float dp_lo = dpl.x, ddp_lo = dpl.y, dp_hi = dph.x, ddp_hi = dph.y;
         const float p_lo = okl ? exp2f(si_lo * sc2 - lse2_lo) : 0.f;
         const float p_hi = okh ? exp2f(si_hi * sc2 - lse2_hi) : 0.f;
@@ -422,7 +455,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         // dShat_k as fp16 A fragment: the interpolation weights times dS of the row
         const unsigned afr[4] = {pack_f16(c0 * ds_lo, c1 * ds_lo), 0u, pack_f16(c7 * ds_lo, 0.f),
                                  pack_f16(c0 * ds_hi, c1 * ds_hi)};
-        const int krow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+        const int krow = L.act_smem[i] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
@@ -494,7 +527,9 @@ cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const QTileMaps& mt,
 }  // namespace
 
 size_t bwd_mma_static_smem() {
-    return sizeof(float) * kWarps * kMmaMaxRungs * 16 * 2 + sizeof(float) * kWarps * kMmaMaxRungs + 64;
+    // dps, gsm, the interval barriers and counters, the four phase barriers
+    return sizeof(float) * kWarps * kMmaMaxRungs * 16 * 2 + sizeof(float) * kWarps * kMmaMaxRungs +
+           (sizeof(unsigned long long) + sizeof(unsigned)) * (kMmaMaxRungs + 1) + 4 * sizeof(unsigned long long) + 64;
 }
 
 int bwd_mma_blocks(const Shape& s) {

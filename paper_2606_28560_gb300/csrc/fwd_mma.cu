@@ -395,7 +395,14 @@ int smem_row_of(const MmaLayout& L, int rel) {
     return -1;
 }
 
-// Active rungs sorted by d (ties by index), with their shared rows.
+int interval_of(const MmaLayout& L, int smem_row) {
+    for (int i = 0; i < L.n_iv; ++i)
+        if (smem_row >= L.iv_smem[i] && smem_row < L.iv_smem[i] + L.iv_len[i]) return i;
+    return 0;
+}
+
+// Active rungs sorted by d (ties by index), with their shared rows and the
+// merged interval of each slab.
 void active_list(const RungParams& r, MmaLayout* L) {
     L->n_act = 0;
     for (int i = 0; i < kMmaMaxRungs; ++i) {
@@ -412,6 +419,8 @@ void active_list(const RungParams& r, MmaLayout* L) {
         L->act_k[i] = k; L->act_s0[i] = r.s0[k]; L->act_smem[i] = L->rung_smem[k];
         L->act_w[i] = r.w[k]; L->act_d[i] = r.d[k];
     }
+    for (int i = 0; i < kMmaMaxRungs; ++i) L->act_iv[i] = i < L->n_act ? interval_of(*L, L->act_smem[i]) : 0;
+    L->win_iv = interval_of(*L, L->win_smem);
 }
 
 void rope_steps(double rope_base, MmaLayout* L) {

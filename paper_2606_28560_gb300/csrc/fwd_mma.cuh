@@ -32,6 +32,8 @@ struct MmaLayout {
     int act_smem[kMmaMaxRungs];
     float act_w[kMmaMaxRungs];
     float act_d[kMmaMaxRungs];
+    int act_iv[kMmaMaxRungs];                     // merged interval that holds the rung's slab
+    int win_iv;                                   // merged interval that holds the window band
     // Staging buffer rows (>= rows).  A kernel that first copies its tile's own
     // rows (128 per tensor: q in the forward; q, dO, o in the query backward)
     // to buffer rows [0, reserved rows) issues the copy boxes that start at or

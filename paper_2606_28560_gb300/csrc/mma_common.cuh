@@ -129,6 +129,26 @@ __device__ __forceinline__ void issue_rows_batch(unsigned char* dst, const CUten
     }
 }
 
+// One thread copies merged interval iv (64-row boxes, then 8-row boxes) under
+// barrier `bar`, which it arms with the interval's byte count first.
+__device__ __forceinline__ void issue_interval(unsigned char* dst, const CUtensorMap* map64, const CUtensorMap* map8,
+                                               const MmaLayout& L, int iv, int i0, int head, unsigned long long* bar) {
+    const int len = L.iv_len[iv], srow = L.iv_smem[iv], grow = i0 + L.iv_start[iv];
+    mbar_expect_tx(bar, (unsigned)len * 128u);
+    int r = 0;
+    for (; r + 64 <= len; r += 64) tma_load_3d(dst + (size_t)(srow + r) * 128, map64, 0, grow + r, head, bar);
+    for (; r < len; r += 8) tma_load_3d(dst + (size_t)(srow + r) * 128, map8, 0, grow + r, head, bar);
+}
+
+// Shared-memory counter increment with acquire-release order (CTA scope);
+// returns the old value.
+__device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
+    unsigned old;
+    asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], %2;\n" : "=r"(old) : "r"(smem_u32(p)), "r"(v)
+                 : "memory");
+    return old;
+}
+
 __device__ __forceinline__ void mma_f16_1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
     asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, "
                  "{%0,%1,%2,%3};\n"
