@@ -318,8 +318,50 @@ def run_gpu(args, rank, world, device):
         del gf
 
     e2e = run_e2e(args, wl, device, dist)
+    stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
-                algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps)
+                algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
+                stack=stack)
+
+
+def run_autograd_stack(device, warm=2, reps=3):
+    """A 16-layer attention stack (q = k = v = the previous output, no
+    projections) through the torch.autograd wrapper, forward and backward of
+    L = sum(out), per alpha schedule, at T = 1024 (B16) and T = 4096 (B4):
+    eager steps, Python and autograd included."""
+    import paper_2606_28560_gb300 as fa
+    from paper_2606_28560_gb300 import inputs
+    f = fa.base("fib", K)
+    res = {}
+    for Bs, Ts in ((16, 1024), (4, 4096)):
+        x = torch.empty((Bs, H, Ts, D), dtype=torch.bfloat16, device=device)
+        inputs.device_normal_(x, 77)
+        x.requires_grad_(True)
+        for kind in ("fixed", "linear", "coprime", "learned"):
+            th = inputs.theta_learned(L, seed=SEED) if kind == "learned" else None
+            alphas = fa.alpha_schedule(kind, L, theta=th)
+            layers = [fa.FibAttention(W=W, offsets=f, theta=fa.theta_of_alpha(float(a)),
+                                      learned=(kind == "learned")).to(device) for a in alphas]
+
+            def step():
+                out = fa.attention_stack(x, layers)
+                out.float().sum().backward()
+                x.grad = None
+
+            for _ in range(warm):
+                step()
+            torch.cuda.synchronize(device)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record()
+            for _ in range(reps):
+                step()
+            e1.record()
+            torch.cuda.synchronize(device)
+            ms = e0.elapsed_time(e1) / reps
+            res[f"T{Ts}_B{Bs}_{kind}"] = {"ms_per_step": round(ms, 3),
+                                          "query_heads_per_s": round(Bs * H * Ts * L / (ms * 1e-3), 1)}
+        del x
+    return res
 
 
 def run_e2e(args, wl, device, dist):
@@ -498,6 +540,7 @@ def main():
                          "algorithmic_bytes_per_launch": r["algo"].get(r["dom"])},
             "kernels": r["kernels"],
             "forward_only_B16H8T1024": r["fwd_sweep"],
+            "autograd_stack_16_layers": r["stack"],
             "cpu_baseline": cpu,
             "e2e": r["e2e"],
             "gpu_launches": r["launches"],

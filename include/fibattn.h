@@ -142,6 +142,21 @@ int fibattn_base(int kind, int K, float* f);
 int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, float* alpha);
 
 /* ---------------------------------------------------------------------------
+ * Coverage of a layer stack (Section 4.2, "Why staggering widens coverage"):
+ * the distinct key distances i - j a query reads.  Layer l (alpha = alphas[l])
+ * reads D_l = {0..W} plus, for each active rung with d_k <= T-1 (the rung
+ * prep of fibattn_rung_params, with T's reach), the floor row's distance
+ * floor(d_k) and, when d_k is fractional, the far row's floor(d_k)+1.
+ * Outputs (each may be NULL): per_layer[l] = |D_l| (L ints); union_count =
+ * |union of D_l|; beyond_window = |union of D_l minus {0..W}|; two_hop =
+ * |union over l of {a + b < T : a in D_l, b in D_l+1}| (what a query's
+ * representation after two successive layers draws on).  Host arrays;
+ * 1 <= L <= 4096, 1 <= T <= 1<<20.
+ * ------------------------------------------------------------------------- */
+int fibattn_coverage(int L, const float* alphas, const float* offsets, int K, int W, int T, int no_dedup,
+                     int* per_layer, int* union_count, int* beyond_window, int* two_hop);
+
+/* ---------------------------------------------------------------------------
  * Forward without a caller-provided workspace.  The paper has no counterpart;
  * this serves callers that cannot allocate device memory -- a host framework
  * that owns all device memory and gives its plugins only tensors, or a hot

@@ -153,6 +153,31 @@ def offsets_fp32(alpha: float, f) -> np.ndarray:
     return out
 
 
+def coverage(alphas, f, W: int, T: int, dedup: bool = True) -> dict:
+    """Distinct key distances a query reads in a stack of layers (Section 4.2,
+    "Why staggering widens coverage"), as plain sets.  Layer l reads the window
+    distances 0..W and, for each rung with d_k <= T-1 (and d_k > W under dedup),
+    the floor row's distance floor(d_k) and, if d_k is fractional, the far row's
+    floor(d_k)+1.  Returns the per-layer counts, the size of the union over
+    layers, the part of it beyond the window, and the size of the union over
+    successive layer pairs of the sums a + b < T."""
+    sets = []
+    for a in alphas:
+        s = set(range(min(W, T - 1) + 1))
+        for dk in offsets_fp32(float(a), f):
+            if dk > T - 1 or (dedup and not dk > W):
+                continue
+            s0 = math.floor(dk)
+            s.add(s0)
+            if dk != s0 and s0 + 1 < T:
+                s.add(s0 + 1)
+        sets.append(s)
+    union = set().union(*sets)
+    hop = {a + b for l in range(len(sets) - 1) for a in sets[l] for b in sets[l + 1] if a + b < T}
+    return dict(per_layer=[len(x) for x in sets], union=len(union), beyond_window=sum(1 for t in union if t > W),
+                two_hop=len(hop))
+
+
 # --------------------------------------------------------------------------
 # Forward / backward (Section 2 "Attended set"; chain rule of that definition)
 # --------------------------------------------------------------------------

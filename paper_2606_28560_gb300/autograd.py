@@ -1,0 +1,98 @@
+"""torch.autograd wrapper of the C-ABI forward and backward.
+
+The paper trains the per-layer scalar alpha = 0.5 + sigmoid(theta) together
+with the model through this attention (arXiv 2606.28560, Section 2, "The
+per-layer scalar" and "Implementation note").  `FibAttentionFunction` runs
+`fibattn_fwd` and `fibattn_bwd`; the forward keeps the RoPE-rotated keys for
+the backward (in place of k, the same size), so the backward does not rotate
+k again.  alpha is a host value of the C ABI -- the kernels' shared-memory
+layout depends on the rung distances -- so a theta held on the GPU is read
+once per call.
+"""
+from __future__ import annotations
+
+import math
+
+import torch
+
+from . import binding as B
+
+
+def alpha_of_theta(theta: float) -> float:
+    """alpha = 0.5 + sigmoid(theta) (Section 2, "The per-layer scalar")."""
+    return 0.5 + 1.0 / (1.0 + math.exp(-theta))
+
+
+class FibAttentionFunction(torch.autograd.Function):
+    """out = attention(q, k, v) over the window and the scaled-Fibonacci rungs
+    at alpha = 0.5 + sigmoid(theta).  Gradients flow to q, k, v and theta
+    (a 0-dim tensor); offsets, W and the options are constants."""
+
+    @staticmethod
+    def forward(ctx, q, k, v, theta, offsets, W, rope_base, scale, dedup):
+        alpha = alpha_of_theta(float(theta))
+        rk = B.rotated_k_like(k)
+        out, lse = B.fwd(q, k, v, alpha, offsets, W, rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk)
+        ctx.save_for_backward(q, k, v, out, lse, rk)
+        ctx.args = (alpha, offsets, W, rope_base, scale, dedup, theta.dtype, theta.device)
+        return out
+
+    @staticmethod
+    def backward(ctx, dout):
+        q, k, v, out, lse, rk = ctx.saved_tensors
+        alpha, offsets, W, rope_base, scale, dedup, tdtype, tdev = ctx.args
+        dq, dk, dv, dth, _ = B.bwd(q, k, v, lse, dout.contiguous(), alpha, offsets, W, out=out,
+                                   rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk)
+        dtheta = dth.reshape(()).to(device=tdev, dtype=tdtype)
+        return dq, dk, dv, dtheta, None, None, None, None, None
+
+
+def fib_attention(q, k, v, theta, offsets=None, W: int = 8, *, rope_base: float = 1e4, scale=None,
+                  dedup: bool = True):
+    """Functional form.  q [B,H,T,64]; k, v [B,Hkv,T,64] (bf16 or fp32, CUDA,
+    contiguous); theta a 0-dim tensor (requires_grad for the learned
+    schedule); offsets the base sequence (default: Fibonacci, K = 15)."""
+    if offsets is None:
+        offsets = B.base("fib", 15)
+    if not torch.is_tensor(theta):
+        theta = torch.tensor(float(theta))
+    return FibAttentionFunction.apply(q, k, v, theta, offsets, W, rope_base, scale, dedup)
+
+
+class FibAttention(torch.nn.Module):
+    """One layer's attention with its own scalar theta (learned unless
+    `learned=False`; alpha = 0.5 + sigmoid(theta))."""
+
+    def __init__(self, W: int = 8, offsets=None, theta: float = 0.0, learned: bool = True, rope_base: float = 1e4,
+                 scale=None, dedup: bool = True):
+        super().__init__()
+        t = torch.tensor(float(theta))
+        if learned:
+            self.theta = torch.nn.Parameter(t)
+        else:
+            self.register_buffer("theta", t)
+        self.W, self.rope_base, self.scale, self.dedup = W, rope_base, scale, dedup
+        self.offsets = B.base("fib", 15) if offsets is None else offsets
+
+    @property
+    def alpha(self) -> float:
+        return alpha_of_theta(float(self.theta))
+
+    def forward(self, q, k, v):
+        return FibAttentionFunction.apply(q, k, v, self.theta, self.offsets, self.W, self.rope_base, self.scale,
+                                          self.dedup)
+
+
+def theta_of_alpha(alpha: float) -> float:
+    """Inverse of alpha_of_theta on (0.5, 1.5); the ends map to -/+ infinity,
+    clamped to +-30 (alpha within 1e-13 of the end)."""
+    a = min(max(alpha, 0.5 + 1e-13), 1.5 - 1e-13)
+    return max(-30.0, min(30.0, math.log((a - 0.5) / (1.5 - a))))
+
+
+def attention_stack(x: torch.Tensor, layers) -> torch.Tensor:
+    """A stack of attention layers without projections: each layer attends
+    with q = k = v = the previous layer's output (the first takes x)."""
+    for layer in layers:
+        x = layer(x, x, x)
+    return x

@@ -145,6 +145,22 @@ def alpha_schedule(kind: str, L: int = 16, theta=None, stride: int = 7) -> np.nd
     return out
 
 
+def coverage(alphas, offsets, W: int, T: int, dedup: bool = True) -> dict:
+    """Distinct key distances of a layer stack (see fibattn_coverage)."""
+    al = np.ascontiguousarray(np.asarray(alphas, dtype=np.float32))
+    f = _offsets(offsets)
+    L = lib()
+    ip = ctypes.POINTER(ctypes.c_int)
+    L.fibattn_coverage.argtypes = [ctypes.c_int, ctypes.POINTER(ctypes.c_float), ctypes.POINTER(ctypes.c_float),
+                                   ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ip, ip, ip, ip]
+    L.fibattn_coverage.restype = ctypes.c_int
+    per = np.zeros(len(al), dtype=np.int32)
+    u, bw, hop = ctypes.c_int(), ctypes.c_int(), ctypes.c_int()
+    _check(L.fibattn_coverage(len(al), _fptr(al), _fptr(f), len(f), int(W), int(T), 0 if dedup else 1,
+                              _iptr(per), ctypes.byref(u), ctypes.byref(bw), ctypes.byref(hop)))
+    return dict(per_layer=per, union=u.value, beyond_window=bw.value, two_hop=hop.value)
+
+
 def rung_params(alpha: float, offsets, W: int, dedup: bool = True):
     f = _offsets(offsets)
     K = len(f)

@@ -455,4 +455,44 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     return FIBATTN_OK;                           // dtheta and dd: written by block 0 of the key pass
 }
 
+int fibattn_coverage(int L, const float* alphas, const float* offsets, int K, int W, int T, int no_dedup,
+                     int* per_layer, int* union_count, int* beyond_window, int* two_hop) {
+    if (L < 1 || L > 4096 || !alphas) return fail(FIBATTN_ERR_INVALID_ARG, "need 1 <= L <= 4096 alphas");
+    if (T < 1 || T > (1 << 20)) return fail(FIBATTN_ERR_INVALID_ARG, "T must be in [1, 2^20]");
+    if (W < 0 || K < 0 || K > kMaxRungs) return fail(FIBATTN_ERR_INVALID_ARG, "need W >= 0 and 0 <= K <= %d", kMaxRungs);
+    std::vector<std::vector<int>> D(L);
+    std::vector<char> uni(T, 0);
+    for (int l = 0; l < L; ++l) {
+        RungParams r;
+        int rc = prep_rungs(alphas[l], offsets, K, W, no_dedup ? 0 : 1, T, &r);
+        if (rc) return rc;
+        std::vector<char> in(T, 0);
+        for (int t = 0; t <= W && t < T; ++t) in[t] = 1;
+        for (int k = 0; k < K; ++k) {
+            if (!((r.active >> k) & 1u)) continue;
+            if (r.s0[k] < T) in[r.s0[k]] = 1;
+            if (r.w[k] != 0.f && r.s0[k] + 1 < T) in[r.s0[k] + 1] = 1;
+        }
+        for (int t = 0; t < T; ++t)
+            if (in[t]) { D[l].push_back(t); uni[t] = 1; }
+        if (per_layer) per_layer[l] = (int)D[l].size();
+    }
+    int u = 0, beyond = 0;
+    for (int t = 0; t < T; ++t)
+        if (uni[t]) { ++u; if (t > W) ++beyond; }
+    if (union_count) *union_count = u;
+    if (beyond_window) *beyond_window = beyond;
+    if (two_hop) {
+        std::vector<char> hop(T, 0);
+        for (int l = 0; l + 1 < L; ++l)
+            for (int a : D[l])
+                for (int b : D[l + 1])
+                    if (a + b < T) hop[a + b] = 1;
+        int n = 0;
+        for (int t = 0; t < T; ++t) n += hop[t];
+        *two_hop = n;
+    }
+    return FIBATTN_OK;
+}
+
 }  // extern "C"
