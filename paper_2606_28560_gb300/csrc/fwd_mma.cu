@@ -17,10 +17,10 @@
 //
 // Precision (bf16 I/O): q~ and k~ enter the score MMAs as fp16 (11-bit
 // significands); P of the window band is the unnormalised exp(s - max) in
-// bf16, so the largest entry of each row is exactly 1; Phat of a rung carries
-// arbitrary interpolation weights and is split into bf16 hi + lo parts (two
-// MMAs), which keeps the weights exact to ~2^-17.  Row sums use the same
-// rounded values.  Accumulation is fp32.
+// bf16, so the largest entry of each row is exactly 1; the entries p w and
+// p (1-w) of a rung's Phat are rounded to bf16 the same way.  Row sums use the
+// same rounded values, so each output is a normalised average of the values.
+// Accumulation is fp32.
 //
 // Staging: the CTA's union of key rows (rotated keys, fp16) and then of value
 // rows (bf16, same buffer) is copied by TMA (3-D tensor maps [heads][T][64],
@@ -280,16 +280,14 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
         const float w = a.r.w[k], w1 = 1.f - w;
         const float plo = exp2f(rs[k][0] - mlo), phi = exp2f(rs[k][1] - mhi);   // 0 when masked
-        llo += plo;
-        lhi += phi;
-        // Phat as bf16 hi + lo A fragments (a1, row g4+8 at columns 2c4.., is zero)
+        // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
+        // take the same rounded entries, as for the window band
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-        const float e00 = c0 * plo, e01 = c1 * plo, e20 = c7 * plo, e30 = c0 * phi, e31 = c1 * phi;
-        const float h00 = bf16_round(e00), h01 = bf16_round(e01), h20 = bf16_round(e20);
-        const float h30 = bf16_round(e30), h31 = bf16_round(e31);
+        const float h00 = bf16_round(c0 * plo), h01 = bf16_round(c1 * plo), h20 = bf16_round(c7 * plo);
+        const float h30 = bf16_round(c0 * phi), h31 = bf16_round(c1 * phi);
+        llo += quad_sum(h00 + h01 + h20);
+        lhi += quad_sum(h30 + h31);
         const unsigned ahi[4] = {pack_bf16(h00, h01), 0u, pack_bf16(h20, 0.f), pack_bf16(h30, h31)};
-        const unsigned alo[4] = {pack_bf16(e00 - h00, e01 - h01), 0u, pack_bf16(e20 - h20, 0.f),
-                                 pack_bf16(e30 - h30, e31 - h31)};
         const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
@@ -297,8 +295,6 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
             mma_bf16_16816(o[n], ahi, b0, b1);
             mma_bf16_16816(o[n + 1], ahi, b2, b3);
-            mma_bf16_16816(o[n], alo, b0, b1);
-            mma_bf16_16816(o[n + 1], alo, b2, b3);
         }
     }
 
