@@ -183,6 +183,19 @@ class Workload:
                    out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], dtheta=self.dth[l],
                    dd=self.dd[l], workspace=self.ws_b, rotated_k=self.rk[l])
 
+    def step_fixed(self, rung_grads: bool):
+        """The same step at alpha = 1 in every layer (integer rung distances);
+        without rung_grads the backward skips dL/dtheta (a fixed schedule)."""
+        fa = self.fa
+        for l in range(self.L):
+            fa.fwd(self.q[l], self.k[l], self.v[l], 1.0, self.f, W, out=self.out[l], lse=self.lse[l],
+                   workspace=self.ws_f, rotated_k=self.rk[l])
+        for l in reversed(range(self.L)):
+            fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], 1.0, self.f, W,
+                   out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l],
+                   dtheta=self.dth[l] if rung_grads else None, dd=self.dd[l] if rung_grads else None,
+                   workspace=self.ws_b, rotated_k=self.rk[l], rung_grads=rung_grads)
+
     def fwd_only(self, W_):
         fa = self.fa
         for l in range(self.L):
@@ -317,11 +330,30 @@ def run_gpu(args, rank, world, device):
                                "fwd_kernel_frac_of_hbm": round(cbytes / (us * 1e-6) / 1e9 / hbm, 4)}
         del gf
 
+    # the integer path: alpha = 1 in every layer, with and without dL/dtheta
+    integer = {}
+    for name, rg in (("alpha1_with_dtheta", True), ("alpha1_no_dtheta", False)):
+        gi = capture(lambda: wl.step_fixed(rg), device, profile=False)
+        for _ in range(2):
+            gi.replay()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(3, args.steps // 3)
+        a0.record(stream)
+        for _ in range(reps):
+            gi.replay()
+        a1.record(stream)
+        torch.cuda.synchronize(device)
+        integer[name] = {"ms_per_step": round(a0.elapsed_time(a1) / reps, 4)}
+        del gi
+    integer["learned_alpha_ms_per_step"] = round(ms_max / args.steps, 4)
+    integer["interpolated_over_integer"] = round(integer["learned_alpha_ms_per_step"] /
+                                                 integer["alpha1_with_dtheta"]["ms_per_step"], 3)
+
     e2e = run_e2e(args, wl, device, dist)
     stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
                 algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
-                stack=stack)
+                stack=stack, integer=integer)
 
 
 def run_autograd_stack(device, warm=2, reps=3):
@@ -541,6 +573,7 @@ def main():
             "kernels": r["kernels"],
             "forward_only_B16H8T1024": r["fwd_sweep"],
             "autograd_stack_16_layers": r["stack"],
+            "integer_vs_interpolated_16_layers": r["integer"],
             "cpu_baseline": cpu,
             "e2e": r["e2e"],
             "gpu_launches": r["launches"],

@@ -102,8 +102,10 @@ int fibattn_fwd(const void* q, const void* k, const void* v,
  * in one pass; without it Delta is accumulated from the slots.
  * Outputs (overwritten, not accumulated): dq [B,H,T,D], dk and dv [B,Hkv,T,D]
  * in `dtype`, gradients with respect to the pre-RoPE q and k; dtheta (device,
- * 1 float) = dL/dtheta with alpha = 0.5 + sigmoid(theta); dd (device, K floats,
- * may be NULL) = dL/dd_k for each rung distance.  dL/dalpha = sum_k f_k dd_k.
+ * 1 float, may be NULL) = dL/dtheta with alpha = 0.5 + sigmoid(theta); dd
+ * (device, K floats, may be NULL) = dL/dd_k for each rung distance.
+ * dL/dalpha = sum_k f_k dd_k.  With both NULL (a fixed alpha schedule, alpha
+ * not trained) the rung-distance gradient is not computed at all.
  * At an integer d_k the distance derivative is one-sided, from above.
  * ------------------------------------------------------------------------- */
 size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K,

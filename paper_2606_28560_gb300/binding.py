@@ -215,11 +215,13 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
 
 def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_base=1e4, scale=None, dedup=True,
         dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None, kernel="auto",
-        rotated_k=None):
+        rotated_k=None, rung_grads=True):
     """Backward pass.  ``out``: the forward output (optional; enables the
     tensor-core query pass).  ``kernel``: "auto", "gather" or "mma".
     ``rotated_k``: the buffer the forward of the same k filled (skips rotating
-    k again).  Returns (dq, dk, dv, dtheta [1], dd [K]) on the device."""
+    k again).  ``rung_grads=False`` skips dL/dtheta and dL/dd_k (a fixed
+    schedule).  Returns (dq, dk, dv, dtheta [1], dd [K]) on the device
+    (dtheta, dd None without rung_grads)."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
@@ -233,17 +235,22 @@ def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_bas
     dq = torch.empty_like(q) if dq is None else dq
     dk = torch.empty_like(k) if dk is None else dk
     dv = torch.empty_like(v) if dv is None else dv
-    dtheta = torch.empty(4, dtype=torch.float32, device=q.device) if dtheta is None else dtheta
-    dd = torch.empty(max(K, 1), dtype=torch.float32, device=q.device) if dd is None else dd
+    if rung_grads:
+        dtheta = torch.empty(4, dtype=torch.float32, device=q.device) if dtheta is None else dtheta
+        dd = torch.empty(max(K, 1), dtype=torch.float32, device=q.device) if dd is None else dd
     need = int(lib().fibattn_bwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
     if workspace is None:
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
     _check(lib().fibattn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr() if out is not None else None,
                              lse.data_ptr(), dout.data_ptr(),
-                             dq.data_ptr(), dk.data_ptr(), dv.data_ptr(), dtheta.data_ptr(), dd.data_ptr(),
+                             dq.data_ptr(), dk.data_ptr(), dv.data_ptr(),
+                             dtheta.data_ptr() if dtheta is not None else None,
+                             dd.data_ptr() if dd is not None else None,
                              B, H, T, D, int(W), float(alpha), _fptr(f), K, code, ctypes.byref(o),
                              workspace.data_ptr(), workspace.numel(), _stream_ptr(stream)))
-    return dq, dk, dv, dtheta[:1], dd[:K]
+    if dtheta is None and dd is None:
+        return dq, dk, dv, None, None
+    return dq, dk, dv, (dtheta[:1] if dtheta is not None else None), (dd[:K] if dd is not None else None)
 
 
 # ------------------------------------------------------------- profiling ----

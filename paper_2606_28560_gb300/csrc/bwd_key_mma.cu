@@ -182,7 +182,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     __syncthreads();
-    if (blockIdx.x == 0) convert_rung_sums(a, red, red64);
+    if (blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
 
     unsigned parity = 0;
     bool ok = true;

@@ -41,7 +41,9 @@ constexpr int kRowsPerWarp = 15;
 __device__ __forceinline__ float bf_lo(unsigned u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 0xffff0000u); }
 
-template <int NT>
+// DD: also the rung-distance gradient dL/dd_k (off when the caller asks for
+// neither dtheta nor dd, e.g. a fixed alpha schedule).
+template <int NT, bool DD>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                      const __grid_constant__ QTileMaps tm, BwdArgs a, MmaLayout L) {
@@ -299,9 +301,12 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         }
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
         const float dp_lo = quad_sum(fmaf(c0, dt[0][0], fmaf(c1, dt[0][1], c7 * dt[1][0])));
-        const float ddp_lo = quad_sum(fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0])));
         const float dp_hi = quad_sum(fmaf(c0, dt[1][2], c1 * dt[1][3]));
-        const float ddp_hi = quad_sum(fmaf(df0, dt[1][2], df1 * dt[1][3]));
+        float ddp_lo = 0.f, ddp_hi = 0.f;
+        if constexpr (DD) {
+            ddp_lo = quad_sum(fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0])));
+            ddp_hi = quad_sum(fmaf(df0, dt[1][2], df1 * dt[1][3]));
+        }
         if (c4 == 0) {
             *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
             *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
@@ -427,9 +432,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         // interpolated score and far-minus-floor raw score of rows g4, g4+8
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
         const float si_lo = quad_sum(fmaf(c0, st[0][0], fmaf(c1, st[0][1], c7 * st[1][0])));
-        const float sd_lo = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
         const float si_hi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3]));
-        const float sd_hi = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
         const float dk = L.act_d[i];
         const bool okl = vlo && dk <= (float)qlo, okh = vhi && dk <= (float)qhi;
         const float2 dpl = *reinterpret_cast<const float2*>(dps[warp][i][g4]);
@@ -443,14 +446,18 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             if (vlo) { Pg[(size_t)slot * s.T + qlo] = p_lo; DSg[(size_t)slot * s.T + qlo] = ds_lo; }
             if (vhi) { Pg[(size_t)slot * s.T + qhi] = p_hi; DSg[(size_t)slot * s.T + qhi] = ds_hi; }
         }
-        // dL/dd_k of this warp's rows, in a fixed order over the rows
-        float g = 0.f;
-        if (c4 == 0)
-            g = p_lo * fmaf(s.scale * sd_lo, e_lo, ddp_lo) + p_hi * fmaf(s.scale * sd_hi, e_hi, ddp_hi);
-        g += __shfl_xor_sync(0xffffffffu, g, 4);
-        g += __shfl_xor_sync(0xffffffffu, g, 8);
-        g += __shfl_xor_sync(0xffffffffu, g, 16);
-        if (lane == 0) gsm[warp][k] = g;
+        if constexpr (DD) {
+            // far-minus-floor raw scores; dL/dd_k of this warp's rows, in a fixed order over the rows
+            const float sd_lo = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
+            const float sd_hi = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
+            float g = 0.f;
+            if (c4 == 0)
+                g = p_lo * fmaf(s.scale * sd_lo, e_lo, ddp_lo) + p_hi * fmaf(s.scale * sd_hi, e_hi, ddp_hi);
+            g += __shfl_xor_sync(0xffffffffu, g, 4);
+            g += __shfl_xor_sync(0xffffffffu, g, 8);
+            g += __shfl_xor_sync(0xffffffffu, g, 16);
+            if (lane == 0) gsm[warp][k] = g;
+        }
 
         // dShat_k as fp16 A fragment: the interpolation weights times dS of the row
         const unsigned afr[4] = {pack_f16(c0 * ds_lo, c1 * ds_lo), 0u, pack_f16(c7 * ds_lo, 0.f),
@@ -508,17 +515,19 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     }
 
     // ---- per-CTA rung partials, warps summed in a fixed order
-    __syncthreads();
-    float x = 0.f;
-    if (tid < a.r.K && ((a.r.active >> tid) & 1u))
-        for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
-    write_rung_partials(a, x);
+    if constexpr (DD) {
+        __syncthreads();
+        float x = 0.f;
+        if (tid < a.r.K && ((a.r.active >> tid) & 1u))
+            for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
+        write_rung_partials(a, x);
+    }
 }
 
 template <int NT>
 cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const QTileMaps& mt, const BwdArgs& a,
                       const MmaLayout& L, unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = bwd_query_mma_kernel<NT>;
+    auto kern = a.want_dd ? bwd_query_mma_kernel<NT, true> : bwd_query_mma_kernel<NT, false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mk, mv, mt, a, L);

@@ -382,7 +382,6 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     BwdArgs a;
     std::memset(&a, 0, sizeof(a));
     if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
-    if (!dtheta) return fail(FIBATTN_ERR_INVALID_ARG, "dtheta is NULL");
     if (!workspace) return fail(FIBATTN_ERR_INVALID_ARG, "workspace is NULL");
     if (B > 0 && (!q || (!k && !o.rotated_k) || !v || !lse || !dout || !dq || !dk || !dv))
         return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor pointer");
@@ -397,6 +396,7 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     char* ws = reinterpret_cast<char*>(workspace);
     a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.dout = dout; a.dq = dq; a.dk = dk; a.dv = dv;
     a.dtheta = dtheta; a.dd = dd;
+    a.want_dd = (dtheta || dd) ? 1 : 0;
     a.qt = ws + L.qt; a.kt = o.rotated_k ? o.rotated_k : ws + L.kt;
     a.P = reinterpret_cast<float*>(ws + L.P); a.DP = reinterpret_cast<float*>(ws + L.DP);
     a.Delta = reinterpret_cast<float*>(ws + L.Delta);
@@ -447,7 +447,7 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         if (e != cudaSuccess) return cuda_fail(e, "backward key-pass launch");
     }
     if (B == 0) {                                // no queries: every gradient is zero
-        e = cudaMemsetAsync(dtheta, 0, sizeof(float), st);
+        e = dtheta ? cudaMemsetAsync(dtheta, 0, sizeof(float), st) : cudaSuccess;
         if (e == cudaSuccess && dd && K > 0) e = cudaMemsetAsync(dd, 0, sizeof(float) * K, st);
         if (e != cudaSuccess) return cuda_fail(e, "zero gradients for an empty batch");
         return FIBATTN_OK;

@@ -61,7 +61,8 @@ struct BwdArgs {
     void* dq;                 // [B,H,T,D]
     void* dk;                 // [B,Hkv,T,D]
     void* dv;
-    float* dtheta;            // device scalar
+    float* dtheta;            // device scalar or nullptr
+    int want_dd;              // compute dL/dd_k (dtheta or dd requested)
     float* dd;                // device [K] or nullptr
     // workspace views
     void* qt;                 // rotated q [B,H,T,D]
@@ -225,7 +226,7 @@ __device__ __forceinline__ void convert_rung_sums(const BwdArgs& a, float* red, 
         if (a.dd) a.dd[t] = v;
     }
     __syncthreads();
-    if (t == 0) {
+    if (t == 0 && a.dtheta) {
         float da = 0.f;
         for (int k = 0; k < a.r.K; ++k) da += a.r.f[k] * red[k];
         *a.dtheta = da * (a.alpha - 0.5f) * (1.5f - a.alpha);

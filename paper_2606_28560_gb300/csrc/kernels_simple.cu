@@ -360,7 +360,7 @@ __global__ void __launch_bounds__(kThreads) bwd_query_kernel(BwdArgs a) {
             if (valid) x += tsm[u][k][0] - dsm[u] * tsm[u][k][1];
         }
     }
-    write_rung_partials(a, x);
+    if (a.want_dd) write_rung_partials(a, x);
 }
 
 // Key-centric pass.  Key row j of kv head hk receives, from every query head
@@ -373,7 +373,7 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
     grid_dependency_sync();
     __shared__ float red[kMaxRungs];
     __shared__ long long red64[(kThreads / 32) * kMaxRungs];
-    if (blockIdx.x == 0) convert_rung_sums(a, red, red64);
+    if (blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
     const Shape s = a.s;
     const int c = threadIdx.x & 3;
     const int tiles = (s.T + kRowsPerBlock - 1) / kRowsPerBlock;

@@ -97,9 +97,9 @@ def test_bwd_rejects_bad_arguments():
     f = np.array([1, 2, 3], dtype=np.float32)
     o = B.Opts(0.0, 0.0, 0, 0, 0, 0)
     ok_ptr = 16
-    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, None, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None, None,
+    rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, None, ok_ptr, ok_ptr, ok_ptr, ok_ptr, None, None, None,
                          1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
-    assert rc == 1 and "dtheta" in lib.fibattn_last_error().decode()
+    assert rc == 1 and "NULL" in lib.fibattn_last_error().decode()       # dv missing
     rc = lib.fibattn_bwd(ok_ptr, ok_ptr, ok_ptr, None, ok_ptr, ok_ptr, ok_ptr, ok_ptr, ok_ptr, 18, None,
                          1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 1, ctypes.byref(o), ok_ptr, 1 << 30, None)
     assert rc == 1

@@ -179,6 +179,24 @@ def test_rotated_keys_from_the_forward(dtype):
         assert torch.equal(a, b)
 
 
+@pytest.mark.parametrize("kernel", ["mma", "gather"])
+def test_backward_without_rung_gradients(kernel):
+    """dtheta = dd = NULL (a fixed schedule): the same dq, dk, dv, bit for bit,
+    without the rung-distance gradient."""
+    q, k, v = inputs.qkv(2, 4, 260, seed=61, dtype=torch.bfloat16, Hkv=2)
+    g = inputs.dout(2, 4, 260, seed=62, dtype=torch.bfloat16)
+    qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), g.cuda()
+    f = _offsets("fib", 15)
+    for alpha in (1.0, 0.83):
+        out, lse = fa.fwd(qc, kc, vc, alpha, f, 8)
+        full = fa.bwd(qc, kc, vc, lse, gc, alpha, f, 8, out=out, kernel=kernel)
+        lean = fa.bwd(qc, kc, vc, lse, gc, alpha, f, 8, out=out, kernel=kernel, rung_grads=False)
+        torch.cuda.synchronize()
+        assert lean[3] is None and lean[4] is None
+        for a, b in zip(full[:3], lean[:3]):
+            assert torch.equal(a, b)
+
+
 def test_empty_batch():
     q = torch.zeros((0, 2, 16, 64), device="cuda")
     out, lse = fa.fwd(q, q, q, 1.0, _offsets("fib", 15), 4)
