@@ -303,12 +303,13 @@ def run_gpu(args, rank, world, device):
                    "algo_GBps": round(algo.get(k, 0) / (v[0] / max(v[1], 1) / 1e3) / 1e9, 1) if v[0] > 0 else None}
                for k, v in prof.items()}
 
-    # forward only at the same shape (W sweep), graphed the same way
+    # forward only at the same shape (W sweep): layer time from a graph without
+    # profiling nodes, the forward kernel's time from a profiled capture
     fwd_sweep = {}
     for W_ in (6, 8, 10, 12):
         wl.fwd_only(W_)
         torch.cuda.synchronize(device)
-        gf = capture(lambda: wl.fwd_only(W_), device)
+        gf = capture(lambda: wl.fwd_only(W_), device, profile=False)
         for _ in range(2):
             gf.replay()
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
@@ -318,17 +319,22 @@ def run_gpu(args, rank, world, device):
             gf.replay()
         a1.record(stream)
         torch.cuda.synchronize(device)
+        layer_us = a0.elapsed_time(a1) / (reps * L) * 1e3
+        del gf
+        gp = capture(lambda: wl.fwd_only(W_), device, profile=True)
+        for _ in range(2):
+            gp.replay()
+        torch.cuda.synchronize(device)
         p = profile_summary()
         profile_enable(False)
+        del gp
         fms, fcnt = p.get("fwd", (0.0, 1))
         us = fms / max(fcnt, 1) * 1e3
-        layer_us = a0.elapsed_time(a1) / (reps * L) * 1e3
         cbytes = 4 * B * H * T * ROW_BYTES
         fwd_sweep[f"W{W_}"] = {"fwd_kernel_us": round(us, 2), "layer_us_incl_rope": round(layer_us, 2),
                                "compulsory_GBps": round(cbytes / (layer_us * 1e-6) / 1e9, 1),
                                "frac_of_hbm": round(cbytes / (layer_us * 1e-6) / 1e9 / hbm, 4),
                                "fwd_kernel_frac_of_hbm": round(cbytes / (us * 1e-6) / 1e9 / hbm, 4)}
-        del gf
 
     # the integer path: alpha = 1 in every layer, with and without dL/dtheta
     integer = {}
@@ -349,11 +355,49 @@ def run_gpu(args, rank, world, device):
     integer["interpolated_over_integer"] = round(integer["learned_alpha_ms_per_step"] /
                                                  integer["alpha1_with_dtheta"]["ms_per_step"], 3)
 
+    gqa = run_gqa_forward(wl, device, args, stream)
     e2e = run_e2e(args, wl, device, dist)
     stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
                 algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
-                stack=stack, integer=integer)
+                stack=stack, integer=integer, gqa=gqa)
+
+
+def run_gqa_forward(wl, device, args, stream):
+    """The forward of the 16 layers at the paper's head split (H = 8 query
+    heads, Hkv = 2 kv heads; groups of 4 share each CTA's staged keys and
+    values), same B, T, W and schedule as the step, graphed."""
+    import paper_2606_28560_gb300 as fa
+    from paper_2606_28560_gb300 import inputs
+    Hkv = 2
+    kv = []
+    for l in range(L):
+        k = torch.empty((B, Hkv, T, D), dtype=torch.bfloat16, device=device)
+        v = torch.empty((B, Hkv, T, D), dtype=torch.bfloat16, device=device)
+        inputs.device_normal_(k, 5000 + 2 * l)
+        inputs.device_normal_(v, 5001 + 2 * l)
+        kv.append((k, v, torch.empty((B, Hkv, T, D), dtype=torch.float16, device=device)))
+
+    def fwd_all():
+        for l in range(L):
+            k, v, rk = kv[l]
+            fa.fwd(wl.q[l], k, v, wl.alphas[l], wl.f, W, out=wl.out[l], lse=wl.lse[l], workspace=wl.ws_f,
+                   rotated_k=rk)
+
+    g = capture(fwd_all, device, profile=False)
+    for _ in range(2):
+        g.replay()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(3, args.steps // 3)
+    a0.record(stream)
+    for _ in range(reps):
+        g.replay()
+    a1.record(stream)
+    torch.cuda.synchronize(device)
+    layer_us = a0.elapsed_time(a1) / (reps * L) * 1e3
+    del g, kv
+    return {"B": B, "H": H, "Hkv": Hkv, "T": T, "W": W, "layer_us_incl_rope": round(layer_us, 2),
+            "query_heads_per_s": round(B * H * T / (layer_us * 1e-6), 1)}
 
 
 def run_autograd_stack(device, warm=2, reps=3):
@@ -574,6 +618,7 @@ def main():
             "forward_only_B16H8T1024": r["fwd_sweep"],
             "autograd_stack_16_layers": r["stack"],
             "integer_vs_interpolated_16_layers": r["integer"],
+            "forward_gqa_16_layers": r["gqa"],
             "cpu_baseline": cpu,
             "e2e": r["e2e"],
             "gpu_launches": r["launches"],

@@ -45,8 +45,13 @@ constexpr float kLn2 = 0.6931471805599453f;
 constexpr int kWarps = kMmaWarps;
 constexpr int kRowsPerWarp = 15;                 // useful query rows of a 16-row tile
 
-template <int NT>
-__global__ void __launch_bounds__(kWarps * 32, 2)
+// TEAMS = 1: a CTA of 8 warps computes one query head's tile; keys and then
+// values are staged into one buffer.  TEAMS = 2 (grouped-query attention): a
+// CTA of 16 warps owns a kv head's tile; keys and values are staged once, into
+// two buffers, and each team of 8 warps loops over its share of the group's
+// query heads (team t takes heads t, t + 2, ...).
+template <int NT, int TEAMS>
+__global__ void __launch_bounds__(kWarps * 32 * TEAMS, TEAMS == 1 ? 2 : 1)
 fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                FwdArgs a, MmaLayout L) {
     grid_dependency_sync();
@@ -54,29 +59,37 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[2];
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
-    const unsigned sbase = smem_u32(buf);
+    unsigned char* vbuf = TEAMS == 1 ? buf : buf + (size_t)L.rows * 128;
+    const unsigned sbase = smem_u32(buf), vbase = smem_u32(vbuf);
 
     const Shape s = a.s;
     const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
-    const int bh = blockIdx.x / tiles;
+    const int unit = blockIdx.x / tiles;          // query head (b H + h), or kv head (b Hkv + hk) for TEAMS = 2
     const int i0 = (blockIdx.x % tiles) * kMmaTile;
-    const int b = bh / s.H, h = bh % s.H, hk = h / s.G;
+    const int b = TEAMS == 1 ? unit / s.H : unit / s.Hkv;
+    const int hk = TEAMS == 1 ? (unit % s.H) / s.G : unit % s.Hkv;
     const int head = b * s.Hkv + hk;
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int tid = threadIdx.x, lane = tid & 31, warp = (tid >> 5) % kWarps, team = (tid >> 5) / kWarps;
     const int g4 = lane >> 2, c4 = lane & 3;
     const int wrel = warp * kRowsPerWarp;         // tile-relative first row of this warp
     const int bw = i0 + wrel;                     // absolute first row
 
-    // ---- issue the key copies (warp 0)
+    // ---- issue the key copies (and for TEAMS = 2 the value copies) (warp 0)
     if (tid == 0) {
         mbar_init(&bars[0], 1);
         mbar_init(&bars[1], 1);
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
-    if (warp == 0) {
+    if (tid < 32) {
         __syncwarp();
         issue_rows(buf, &tmK.m64, &tmK.m8, L, i0, head, &bars[0], lane);
+        if (TEAMS == 2) issue_rows(vbuf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
     }
+    __syncthreads();                              // barrier init visible
+
+#pragma unroll 1
+    for (int hq = TEAMS == 1 ? 0 : team; hq < (TEAMS == 1 ? 1 : s.G); hq += TEAMS) {
+    const int bh = TEAMS == 1 ? unit : b * s.H + hk * s.G + hq;
 
     // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32)
     // Thread dims: 16kc + 2c4 + {0,1} and 16kc + 8 + 2c4 + {0,1} for kc = 0..3.
@@ -139,7 +152,6 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
     const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
 
-    __syncthreads();                              // barrier init visible
     const bool ok_k = mbar_wait(&bars[0], 0);
 
     // ---- window band scores: keys [bw - Wp, bw + 16), n-tile j covers 8 keys
@@ -217,10 +229,12 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         mhi = fmaxf(mhi, rs[k][1]);
     }
 
-    // ---- all warps are done with the keys: stage the values into the same buffer
-    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-    __syncthreads();
-    if (warp == 0) issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
+    if (TEAMS == 1) {
+        // ---- all warps are done with the keys: stage the values into the same buffer
+        asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+        __syncthreads();
+        if (warp == 0) issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
+    }
 
     // ---- probabilities (unnormalised, row max -> exactly 1) while values arrive
     if (mlo == -INFINITY) mlo = 0.f;              // rows beyond T: keep arithmetic finite
@@ -253,7 +267,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
+            ldsm_x4_t(row_chunk(vbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
             mma_bf16_16816(o[n], afr, b0, b1);
             mma_bf16_16816(o[n + 1], afr, b2, b3);
         }
@@ -264,7 +278,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
         for (int n = 0; n < 8; n += 4) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 3)), b0, b1, b2, b3);
+            ldsm_x4_t(row_chunk(vbase, vrow, n + (lane >> 3)), b0, b1, b2, b3);
             mma_bf16_1688(o[n], pa[kk][0], pa[kk][1], b0);
             mma_bf16_1688(o[n + 1], pa[kk][0], pa[kk][1], b1);
             mma_bf16_1688(o[n + 2], pa[kk][0], pa[kk][1], b2);
@@ -292,7 +306,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
+            ldsm_x4_t(row_chunk(vbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
             mma_bf16_16816(o[n], ahi, b0, b1);
             mma_bf16_16816(o[n + 1], ahi, b2, b3);
         }
@@ -317,17 +331,18 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][2] * inv_hi, o[n][3] * inv_hi);
         if (c4 == 0) a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
     }
+    }                                             // query heads of the group
 }
 
 // ------------------------------------------------------------ host side ----
 
-template <int NT>
+template <int NT, int TEAMS>
 cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const FwdArgs& a, const MmaLayout& L,
                       unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = fwd_mma_kernel<NT>;
+    auto kern = fwd_mma_kernel<NT, TEAMS>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mk, mv, a, L);
+    return launch_kernel(kern, dim3(grid), dim3(kWarps * 32 * TEAMS), smem, st, mk, mv, a, L);
 }
 
 }  // namespace
@@ -358,6 +373,8 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
 }
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.buf_rows * 128 + 1024; }
+
+size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - 64; }
 
 namespace {
 
@@ -507,18 +524,29 @@ bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, siz
 
 cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st) {
     const long long tiles = (a.s.T + kMmaTile - 1) / kMmaTile;
-    const long long grid = tiles * a.s.B * a.s.H;
-    if (grid <= 0) return cudaSuccess;
     RowMaps mk, mv;
     const int heads = a.s.B * a.s.Hkv;
+    if (tiles * a.s.B * a.s.H <= 0) return cudaSuccess;
     if (!encode_row_maps(&mk, a.kt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
         !encode_row_maps(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
         return cudaErrorInvalidValue;
+    // Grouped-query attention: one CTA per kv head's tile with both staged
+    // tensors resident, when they fit.
+    const size_t smem2 = 2 * (size_t)L.rows * 128 + 1024;
+    if (a.s.G >= 2 && smem2 <= fwd_mma_gqa_smem_limit()) {
+        const unsigned grid = (unsigned)(tiles * heads);
+        switch (L.nt) {
+        case 2: return launch_nt<2, 2>(mk, mv, a, L, grid, smem2, st);
+        case 3: return launch_nt<3, 2>(mk, mv, a, L, grid, smem2, st);
+        default: return launch_nt<4, 2>(mk, mv, a, L, grid, smem2, st);
+        }
+    }
+    const unsigned grid = (unsigned)(tiles * a.s.B * a.s.H);
     const size_t smem = fwd_mma_smem_bytes(L);
     switch (L.nt) {
-    case 2: return launch_nt<2>(mk, mv, a, L, (unsigned)grid, smem, st);
-    case 3: return launch_nt<3>(mk, mv, a, L, (unsigned)grid, smem, st);
-    default: return launch_nt<4>(mk, mv, a, L, (unsigned)grid, smem, st);
+    case 2: return launch_nt<2, 1>(mk, mv, a, L, grid, smem, st);
+    case 3: return launch_nt<3, 1>(mk, mv, a, L, grid, smem, st);
+    default: return launch_nt<4, 1>(mk, mv, a, L, grid, smem, st);
     }
 }
 

@@ -54,6 +54,9 @@ bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, siz
 // the first key of a tile (win_smem: relative row 0; rung_smem[k]: row s0_k).
 bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
 size_t fwd_mma_smem_bytes(const MmaLayout& L);
+// Dynamic shared memory a grouped-query forward CTA may use (keys and values
+// both resident).
+size_t fwd_mma_gqa_smem_limit();
 // 3-D tensor map [heads][T][64] of 2-byte rows, boxes of box_rows rows,
 // 128-byte swizzle; rows outside [0, T) read as zero.
 bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt, int T, int heads, int box_rows);

@@ -266,6 +266,21 @@ def test_config4_bf16_backward_learned_alpha():
             check_bwd(q, k, v, g, float(alphas[layer]), f, 8, kernel="gather")
 
 
+def test_gqa_paper_shape_fwd_bwd():
+    """The paper's head split (H = 8 query heads, Hkv = 2 kv heads: groups of
+    4 sharing staged keys and values), B = 4, T = 1024, W = 8, learned alpha:
+    forward and backward against the oracle in full."""
+    theta = inputs.theta_learned(16, seed=3)
+    alphas = fa.alpha_schedule("learned", 16, theta=theta)
+    f = _offsets("fib", 15)
+    for layer in (2, 11):
+        s = inputs.layer_seed(5, layer)
+        q, k, v = inputs.qkv(4, 8, 1024, seed=s, dtype=torch.bfloat16, Hkv=2)
+        g = inputs.dout(4, 8, 1024, seed=s, dtype=torch.bfloat16)
+        check_fwd(q, k, v, float(alphas[layer]), f, 8)
+        check_bwd(q, k, v, g, float(alphas[layer]), f, 8, kernel="mma")
+
+
 @pytest.mark.parametrize("base,K", [("fib", 15), ("pow2", 10)])
 def test_config5_bf16_long_stress(base, K):
     """B=2 H=8 T=16384 W=12, linear stagger, Fibonacci vs power-of-2 base:
