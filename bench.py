@@ -219,6 +219,36 @@ def algorithmic_bytes():
     }
 
 
+# DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch,
+# from an `ncu --set full` capture of `bench.py --ncu-case bwd` (B=32, the same
+# H, T, D, W); every launch reads and writes each of its tensors once, so the
+# bytes scale with B.  The counters belong to the sources hashed here: once a
+# file of the kernel changes, the figure is reported as null until the next
+# capture.
+NCU_TRAFFIC = {
+    "bwd_query_mma": {"bytes_at_b32": 169047552 + 73504768,
+                      "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
+                      "sha256": "1d0b53c2b14bffabbce8a4e0e9e9af35c77db54b53349cbfedd61397a0ad6a5e"},
+}
+
+
+def sources_sha256(names) -> str:
+    import hashlib
+    h = hashlib.sha256()
+    for n in names:
+        with open(os.path.join(ROOT, "paper_2606_28560_gb300", "csrc", n), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def ncu_traffic(kernel: str):
+    """Per-launch DRAM bytes of `kernel` at the bench's B, or None."""
+    e = NCU_TRAFFIC.get(kernel)
+    if e is None or sources_sha256(e["sources"]) != e["sha256"]:
+        return None
+    return round(e["bytes_at_b32"] * B / 32)
+
+
 def capture(fn, device, profile=True):
     """Capture fn() (library launches on torch's current stream) into a CUDA
     graph.  With profile, the library's per-kernel events become event nodes of
@@ -612,7 +642,7 @@ def main():
                       "per-kernel times from a second capture of the step with event nodes around each kernel",
             "roofline": {"bound": "hbm", "kernel": r["dom"], "achieved": round(r["achieved"], 1),
                          "peak": r["hbm"], "unit": "GB/s", "frac": round(r["achieved"] / r["hbm"], 4),
-                         "traffic": None, "peak_source": r["peak_kind"],
+                         "traffic": ncu_traffic(r["dom"]), "peak_source": r["peak_kind"],
                          "algorithmic_bytes_per_launch": r["algo"].get(r["dom"])},
             "kernels": r["kernels"],
             "forward_only_B16H8T1024": r["fwd_sweep"],
