@@ -164,6 +164,11 @@ class Workload:
         self.out = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
         # rotated keys of each layer, written by its forward and read by its backward
         self.rk = [torch.empty(shp, dtype=torch.float16, device=device) for _ in range(layers)]
+        # forward residuals of each layer (rotated q, p per slot, rung score
+        # differences), read by its backward instead of recomputing the scores
+        self.res = [torch.empty(fa.residual_bytes(B, H, T, W, K, bf), dtype=torch.uint8, device=device)
+                    for _ in range(layers)]
+        self.use_res = True
         self.lse = [torch.empty((B, H, T), dtype=torch.float32, device=device) for _ in range(layers)]
         self.dq = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
         self.dk = [torch.empty(shp, dtype=bf, device=device) for _ in range(layers)]
@@ -173,15 +178,18 @@ class Workload:
         self.ws_f = torch.empty(fa.fwd_workspace_bytes(B, H, T, W, K, bf), dtype=torch.uint8, device=device)
         self.ws_b = torch.empty(fa.bwd_workspace_bytes(B, H, T, W, K, bf), dtype=torch.uint8, device=device)
 
+    def _res(self, l):
+        return self.res[l] if self.use_res else None
+
     def step(self):
         fa = self.fa
         for l in range(self.L):
             fa.fwd(self.q[l], self.k[l], self.v[l], self.alphas[l], self.f, W, out=self.out[l], lse=self.lse[l],
-                   workspace=self.ws_f, rotated_k=self.rk[l])
+                   workspace=self.ws_f, rotated_k=self.rk[l], residuals=self._res(l))
         for l in reversed(range(self.L)):
             fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], self.alphas[l], self.f, W,
                    out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], dtheta=self.dth[l],
-                   dd=self.dd[l], workspace=self.ws_b, rotated_k=self.rk[l])
+                   dd=self.dd[l], workspace=self.ws_b, rotated_k=self.rk[l], residuals=self._res(l))
 
     def step_fixed(self, rung_grads: bool):
         """The same step at alpha = 1 in every layer (integer rung distances);
@@ -189,12 +197,12 @@ class Workload:
         fa = self.fa
         for l in range(self.L):
             fa.fwd(self.q[l], self.k[l], self.v[l], 1.0, self.f, W, out=self.out[l], lse=self.lse[l],
-                   workspace=self.ws_f, rotated_k=self.rk[l])
+                   workspace=self.ws_f, rotated_k=self.rk[l], residuals=self._res(l))
         for l in reversed(range(self.L)):
             fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], 1.0, self.f, W,
                    out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l],
                    dtheta=self.dth[l] if rung_grads else None, dd=self.dd[l] if rung_grads else None,
-                   workspace=self.ws_b, rotated_k=self.rk[l], rung_grads=rung_grads)
+                   workspace=self.ws_b, rotated_k=self.rk[l], rung_grads=rung_grads, residuals=self._res(l))
 
     def fwd_only(self, W_):
         fa = self.fa
@@ -203,19 +211,32 @@ class Workload:
                    workspace=self.ws_f, rotated_k=self.rk[l])
 
 
-def algorithmic_bytes():
+def algorithmic_bytes(residuals=True):
     """Bytes each kernel must move once per launch (bf16 rows of 128 B,
-    fp32 lse and fp32 P / dS slots).  S = W + 1 + K slots per query."""
+    fp32 lse and fp32 P / dS slots).  S = W + 1 + K slots per query.  With
+    the forward residuals the forward also writes q~ (fp16 rows), p per slot
+    and the rung score differences, and the query pass reads those instead of
+    q, lse and the rotated keys' scores."""
     n = B * H * T
     S = W + 1 + K
     rows = n * ROW_BYTES
+    if residuals:
+        return {
+            # Q, K~, V read; O, q~ written; lse, p per slot, sd written
+            "fwd": 5 * rows + 4 * n + 4 * n * S + 4 * n * K,
+            "rope_k": 2 * rows,
+            # dO, O, K~, V read; dQ written; p, sd read; dS written
+            "bwd_query_mma": 5 * rows + 2 * 4 * n * S + 4 * n * K,
+            "bwd_key_mma": 4 * rows + 2 * 4 * n * S,       # Q~ dO read, dK dV written, P/dS read
+        }
     return {
         "fwd": 4 * rows + 4 * n,                           # Q, K~, V read; O written; lse
         "rope_k": 2 * rows, "rope_q": 2 * rows,            # read, write rotated
         "bwd_query": 5 * rows + 4 * n + 2 * 4 * n * S,     # Q~ K~ V dO read, dQ written, lse, P/dS written
-        # Q, dO, O, K~, V read; dQ, Q~ written; lse read, Delta written; P/dp written
-        "bwd_query_mma": 7 * rows + 2 * 4 * n + 2 * 4 * n * S,
+        # Q, dO, O, K~, V read; dQ, Q~ written; lse read; P/dS written
+        "bwd_query_mma": 7 * rows + 4 * n + 2 * 4 * n * S,
         "bwd_key": 4 * rows + 2 * 4 * n * S,               # Q~ dO read, dK dV written, P/dS read
+        "bwd_key_mma": 4 * rows + 2 * 4 * n * S,
     }
 
 
@@ -385,12 +406,30 @@ def run_gpu(args, rank, world, device):
     integer["interpolated_over_integer"] = round(integer["learned_alpha_ms_per_step"] /
                                                  integer["alpha1_with_dtheta"]["ms_per_step"], 3)
 
+    # the same step with a backward that recomputes the scores (no residuals)
+    wl.use_res = False
+    gr = capture(wl.step, device, profile=False)
+    for _ in range(2):
+        gr.replay()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    reps = max(3, args.steps // 3)
+    a0.record(stream)
+    for _ in range(reps):
+        gr.replay()
+    a1.record(stream)
+    torch.cuda.synchronize(device)
+    wl.use_res = True
+    del gr
+    recompute = {"ms_per_step": round(a0.elapsed_time(a1) / reps, 4),
+                 "residuals_ms_per_step": round(ms_max / args.steps, 4)}
+    recompute["residuals_speedup"] = round(recompute["ms_per_step"] / recompute["residuals_ms_per_step"], 3)
+
     gqa = run_gqa_forward(wl, device, args, stream)
     e2e = run_e2e(args, wl, device, dist)
     stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
                 algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
-                stack=stack, integer=integer, gqa=gqa)
+                stack=stack, integer=integer, gqa=gqa, recompute=recompute)
 
 
 def run_gqa_forward(wl, device, args, stream):
@@ -573,7 +612,10 @@ def run_reference(args, rank, world):
 def ncu_case(which: str):
     """A small fixed case for ncu captures of one kernel: B=32 H=8 T=1024 W=8,
     two layers of distinct buffers (Q, K, V, O of one layer = 134 MB, larger
-    than L2), one forward (and backward) per layer after one warm-up pass."""
+    than L2), one forward (and backward) per layer after one warm-up pass, the
+    path the bench times: the forward keeps its rotated keys and residuals,
+    the backward reads them (per layer and pass: RoPE of k, forward, query
+    pass, key pass)."""
     import __graft_entry__
     __graft_entry__.build()
     import paper_2606_28560_gb300 as fa
@@ -586,12 +628,12 @@ def ncu_case(which: str):
         ts = [torch.empty((Bc, H, T, D), dtype=torch.bfloat16, device=dev) for _ in range(4)]
         for j, t in enumerate(ts):
             inputs.device_normal_(t, 1000 + 10 * l + j)
-        bufs.append(ts)
+        bufs.append(ts + [fa.residuals_like(ts[0], W, K), fa.rotated_k_like(ts[1])])
     for rep in range(2):
-        for l, (q, k, v, g) in enumerate(bufs):
-            out, lse = fa.fwd(q, k, v, 0.8 + 0.1 * l, f, W)
+        for l, (q, k, v, g, res, rk) in enumerate(bufs):
+            out, lse = fa.fwd(q, k, v, 0.8 + 0.1 * l, f, W, residuals=res, rotated_k=rk)
             if which == "bwd":
-                fa.bwd(q, k, v, lse, g, 0.8 + 0.1 * l, f, W, out=out)
+                fa.bwd(q, k, v, lse, g, 0.8 + 0.1 * l, f, W, out=out, residuals=res, rotated_k=rk)
     torch.cuda.synchronize(dev)
     print(f"ncu case {which} done")
 
@@ -648,6 +690,7 @@ def main():
             "forward_only_B16H8T1024": r["fwd_sweep"],
             "autograd_stack_16_layers": r["stack"],
             "integer_vs_interpolated_16_layers": r["integer"],
+            "backward_recomputing_scores_16_layers": r["recompute"],
             "forward_gqa_16_layers": r["gqa"],
             "cpu_baseline": cpu,
             "e2e": r["e2e"],

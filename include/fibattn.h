@@ -19,6 +19,8 @@
  *     (the base sequence f_k, e.g. 1,2,3,5,...,987) read during the call only.
  *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default stream).
  *     Device work is asynchronous on that stream; a call returns after launch.
+ *     Work goes to the calling thread's current device; a compute call makes
+ *     that device's primary context current on the thread if none is.
  *   - Return value is a fibattn_status.  Argument errors are reported before
  *     any launch.  Faults raised asynchronously by the device surface at the
  *     caller's next synchronisation.  fibattn_last_error() gives a thread-local
@@ -73,6 +75,26 @@ typedef struct {
                           them from there instead of rotating k again (k may then
                           be NULL): a caller that keeps this buffer from the
                           forward to the backward keeps it in place of k. */
+    void* residuals;   /* optional device buffer of fibattn_residual_bytes(...) bytes,
+                          16-byte aligned [NULL].  Given it, fibattn_fwd also writes
+                          what the backward would otherwise recompute from q and k:
+                          the RoPE-rotated queries (fp16 [B][H][T][D]), the
+                          softmax probability of every slot (fp32 [B][H][S][T],
+                          S = W + 1 + K: window distances 0..W, then rung k at
+                          W + 1 + k; 0 where not attended; rungs that are never
+                          read -- dropped by dedup or beyond T's reach -- are
+                          left unwritten) and the far-minus-floor raw score
+                          q~ . (k~_far - k~_floor) of every rung (fp32
+                          [B][H][K][T]); the three arrays follow one another in
+                          that order, each starting at the next multiple of 256
+                          bytes.  Only the tensor-core forward writes them:
+                          bf16 I/O, and fwd_kernel 0 or 3 with its layout applying;
+                          otherwise fibattn_fwd fails with FIBATTN_ERR_UNSUPPORTED
+                          before any launch.  fibattn_bwd given the buffer filled by
+                          the forward of the same inputs and parameters reads them
+                          in its tensor-core passes instead of recomputing the
+                          scores; when its tensor-core passes do not apply it
+                          ignores the buffer. */
 } fibattn_opts;
 
 /* ---------------------------------------------------------------------------
@@ -119,6 +141,10 @@ int fibattn_bwd(const void* q, const void* k, const void* v,
                 int dtype, const fibattn_opts* opts,
                 void* workspace, size_t workspace_bytes, void* stream);
 
+/* Bytes of the forward residuals (fibattn_opts.residuals) for these sizes;
+ * 0 for invalid sizes or fp32 I/O (no residuals). */
+size_t fibattn_residual_bytes(int B, int H, int T, int D, int W, int K, int dtype);
+
 /* Thread-local message for the last non-OK status returned on this thread. */
 const char* fibattn_last_error(void);
 
@@ -157,6 +183,26 @@ int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, floa
  * ------------------------------------------------------------------------- */
 int fibattn_coverage(int L, const float* alphas, const float* offsets, int K, int W, int T, int no_dedup,
                      int* per_layer, int* union_count, int* beyond_window, int* two_hop);
+
+/* ---------------------------------------------------------------------------
+ * Shared-memory staging layout of the tensor-core kernels (host-side, no GPU;
+ * a diagnostic without counterpart in the paper).  A CTA of these kernels owns
+ * a tile of 120 consecutive queries (kind 0: the forward and the backward
+ * query pass) or keys (kind 1: the backward key pass) and stages the rows its
+ * warps read: for kind 0 the window band [-Wp, 121) and, per staged rung k,
+ * the slab [-s0_k - 1, 121 - s0_k) relative to the tile's first query (Wp =
+ * 0, 8 or 16 for W = 0, <= 8, <= 16); for kind 1 the band [0, 121 + Wp) and
+ * the slabs [s0_k, s0_k + 121) relative to the first key.  Overlapping row
+ * ranges are merged and each merged interval is rounded up to whole 8-row
+ * copies.  Outputs (host arrays of at least 17 ints, any may be NULL):
+ * n_iv intervals with relative first row iv_start, row count iv_len and first
+ * shared row iv_smem; slab_row[k] (K ints) = shared row of the first row of
+ * rung k's slab, -1 when the rung is not staged (dropped by dedup or beyond
+ * T's reach).  FIBATTN_ERR_UNSUPPORTED when the tensor-core kernels do not
+ * apply (W > 16 or K > 16).
+ * ------------------------------------------------------------------------- */
+int fibattn_staging_layout(int kind, int T, int W, float alpha, const float* offsets, int K, int no_dedup,
+                           int* n_iv, int* iv_start, int* iv_len, int* iv_smem, int* slab_row);
 
 /* ---------------------------------------------------------------------------
  * Forward without a caller-provided workspace.  The paper has no counterpart;

@@ -4,11 +4,12 @@ from ``csrc/`` and exposed through the C ABI of ``include/fibattn.h``; this
 package only marshals arguments to it.
 """
 from .binding import (FibattnError, alpha_schedule, base, bwd, bwd_workspace_bytes, coverage, fwd,  # noqa: F401
-                      fwd_workspace_bytes, lib, library_path, rotated_k_like, rung_params)
+                      fwd_workspace_bytes, lib, library_path, residual_bytes, residual_views, residuals_like,
+                      rotated_k_like, rung_params, staging_layout)
 from .autograd import (FibAttention, FibAttentionFunction, alpha_of_theta, attention_stack,  # noqa: F401
                        fib_attention, theta_of_alpha)
 
 __all__ = ["fwd", "bwd", "fwd_workspace_bytes", "bwd_workspace_bytes", "rung_params", "base",
            "alpha_schedule", "lib", "library_path", "FibattnError", "rotated_k_like", "FibAttention",
            "FibAttentionFunction", "fib_attention", "attention_stack", "alpha_of_theta", "theta_of_alpha",
-           "coverage"]
+           "coverage", "residual_bytes", "residuals_like", "residual_views", "staging_layout"]

@@ -5,7 +5,9 @@ with the model through this attention (arXiv 2606.28560, Section 2, "The
 per-layer scalar" and "Implementation note").  `FibAttentionFunction` runs
 `fibattn_fwd` and `fibattn_bwd`; the forward keeps the RoPE-rotated keys for
 the backward (in place of k, the same size), so the backward does not rotate
-k again.  alpha is a host value of the C ABI -- the kernels' shared-memory
+k again, and with bf16 I/O also its residuals (the rotated queries, p of every
+attended slot and the rung score differences), so the backward does not
+recompute the scores.  alpha is a host value of the C ABI -- the kernels' shared-memory
 layout depends on the rung distances -- so a theta held on the GPU is read
 once per call.
 """
@@ -32,17 +34,32 @@ class FibAttentionFunction(torch.autograd.Function):
     def forward(ctx, q, k, v, theta, offsets, W, rope_base, scale, dedup):
         alpha = alpha_of_theta(float(theta))
         rk = B.rotated_k_like(k)
-        out, lse = B.fwd(q, k, v, alpha, offsets, W, rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk)
-        ctx.save_for_backward(q, k, v, out, lse, rk)
+        kw = dict(rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk)
+        res = None
+        if q.dtype == torch.bfloat16:
+            # the tensor-core forward also keeps p, the rung score differences and
+            # the rotated queries, so the backward does not recompute the scores
+            res = B.residuals_like(q, W, len(offsets))
+            try:
+                out, lse = B.fwd(q, k, v, alpha, offsets, W, residuals=res, **kw)
+            except B.FibattnError as e:
+                if e.status != B.FIBATTN_ERR_UNSUPPORTED:
+                    raise
+                res = None
+        if res is None:
+            out, lse = B.fwd(q, k, v, alpha, offsets, W, **kw)
+            res = torch.empty(0, dtype=torch.uint8, device=q.device)
+        ctx.save_for_backward(q, k, v, out, lse, rk, res)
         ctx.args = (alpha, offsets, W, rope_base, scale, dedup, theta.dtype, theta.device)
         return out
 
     @staticmethod
     def backward(ctx, dout):
-        q, k, v, out, lse, rk = ctx.saved_tensors
+        q, k, v, out, lse, rk, res = ctx.saved_tensors
         alpha, offsets, W, rope_base, scale, dedup, tdtype, tdev = ctx.args
         dq, dk, dv, dth, _ = B.bwd(q, k, v, lse, dout.contiguous(), alpha, offsets, W, out=out,
-                                   rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk)
+                                   rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk,
+                                   residuals=res if res.numel() else None)
         dtheta = dth.reshape(()).to(device=tdev, dtype=tdtype)
         return dq, dk, dv, dtheta, None, None, None, None, None
 

@@ -18,6 +18,7 @@ from . import build as _build
 
 FIBATTN_F32 = 0
 FIBATTN_BF16 = 1
+FIBATTN_ERR_UNSUPPORTED = 2
 _STATUS = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "CUDA", 4: "INTERNAL"}
 
 _lock = threading.Lock()
@@ -33,7 +34,7 @@ class FibattnError(RuntimeError):
 class Opts(ctypes.Structure):
     _fields_ = [("rope_base", ctypes.c_float), ("scale", ctypes.c_float),
                 ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int), ("fwd_kernel", ctypes.c_int),
-                ("bwd_kernel", ctypes.c_int), ("rotated_k", ctypes.c_void_p)]
+                ("bwd_kernel", ctypes.c_int), ("rotated_k", ctypes.c_void_p), ("residuals", ctypes.c_void_p)]
 
 
 def library_path() -> str:
@@ -70,6 +71,8 @@ def lib():
             L.fibattn_base.restype = ci
             L.fibattn_alpha_schedule.argtypes = [ci, ci, fp, ci, fp]
             L.fibattn_alpha_schedule.restype = ci
+            L.fibattn_residual_bytes.argtypes = [ci] * 7
+            L.fibattn_residual_bytes.restype = sz
             _lib = L
     return _lib
 
@@ -92,10 +95,52 @@ BWD_KERNELS = {"auto": 0, "gather": 1, "mma": 2}
 
 
 def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto", bwd_kernel="auto",
-          rotated_k=None) -> Opts:
+          rotated_k=None, residuals=None) -> Opts:
     return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1,
                 FWD_KERNELS[fwd_kernel], BWD_KERNELS[bwd_kernel],
-                rotated_k.data_ptr() if rotated_k is not None else None)
+                rotated_k.data_ptr() if rotated_k is not None else None,
+                residuals.data_ptr() if residuals is not None else None)
+
+
+def residual_bytes(B, H, T, W, K, dtype=torch.bfloat16, D=64) -> int:
+    """Size of the forward residuals (``residuals=``); 0 for fp32 I/O."""
+    code = FIBATTN_BF16 if dtype == torch.bfloat16 else FIBATTN_F32
+    return int(lib().fibattn_residual_bytes(B, H, T, D, W, K, code))
+
+
+def residuals_like(q: torch.Tensor, W: int, K: int) -> torch.Tensor:
+    """A buffer for the forward residuals of queries like q (bf16 I/O): the
+    forward fills it, the backward of the same inputs reads it."""
+    B, H, T, D = q.shape
+    n = residual_bytes(B, H, T, W, K, q.dtype, D)
+    if n == 0:
+        raise ValueError("forward residuals need bf16 I/O")
+    return torch.empty(n, dtype=torch.uint8, device=q.device)
+
+
+def residual_views(res: torch.Tensor, B, H, T, W, K):
+    """Views of a residual buffer: rotated q (fp16 [B,H,T,64]), p per slot
+    (fp32 [B,H,W+1+K,T]) and far-minus-floor rung scores (fp32 [B,H,K,T]);
+    the arrays follow one another, each from the next multiple of 256 bytes."""
+    def up(x):
+        return (x + 255) // 256 * 256
+    n = B * H * T
+    S = W + 1 + K
+    o_p = up(n * 64 * 2)
+    o_sd = o_p + up(n * S * 4)
+    qt = res[:n * 128].view(torch.float16).view(B, H, T, 64)
+    P = res[o_p:o_p + n * S * 4].view(torch.float32).view(B, H, S, T)
+    sd = res[o_sd:o_sd + n * K * 4].view(torch.float32).view(B, H, K, T)
+    return qt, P, sd
+
+
+def _check_residuals(res, q, W, K):
+    if res is None:
+        return
+    B, H, T, D = q.shape
+    if not (res.is_cuda and res.is_contiguous() and res.numel() * res.element_size() >=
+            residual_bytes(B, H, T, W, K, q.dtype, D)):
+        raise ValueError("residuals must be a contiguous CUDA buffer of residual_bytes(...) bytes")
 
 
 def rotated_k_like(k: torch.Tensor) -> torch.Tensor:
@@ -161,6 +206,27 @@ def coverage(alphas, offsets, W: int, T: int, dedup: bool = True) -> dict:
     return dict(per_layer=per, union=u.value, beyond_window=bw.value, two_hop=hop.value)
 
 
+def staging_layout(kind: str, T: int, W: int, alpha: float, offsets, dedup: bool = True) -> dict:
+    """Shared-memory staging layout of the tensor-core kernels (see
+    fibattn_staging_layout): kind "query" (forward, backward query pass) or
+    "key" (backward key pass).  Returns the merged intervals (start, len,
+    smem arrays) and slab_row per rung (-1 when not staged)."""
+    f = _offsets(offsets)
+    K = len(f)
+    L = lib()
+    ip = ctypes.POINTER(ctypes.c_int)
+    L.fibattn_staging_layout.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_float,
+                                         ctypes.POINTER(ctypes.c_float), ctypes.c_int, ctypes.c_int, ip, ip, ip, ip, ip]
+    L.fibattn_staging_layout.restype = ctypes.c_int
+    n = ctypes.c_int()
+    st, ln, sm = (np.zeros(64, np.int32) for _ in range(3))
+    slab = np.zeros(max(K, 1), np.int32)
+    _check(L.fibattn_staging_layout({"query": 0, "key": 1}[kind], int(T), int(W), float(alpha), _fptr(f), K,
+                                    0 if dedup else 1, ctypes.byref(n), _iptr(st), _iptr(ln), _iptr(sm), _iptr(slab)))
+    m = n.value
+    return dict(start=st[:m].copy(), len=ln[:m].copy(), smem=sm[:m].copy(), slab_row=slab[:K].copy())
+
+
 def rung_params(alpha: float, offsets, W: int, dedup: bool = True):
     f = _offsets(offsets)
     K = len(f)
@@ -186,16 +252,20 @@ def bwd_workspace_bytes(B, H, T, W, K, dtype, Hkv=None, D=64) -> int:
 
 
 def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
-        out=None, lse=None, workspace=None, stream=None, kernel="auto", rotated_k=None):
+        out=None, lse=None, workspace=None, stream=None, kernel="auto", rotated_k=None, residuals=None):
     """Forward pass.  q [B,H,T,64]; k, v [B,Hkv,T,64] (fp32 or bf16, CUDA,
     contiguous).  ``kernel``: "auto", "gather", "staged" or "mma".
     ``rotated_k``: optional buffer (``rotated_k_like(k)``) that receives the
-    rotated keys for a later ``bwd(..., rotated_k=...)``.  Returns (out, lse)."""
+    rotated keys for a later ``bwd(..., rotated_k=...)``.  ``residuals``:
+    optional buffer (``residuals_like(q, W, K)``) that receives the rotated
+    queries, p of every slot and the rung score differences for a later
+    ``bwd(..., residuals=...)`` (tensor-core forward only).  Returns (out, lse)."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
     _check_rotated(rotated_k, k)
-    o = _opts(rope_base, scale, Hkv, dedup, kernel, rotated_k=rotated_k)
+    _check_residuals(residuals, q, W, len(f))
+    o = _opts(rope_base, scale, Hkv, dedup, kernel, rotated_k=rotated_k, residuals=residuals)
     code = _dtype_code(q)
     for t in (q, k, v):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
@@ -215,19 +285,22 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
 
 def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_base=1e4, scale=None, dedup=True,
         dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None, kernel="auto",
-        rotated_k=None, rung_grads=True):
+        rotated_k=None, rung_grads=True, residuals=None):
     """Backward pass.  ``out``: the forward output (optional; enables the
     tensor-core query pass).  ``kernel``: "auto", "gather" or "mma".
     ``rotated_k``: the buffer the forward of the same k filled (skips rotating
-    k again).  ``rung_grads=False`` skips dL/dtheta and dL/dd_k (a fixed
-    schedule).  Returns (dq, dk, dv, dtheta [1], dd [K]) on the device
-    (dtheta, dd None without rung_grads)."""
+    k again).  ``residuals``: the buffer the forward of the same inputs filled
+    (the tensor-core passes then read p, the rung score differences and the
+    rotated queries instead of recomputing them).  ``rung_grads=False`` skips
+    dL/dtheta and dL/dd_k (a fixed schedule).  Returns (dq, dk, dv, dtheta [1],
+    dd [K]) on the device (dtheta, dd None without rung_grads)."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
     K = len(f)
     _check_rotated(rotated_k, k)
-    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel, rotated_k=rotated_k)
+    _check_residuals(residuals, q, W, K)
+    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel, rotated_k=rotated_k, residuals=residuals)
     code = _dtype_code(q)
     for t in (q, k, v, dout) + ((out,) if out is not None else ()):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):

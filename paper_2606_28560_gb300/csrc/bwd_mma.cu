@@ -41,9 +41,19 @@ constexpr int kRowsPerWarp = 15;
 __device__ __forceinline__ float bf_lo(unsigned u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 0xffff0000u); }
 
+// 4-byte asynchronous copy global -> shared; zero-filled when !full.
+__device__ __forceinline__ void cp_async4(const float* dst, const float* src, bool full) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n"
+                 :: "r"(smem_u32(dst)), "l"(src), "r"(full ? 4 : 0) : "memory");
+}
+
 // DD: also the rung-distance gradient dL/dd_k (off when the caller asks for
 // neither dtheta nor dd, e.g. a fixed alpha schedule).
-template <int NT, bool DD>
+// SV: p of every slot and the far-minus-floor rung scores come from the
+// forward's residuals (p and the rotated queries serve the key pass too), so
+// the scores are not recomputed: dS = p (dp - Delta) is formed in the value
+// phase and the key phase only accumulates dq~.
+template <int NT, bool DD, bool SV>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                      const __grid_constant__ QTileMaps tm, BwdArgs a, MmaLayout L) {
@@ -51,7 +61,12 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     constexpr int Wp = NT * 8 - 16;
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[4];        // V (first batch), K~, V (second batch), tile rows
-    __shared__ float dps[kWarps][kMmaMaxRungs][16][2];   // rung dp, ddp of each tile row
+    // !SV: rung dp, ddp of each warp's tile rows.  SV: p (replaced by dS once
+    // known) and sd of each active rung (list order) and tile row.
+    constexpr int kXs = SV ? 2 * kMmaMaxRungs * kMmaTile : kWarps * kMmaMaxRungs * 16 * 2;
+    __shared__ __align__(16) float xs[kXs];
+    auto dps = reinterpret_cast<float (*)[kMmaMaxRungs][16][2]>(xs);
+    auto psd = reinterpret_cast<float (*)[kMmaMaxRungs][kMmaTile]>(xs);
     __shared__ float gsm[kWarps][kMmaMaxRungs];           // per-warp rung-gradient sums
     __shared__ unsigned long long kbar[kMmaMaxRungs + 1]; // key rows of each merged interval
     __shared__ unsigned rel_cnt[kMmaMaxRungs + 1];        // warps done with an interval's value rows
@@ -82,10 +97,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     if (warp == 0) {
         __syncwarp();
         if (lane == 0) {
-            mbar_expect_tx(&bars[3], 3u * 128u * 128u);
+            mbar_expect_tx(&bars[3], (SV ? 2u : 3u) * 128u * 128u);
             const CUtensorMap* maps[3] = {&tm.q, &tm.g, &tm.o};
 #pragma unroll
-            for (int t = 0; t < 3; ++t)
+            for (int t = SV ? 1 : 0; t < 3; ++t)
 #pragma unroll
                 for (int hb = 0; hb < 2; ++hb)
                     tma_load_3d(buf + (size_t)(128 * t + 64 * hb) * 128, maps[t], 0, i0 + 64 * hb, bh, &bars[3]);
@@ -97,6 +112,33 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
     const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
     const size_t rowbase = (size_t)bh * s.T;
+    float* Pg = a.Ps + (size_t)bh * a.S * s.T;       // [slot][T] of this head
+    float* DSg = a.DSs + (size_t)bh * a.S * s.T;
+
+    // SV: the residual p of the window band at this thread's accumulator
+    // entries (registers), and p and sd of the active rungs for the tile's
+    // rows (shared memory, 4-byte asynchronous copies by every thread)
+    float pb[NT][4];
+    if constexpr (SV) {
+#pragma unroll
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool hi = e >= 2;
+                const int r = hi ? g4 + 8 : g4;
+                const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
+                pb[j][e] = ((hi ? vhi : vlo) && t >= 0 && t <= s.W) ? Pg[(size_t)t * s.T + bw + r] : 0.f;
+            }
+        const float* SDg = DD ? a.res_sd + (size_t)bh * a.r.K * s.T : nullptr;
+        for (int u = tid; u < L.n_act * kMmaTile; u += kWarps * 32) {
+            const int i = u / kMmaTile, r = u - i * kMmaTile;
+            const bool in = i0 + r < s.T;
+            const int q = in ? i0 + r : 0, k = L.act_k[i];
+            cp_async4(&psd[0][i][r], Pg + (size_t)(s.W + 1 + k) * s.T + q, in);
+            if (DD) cp_async4(&psd[1][i][r], SDg + (size_t)k * s.T + q, in);
+        }
+        asm volatile("cp.async.commit_group;\n" ::: "memory");
+    }
 
     __syncthreads();                              // barrier init visible
     bool ok_v = mbar_wait(&bars[3], 0);
@@ -132,7 +174,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 
     // ---- q~ as fp16 A fragments (RoPE pairs m, m+32 in the same thread)
     unsigned qa[4][4];
-    {
+    if constexpr (!SV) {
         unsigned qr[4][4];
         tile_frags(0, qr);
         float cs[2][4], sn[2][4];
@@ -182,23 +224,30 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     }
     // ---- q~ rows to the workspace (for the key pass): written in place of the
     // staged q rows, then stored by TMA (rows past T are clipped); the value
-    // rows of the second batch follow once the store has read them
-    __syncthreads();                              // every warp has read the tile rows
-#pragma unroll
-    for (int half = 0; half < 2; ++half) {
-        if (g4 + 8 * half >= kRowsPerWarp) continue;
-        const int row = wrel + g4 + 8 * half;
-#pragma unroll
-        for (int kc = 0; kc < 4; ++kc) {
-            asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc) + 4 * c4), "r"(qa[kc][half]));
-            asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc + 1) + 4 * c4),
-                         "r"(qa[kc][2 + half]));
-        }
+    // rows of the second batch follow once the store has read them.  (SV: the
+    // forward wrote them; the second batch follows once the tile rows are read.)
+    if constexpr (SV) {
+        asm volatile("cp.async.wait_group 0;\n" ::: "memory");
+        asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
     }
-    asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-    __syncthreads();
+    __syncthreads();                              // every warp has read the tile rows (SV: residuals landed)
+    if constexpr (!SV) {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            if (g4 + 8 * half >= kRowsPerWarp) continue;
+            const int row = wrel + g4 + 8 * half;
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc) + 4 * c4), "r"(qa[kc][half]));
+                asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc + 1) + 4 * c4),
+                             "r"(qa[kc][2 + half]));
+            }
+        }
+        asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+        __syncthreads();
+    }
     if (warp == 0) {
-        if (lane == 0) {
+        if (!SV && lane == 0) {
 #pragma unroll
             for (int t = 0; t < 3; ++t)                // 3 boxes of 40 rows: the tile's 120 queries
                 asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];\n"
@@ -210,12 +259,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         __syncwarp();
         issue_rows_batch(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[2], lane, true);
     }
-    const float lse2_lo = vlo ? a.lse[rowbase + qlo] * kLog2e : 0.f;
-    const float lse2_hi = vhi ? a.lse[rowbase + qhi] * kLog2e : 0.f;
-    if (c4 == 0) {
-        if (vlo) a.Delta[rowbase + qlo] = dlt_lo;
-        if (vhi) a.Delta[rowbase + qhi] = dlt_hi;
-    }
+    const float lse2_lo = (!SV && vlo) ? a.lse[rowbase + qlo] * kLog2e : 0.f;
+    const float lse2_hi = (!SV && vhi) ? a.lse[rowbase + qhi] * kLog2e : 0.f;
 
     // Columns of a rung slab: row r's far row is x = r (weight w), its floor
     // row x = r+1 (weight 1-w).  Of this thread's accumulator and A-fragment
@@ -256,6 +301,25 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
             mma_bf16_16816(dpw[j], da[kc], b0, b1);
             mma_bf16_16816(dpw[j], da[kc + 1], b2, b3);
+        }
+    }
+    // window band dS = p (dp - Delta) as fp16 A fragments (SV: here; else in
+    // the key phase, once the scores are known); dS per slot to the workspace
+    unsigned dsa[NT][2];
+    if constexpr (SV) {
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+            float dsv[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool hi = e >= 2;
+                const int r = hi ? g4 + 8 : g4;
+                const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
+                dsv[e] = pb[j][e] * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
+                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) DSg[(size_t)t * s.T + bw + r] = dsv[e];
+            }
+            dsa[j][0] = pack_f16(dsv[0], dsv[1]);
+            dsa[j][1] = pack_f16(dsv[2], dsv[3]);
         }
     }
     // Rungs in increasing d; those masked for every row of the warp's tile
@@ -307,7 +371,30 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             ddp_lo = quad_sum(fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0])));
             ddp_hi = quad_sum(fmaf(df0, dt[1][2], df1 * dt[1][3]));
         }
-        if (c4 == 0) {
+        if constexpr (SV) {
+            // dS from the residual p; dL/dd_k of this warp's rows (fixed order over
+            // the rows); dS replaces p in shared memory for the key phase
+            const int rlo = wrel + g4, rhi = wrel + g4 + 8;
+            const float p_lo = vlo ? psd[0][i][rlo] : 0.f, p_hi = vhi ? psd[0][i][rhi] : 0.f;
+            const float e_lo = dp_lo - dlt_lo, e_hi = dp_hi - dlt_hi;
+            const float ds_lo = p_lo * e_lo, ds_hi = p_hi * e_hi;
+            if constexpr (DD) {
+                const float sd_lo = vlo ? psd[1][i][rlo] : 0.f, sd_hi = vhi ? psd[1][i][rhi] : 0.f;
+                float g = 0.f;
+                if (c4 == 0)
+                    g = p_lo * fmaf(s.scale * sd_lo, e_lo, ddp_lo) + p_hi * fmaf(s.scale * sd_hi, e_hi, ddp_hi);
+                g += __shfl_xor_sync(0xffffffffu, g, 4);
+                g += __shfl_xor_sync(0xffffffffu, g, 8);
+                g += __shfl_xor_sync(0xffffffffu, g, 16);
+                if (lane == 0) gsm[warp][L.act_k[i]] = g;
+            }
+            __syncwarp();                         // the quad has read p before it is replaced
+            if (c4 == 0) {
+                const size_t slot = (size_t)(s.W + 1 + L.act_k[i]) * s.T;
+                if (vlo) { psd[0][i][rlo] = ds_lo; DSg[slot + qlo] = ds_lo; }
+                if (vhi) { psd[0][i][rhi] = ds_hi; DSg[slot + qhi] = ds_hi; }
+            }
+        } else if (c4 == 0) {
             *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
             *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
         }
@@ -325,16 +412,16 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     };
 
     const float sc2 = s.scale * kLog2e;
-    float* Pg = a.Ps + (size_t)bh * a.S * s.T;       // [slot][T] of this head
-    float* DSg = a.DSs + (size_t)bh * a.S * s.T;
 
     float dq[8][4];
 #pragma unroll
     for (int n = 0; n < 8; ++n) dq[n][0] = dq[n][1] = dq[n][2] = dq[n][3] = 0.f;
 
-    // ---- window band: scores, p, dS; P and dp per slot to the workspace
+    // ---- window band: scores, p, dS; P and dS per slot to the workspace (SV:
+    // dS is known); dq~ += dS_band K~_band
     need_keys(L.win_iv);
-    {
+    if constexpr (SV) __syncwarp();               // dS of the value phase, written by the quad's lane 0
+    if constexpr (!SV) {
         float sw[NT][4];
 #pragma unroll
         for (int j = 0; j < NT; ++j) {
@@ -348,7 +435,6 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 mma_f16_16816(sw[j], qa[kc + 1], b2, b3);
             }
         }
-        unsigned dsa[NT][2];
 #pragma unroll
         for (int j = 0; j < NT; ++j) {
             float dsv[4];
@@ -372,7 +458,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             dsa[j][0] = pack_f16(dsv[0], dsv[1]);
             dsa[j][1] = pack_f16(dsv[2], dsv[3]);
         }
-        // dq~ += dS_band K~_band
+    }
+    {
 #pragma unroll
         for (int kk = 0; kk + 1 < NT; kk += 2) {
             const unsigned afr[4] = {dsa[kk][0], dsa[kk][1], dsa[kk + 1][0], dsa[kk + 1][1]};
@@ -403,60 +490,68 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     // ---- rungs that no row of the tile attends: zero slots for the key pass
     for (int i = n_use; i < L.n_act; ++i) {
         const int slot = s.W + 1 + L.act_k[i];
-        if (c4 == 0) {
-            if (vlo) { Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
-            if (vhi) { Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
+        if (c4 == 0) {                            // (SV: the forward wrote p = 0 there)
+            if (vlo) { if (!SV) Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
+            if (vhi) { if (!SV) Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
         }
         if (lane == 0) gsm[warp][L.act_k[i]] = 0.f;
     }
-    // ---- rungs: scores, p, dS, dL/dd_k; dq~ += dShat_k K~_slab
+    // ---- rungs: scores, p, dS, dL/dd_k (SV: dS from the value phase);
+    // dq~ += dShat_k K~_slab
 #pragma unroll 1
     for (int i = 0; i < n_use; ++i) {
         need_keys(L.act_iv[i]);
-        const int k = L.act_k[i];
-        const int slot = s.W + 1 + k;
         const float w = L.act_w[i], w1 = 1.f - w;
-        float st[2][4];
-#pragma unroll
-        for (int t = 0; t < 2; ++t) {
-            st[t][0] = st[t][1] = st[t][2] = st[t][3] = 0.f;
-            const int krow = L.act_smem[i] + wrel + 8 * t + (lane & 7);
-#pragma unroll
-            for (int kc = 0; kc < 4; kc += 2) {
-                unsigned b0, b1, b2, b3;
-                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
-                mma_f16_16816(st[t], qa[kc], b0, b1);
-                mma_f16_16816(st[t], qa[kc + 1], b2, b3);
-            }
-        }
-        // interpolated score and far-minus-floor raw score of rows g4, g4+8
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-        const float si_lo = quad_sum(fmaf(c0, st[0][0], fmaf(c1, st[0][1], c7 * st[1][0])));
-        const float si_hi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3]));
-        const float dk = L.act_d[i];
-        const bool okl = vlo && dk <= (float)qlo, okh = vhi && dk <= (float)qhi;
-        const float2 dpl = *reinterpret_cast<const float2*>(dps[warp][i][g4]);
-        const float2 dph = *reinterpret_cast<const float2*>(dps[warp][i][g4 + 8]);
-        const float dp_lo = dpl.x, ddp_lo = dpl.y, dp_hi = dph.x, ddp_hi = dph.y;
-        const float p_lo = okl ? exp2f(si_lo * sc2 - lse2_lo) : 0.f;
-        const float p_hi = okh ? exp2f(si_hi * sc2 - lse2_hi) : 0.f;
-        const float e_lo = dp_lo - dlt_lo, e_hi = dp_hi - dlt_hi;
-        const float ds_lo = p_lo * e_lo, ds_hi = p_hi * e_hi;
-        if (c4 == 0) {
-            if (vlo) { Pg[(size_t)slot * s.T + qlo] = p_lo; DSg[(size_t)slot * s.T + qlo] = ds_lo; }
-            if (vhi) { Pg[(size_t)slot * s.T + qhi] = p_hi; DSg[(size_t)slot * s.T + qhi] = ds_hi; }
-        }
-        if constexpr (DD) {
-            // far-minus-floor raw scores; dL/dd_k of this warp's rows, in a fixed order over the rows
-            const float sd_lo = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
-            const float sd_hi = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
-            float g = 0.f;
-            if (c4 == 0)
-                g = p_lo * fmaf(s.scale * sd_lo, e_lo, ddp_lo) + p_hi * fmaf(s.scale * sd_hi, e_hi, ddp_hi);
-            g += __shfl_xor_sync(0xffffffffu, g, 4);
-            g += __shfl_xor_sync(0xffffffffu, g, 8);
-            g += __shfl_xor_sync(0xffffffffu, g, 16);
-            if (lane == 0) gsm[warp][k] = g;
+        float ds_lo, ds_hi;
+        if constexpr (SV) {
+            ds_lo = vlo ? psd[0][i][wrel + g4] : 0.f;
+            ds_hi = vhi ? psd[0][i][wrel + g4 + 8] : 0.f;
+        } else {
+            const int k = L.act_k[i];
+            const int slot = s.W + 1 + k;
+            float st[2][4];
+#pragma unroll
+            for (int t = 0; t < 2; ++t) {
+                st[t][0] = st[t][1] = st[t][2] = st[t][3] = 0.f;
+                const int krow = L.act_smem[i] + wrel + 8 * t + (lane & 7);
+#pragma unroll
+                for (int kc = 0; kc < 4; kc += 2) {
+                    unsigned b0, b1, b2, b3;
+                    ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                    mma_f16_16816(st[t], qa[kc], b0, b1);
+                    mma_f16_16816(st[t], qa[kc + 1], b2, b3);
+                }
+            }
+            // interpolated score and far-minus-floor raw score of rows g4, g4+8
+            const float si_lo = quad_sum(fmaf(c0, st[0][0], fmaf(c1, st[0][1], c7 * st[1][0])));
+            const float si_hi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3]));
+            const float dk = L.act_d[i];
+            const bool okl = vlo && dk <= (float)qlo, okh = vhi && dk <= (float)qhi;
+            const float2 dpl = *reinterpret_cast<const float2*>(dps[warp][i][g4]);
+            const float2 dph = *reinterpret_cast<const float2*>(dps[warp][i][g4 + 8]);
+            const float dp_lo = dpl.x, ddp_lo = dpl.y, dp_hi = dph.x, ddp_hi = dph.y;
+            const float p_lo = okl ? exp2f(si_lo * sc2 - lse2_lo) : 0.f;
+            const float p_hi = okh ? exp2f(si_hi * sc2 - lse2_hi) : 0.f;
+            const float e_lo = dp_lo - dlt_lo, e_hi = dp_hi - dlt_hi;
+            ds_lo = p_lo * e_lo;
+            ds_hi = p_hi * e_hi;
+            if (c4 == 0) {
+                if (vlo) { Pg[(size_t)slot * s.T + qlo] = p_lo; DSg[(size_t)slot * s.T + qlo] = ds_lo; }
+                if (vhi) { Pg[(size_t)slot * s.T + qhi] = p_hi; DSg[(size_t)slot * s.T + qhi] = ds_hi; }
+            }
+            if constexpr (DD) {
+                // far-minus-floor raw scores; dL/dd_k of this warp's rows, in a fixed order over the rows
+                const float sd_lo = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
+                const float sd_hi = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
+                float g = 0.f;
+                if (c4 == 0)
+                    g = p_lo * fmaf(s.scale * sd_lo, e_lo, ddp_lo) + p_hi * fmaf(s.scale * sd_hi, e_hi, ddp_hi);
+                g += __shfl_xor_sync(0xffffffffu, g, 4);
+                g += __shfl_xor_sync(0xffffffffu, g, 8);
+                g += __shfl_xor_sync(0xffffffffu, g, 16);
+                if (lane == 0) gsm[warp][k] = g;
+            }
         }
 
         // dShat_k as fp16 A fragment: the interpolation weights times dS of the row
@@ -522,12 +617,18 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             for (int wv = 0; wv < kWarps; ++wv) x += gsm[wv][tid];
         write_rung_partials(a, x);
     }
+    // ---- no copy may outlive the CTA: the key rows of intervals that no rung
+    // of this warp read were issued (by the last warp to release them) but not
+    // waited for, and the rotated-query store may still be writing
+    for (int j = 0; j < L.n_iv; ++j) need_keys(j);
+    if (!SV && tid == 0) asm volatile("cp.async.bulk.wait_group 0;\n" ::: "memory");
 }
 
 template <int NT>
 cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const QTileMaps& mt, const BwdArgs& a,
                       const MmaLayout& L, unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = a.want_dd ? bwd_query_mma_kernel<NT, true> : bwd_query_mma_kernel<NT, false>;
+    auto kern = a.saved ? (a.want_dd ? bwd_query_mma_kernel<NT, true, true> : bwd_query_mma_kernel<NT, false, true>)
+                        : (a.want_dd ? bwd_query_mma_kernel<NT, true, false> : bwd_query_mma_kernel<NT, false, false>);
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mk, mv, mt, a, L);

@@ -45,7 +45,6 @@ int fail(int code, const char* fmt, ...) {
 
 size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
 
-size_t elem_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
 // rotated q/k rows in the workspace: fp32 (fp32 I/O) or fp16 (bf16 I/O)
 size_t rot_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
 
@@ -53,6 +52,7 @@ struct Resolved {
     float rope_base, scale;
     int Hkv, dedup, fwd_kernel, bwd_kernel;
     void* rotated_k;
+    void* residuals;
 };
 
 int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
@@ -65,6 +65,8 @@ int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
     r->bwd_kernel = o ? o->bwd_kernel : 0;
     r->rotated_k = o ? o->rotated_k : nullptr;
     if ((uintptr_t)r->rotated_k & 15u) return fail(FIBATTN_ERR_INVALID_ARG, "rotated_k must be 16-byte aligned");
+    r->residuals = o ? o->residuals : nullptr;
+    if ((uintptr_t)r->residuals & 15u) return fail(FIBATTN_ERR_INVALID_ARG, "residuals must be 16-byte aligned");
     if (r->bwd_kernel < 0 || r->bwd_kernel > 2) return fail(FIBATTN_ERR_INVALID_ARG, "bwd_kernel must be 0, 1 or 2");
     if (!(r->rope_base > 1.f) || !std::isfinite(r->rope_base))
         return fail(FIBATTN_ERR_INVALID_ARG, "rope_base must be finite and > 1 (got %g)", (double)r->rope_base);
@@ -129,6 +131,22 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
     return s;
 }
 
+// Forward residuals (fibattn_opts.residuals): rotated q (fp16), p per slot
+// (slot-major), far-minus-floor rung scores (rung-major).
+struct ResLayout {
+    size_t qt, P, sd, total;
+};
+
+ResLayout res_layout(int B, int H, int T, int W, int K) {
+    ResLayout L;
+    const size_t n = (size_t)B * H * T;
+    L.qt = 0;
+    L.P = align256(n * kHeadDim * 2);
+    L.sd = L.P + align256(n * ((size_t)W + 1 + K) * 4);
+    L.total = L.sd + align256(n * (size_t)K * 4);
+    return L;
+}
+
 struct BwdLayout {
     size_t qt, kt, P, DP, Delta, rpart, total;
 };
@@ -155,6 +173,17 @@ BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype, bool
 
 int cuda_fail(cudaError_t e, const char* what) {
     return fail(FIBATTN_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Tensor maps are encoded through the driver, which needs a current context,
+// and a host thread that has made no runtime call yet (e.g. a framework's
+// backward worker) has none: make the primary context of the thread's current
+// device current before the first encode or launch.
+int bind_context() {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaSetDevice(dev);
+    return e == cudaSuccess ? FIBATTN_OK : cuda_fail(e, "binding the current device's context");
 }
 
 // ---------------------------------------------------------------- profiler --
@@ -249,6 +278,11 @@ int fibattn_profile_summary(int index, char* name, int name_len, double* total_m
 
 const char* fibattn_last_error(void) { return g_err.c_str(); }
 
+size_t fibattn_residual_bytes(int B, int H, int T, int D, int W, int K, int dtype) {
+    if (check_shape(B, H, T, D, W, K, dtype) || dtype != FIBATTN_BF16) return 0;
+    return res_layout(B, H, T, W, K).total;
+}
+
 int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup,
                         float* d, int* s0, float* w, int* active) {
     if (K < 0 || K > kMaxRungs) return fail(FIBATTN_ERR_INVALID_ARG, "K must be in [0, %d]", kMaxRungs);
@@ -333,12 +367,6 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     a.q = q; a.k = k; a.v = v; a.out = out; a.lse = lse; a.kt = kt;
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool bf16 = dtype == FIBATTN_BF16;
-    cudaError_t e;
-    {
-        ProfScope p("rope_k", st);
-        e = launch_rope_rows(k, kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
-    }
-    if (e != cudaSuccess) return cuda_fail(e, "rope prologue launch");
     // bf16 I/O: the tensor-core kernel when its layout applies (W <= 16,
     // K <= 16, shared memory fits), else the staged CUDA-core kernel, else the
     // row-gather kernel (also the fp32 I/O path).
@@ -351,6 +379,24 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     if ((o.fwd_kernel == 3 && !mma_ok) || (o.fwd_kernel == 2 && !staged_ok))
         return fail(FIBATTN_ERR_UNSUPPORTED, "requested forward kernel does not apply to these arguments "
                                              "(bf16 I/O, W <= 16, K <= 16, shared-memory layout)");
+    if (o.residuals) {
+        if (!mma_ok)
+            return fail(FIBATTN_ERR_UNSUPPORTED, "forward residuals need the tensor-core forward (bf16 I/O, "
+                                                 "fwd_kernel 0 or 3, W <= 16, K <= 16, shared-memory layout)");
+        const ResLayout R = res_layout(B, H, T, W, K);
+        char* rb = reinterpret_cast<char*>(o.residuals);
+        a.res_qt = rb + R.qt;
+        a.res_P = reinterpret_cast<float*>(rb + R.P);
+        a.res_sd = reinterpret_cast<float*>(rb + R.sd);
+    }
+    a.S = W + 1 + K;
+    if ((rc = bind_context())) return rc;
+    cudaError_t e;
+    {
+        ProfScope p("rope_k", st);
+        e = launch_rope_rows(k, kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "rope prologue launch");
     if (mma_ok) {
         ProfScope p("fwd", st);
         e = launch_fwd_mma(a, ML, st);
@@ -417,7 +463,16 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         return fail(FIBATTN_ERR_UNSUPPORTED, "tensor-core backward needs bf16, out, W <= 16, K <= 16 and a staged row "
                                              "union that fits shared memory");
     if (mma_ok) a.nblk_q = bwd_mma_blocks(a.s);
+    if (mma_ok && o.residuals) {                 // p, sd and q~ from the forward
+        const ResLayout R = res_layout(B, H, T, W, K);
+        char* rb = reinterpret_cast<char*>(o.residuals);
+        a.saved = 1;
+        a.qt = rb + R.qt;
+        a.Ps = reinterpret_cast<float*>(rb + R.P);
+        a.res_sd = reinterpret_cast<const float*>(rb + R.sd);
+    }
     cudaError_t e;
+    if ((rc = bind_context())) return rc;
     if (B > 0) {
         if (!mma_ok) {
             ProfScope p("rope_q", st);
@@ -453,6 +508,33 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         return FIBATTN_OK;
     }
     return FIBATTN_OK;                           // dtheta and dd: written by block 0 of the key pass
+}
+
+int fibattn_staging_layout(int kind, int T, int W, float alpha, const float* offsets, int K, int no_dedup,
+                           int* n_iv, int* iv_start, int* iv_len, int* iv_smem, int* slab_row) {
+    if (kind != 0 && kind != 1) return fail(FIBATTN_ERR_INVALID_ARG, "kind must be 0 or 1");
+    if (T < 1 || T > (1 << 20)) return fail(FIBATTN_ERR_INVALID_ARG, "T must be in [1, 2^20]");
+    if (W < 0 || W > kMaxWindow || K < 0 || K > kMaxRungs)
+        return fail(FIBATTN_ERR_INVALID_ARG, "need 0 <= W <= %d and 0 <= K <= %d", kMaxWindow, kMaxRungs);
+    RungParams r;
+    int rc = prep_rungs(alpha, offsets, K, W, no_dedup ? 0 : 1, T, &r);
+    if (rc) return rc;
+    Shape s;
+    std::memset(&s, 0, sizeof(s));
+    s.B = 1; s.H = 1; s.Hkv = 1; s.G = 1; s.T = T; s.W = W;
+    MmaLayout L;
+    std::memset(&L, 0, sizeof(L));
+    const size_t no_limit = ~(size_t)0;
+    const bool ok = kind == 0 ? build_mma_layout(s, r, 1e4, no_limit, &L) : build_key_layout(s, r, 1e4, no_limit, &L);
+    if (!ok) return fail(FIBATTN_ERR_UNSUPPORTED, "the tensor-core layout needs W <= 16 and K <= %d", kMmaMaxRungs);
+    if (n_iv) *n_iv = L.n_iv;
+    for (int i = 0; i < L.n_iv; ++i) {
+        if (iv_start) iv_start[i] = L.iv_start[i];
+        if (iv_len) iv_len[i] = L.iv_len[i];
+        if (iv_smem) iv_smem[i] = L.iv_smem[i];
+    }
+    for (int k = 0; k < K && slab_row; ++k) slab_row[k] = ((r.active >> k) & 1u) ? L.rung_smem[k] : -1;
+    return FIBATTN_OK;
 }
 
 int fibattn_coverage(int L, const float* alphas, const float* offsets, int K, int W, int T, int no_dedup,

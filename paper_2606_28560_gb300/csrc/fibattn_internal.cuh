@@ -46,6 +46,14 @@ struct FwdArgs {
     const void* v;            // [B,Hkv,T,D]
     void* out;                // [B,H,T,D]
     float* lse;               // [B,H,T]
+    // Optional residuals for the backward (tensor-core forward only; all
+    // nullptr when not asked for): the rotated queries, the probability of
+    // every slot (0 where not attended) and the far-minus-floor raw score of
+    // every rung row.
+    void* res_qt;             // fp16 [B,H,T,D]
+    float* res_P;             // slot-major [B,H,S,T], S = W + 1 + K
+    float* res_sd;            // rung-major [B,H,K,T]
+    int S;
     Shape s;
     RungParams r;
     RopeParams rope;
@@ -73,6 +81,9 @@ struct BwdArgs {
     float* Ps;                // tensor-core path, slot-major [B,H,S,T]: p      (P region)
     float* DSs;               //                                      dS = p (dp - Delta)  (DP region)
     long long* rpart;         // per query-pass block dL/dd_k partials, 2^-32 fixed point [kMaxRungs][nblk_q]
+    const float* res_sd;      // forward residual far-minus-floor rung scores [B,H,K,T], or nullptr;
+                              // when the forward residuals are used, Ps and qt point into them
+    int saved;                // tensor-core passes read p (Ps), sd and q~ (qt) from the forward residuals
     int nblk_q;               // query-pass blocks
     int S;                    // slots per query = W + 1 + K
     float alpha;

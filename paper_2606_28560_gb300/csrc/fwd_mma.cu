@@ -50,7 +50,10 @@ constexpr int kRowsPerWarp = 15;                 // useful query rows of a 16-ro
 // CTA of 16 warps owns a kv head's tile; keys and values are staged once, into
 // two buffers, and each team of 8 warps loops over its share of the group's
 // query heads (team t takes heads t, t + 2, ...).
-template <int NT, int TEAMS>
+// SAVE: also write the residuals the tensor-core backward reads instead of
+// recomputing the scores -- the rotated queries, p of every slot (normalised,
+// fp32; 0 where not attended) and the far-minus-floor raw score of every rung.
+template <int NT, int TEAMS, bool SAVE>
 __global__ void __launch_bounds__(kWarps * 32 * TEAMS, TEAMS == 1 ? 2 : 1)
 fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                FwdArgs a, MmaLayout L) {
@@ -151,6 +154,19 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const int qlo = bw + g4, qhi = bw + g4 + 8;   // absolute queries of this thread's rows
     const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
     const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
+    const size_t rowbase = (size_t)bh * s.T;
+    if constexpr (SAVE) {                         // rotated query rows 0..14 of the warp's tile
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            if (!(half ? vhi : vlo)) continue;
+            __half* row = reinterpret_cast<__half*>(a.res_qt) + (rowbase + (half ? qhi : qlo)) * kHeadDim;
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                *reinterpret_cast<unsigned*>(row + 16 * kc + 2 * c4) = qa[kc][half];
+                *reinterpret_cast<unsigned*>(row + 16 * kc + 8 + 2 * c4) = qa[kc][2 + half];
+            }
+        }
+    }
 
     const bool ok_k = mbar_wait(&bars[0], 0);
 
@@ -198,6 +214,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const float ia0 = dl == 1 ? 1.f : 0.f, ib0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f);
     const float ia1 = dl == 0 ? 1.f : 0.f, ib1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
     const float m7 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
+    // far-minus-floor pattern (residual sd): +1 at the far entry, -1 at the floor entry
+    const float df0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f), df1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
     float rs[kMmaMaxRungs][2];
 #pragma unroll
     for (int k = 0; k < kMmaMaxRungs; ++k) { rs[k][0] = -INFINITY; rs[k][1] = -INFINITY; }
@@ -227,6 +245,15 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         rs[k][1] = (vhi && dk <= (float)qhi) ? phi : -INFINITY;
         mlo = fmaxf(mlo, rs[k][0]);
         mhi = fmaxf(mhi, rs[k][1]);
+        if constexpr (SAVE) {
+            const float sdl = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
+            const float sdh = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
+            if (c4 == 0) {
+                float* sd = a.res_sd + ((size_t)bh * a.r.K + k) * s.T;
+                if (vlo) sd[qlo] = sdl;
+                if (vhi) sd[qhi] = sdh;
+            }
+        }
     }
 
     if (TEAMS == 1) {
@@ -252,6 +279,47 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     }
     llo = quad_sum(llo);
     lhi = quad_sum(lhi);
+
+    if constexpr (SAVE) {
+        // ---- residuals need the row sums before the value product: rung p in
+        // place of the scores (0 when masked) and its bf16 entries summed here,
+        // in the order the value loop would take them
+#pragma unroll
+        for (int k = 0; k < kMmaMaxRungs; ++k) {
+            if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
+            if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
+            const float w = a.r.w[k], w1 = 1.f - w;
+            rs[k][0] = exp2f(rs[k][0] - mlo);
+            rs[k][1] = exp2f(rs[k][1] - mhi);
+            const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+            llo += quad_sum(bf16_round(c0 * rs[k][0]) + bf16_round(c1 * rs[k][0]) + bf16_round(c7 * rs[k][0]));
+            lhi += quad_sum(bf16_round(c0 * rs[k][1]) + bf16_round(c1 * rs[k][1]));
+        }
+        // ---- residual p = exp2(s - m) / l of every slot of rows 0..14 (0 where
+        // not attended, also for rungs no row of the warp attends)
+        const float ilo = 1.f / llo, ihi = 1.f / lhi;
+        float* Pg = a.res_P + (size_t)bh * a.S * s.T;
+#pragma unroll
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const bool hi = e >= 2;
+                const int r = hi ? g4 + 8 : g4;
+                const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
+                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W)
+                    Pg[(size_t)t * s.T + bw + r] = exp2f(sw[j][e] - (hi ? mhi : mlo)) * (hi ? ihi : ilo);
+            }
+        if (c4 == 0) {
+#pragma unroll
+            for (int k = 0; k < kMmaMaxRungs; ++k) {
+                if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
+                const bool use = a.r.d[k] <= (float)(bw + kRowsPerWarp - 1);
+                float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
+                if (vlo) row[qlo] = use ? rs[k][0] * ilo : 0.f;
+                if (vhi) row[qhi] = use ? rs[k][1] * ihi : 0.f;
+            }
+        }
+    }
 
     const bool ok_v = mbar_wait(&bars[1], 0);
 
@@ -293,14 +361,17 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
         if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
         const float w = a.r.w[k], w1 = 1.f - w;
-        const float plo = exp2f(rs[k][0] - mlo), phi = exp2f(rs[k][1] - mhi);   // 0 when masked
+        // p, 0 when masked (SAVE: already formed, and the row sums taken)
+        const float plo = SAVE ? rs[k][0] : exp2f(rs[k][0] - mlo), phi = SAVE ? rs[k][1] : exp2f(rs[k][1] - mhi);
         // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
         // take the same rounded entries, as for the window band
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
         const float h00 = bf16_round(c0 * plo), h01 = bf16_round(c1 * plo), h20 = bf16_round(c7 * plo);
         const float h30 = bf16_round(c0 * phi), h31 = bf16_round(c1 * phi);
-        llo += quad_sum(h00 + h01 + h20);
-        lhi += quad_sum(h30 + h31);
+        if constexpr (!SAVE) {
+            llo += quad_sum(h00 + h01 + h20);
+            lhi += quad_sum(h30 + h31);
+        }
         const unsigned ahi[4] = {pack_bf16(h00, h01), 0u, pack_bf16(h20, 0.f), pack_bf16(h30, h31)};
         const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
@@ -316,7 +387,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const bool ok = ok_k && ok_v;
     const float inv_lo = ok ? 1.f / llo : __int_as_float(0x7fc00000);
     const float inv_hi = ok ? 1.f / lhi : __int_as_float(0x7fc00000);
-    __nv_bfloat16* O = reinterpret_cast<__nv_bfloat16*>(a.out) + ((size_t)bh * s.T) * kHeadDim;
+    __nv_bfloat16* O = reinterpret_cast<__nv_bfloat16*>(a.out) + rowbase * kHeadDim;
     if (vlo && wrel + g4 < kMmaTile) {
         __nv_bfloat16* row = O + (size_t)qlo * kHeadDim;
 #pragma unroll
@@ -339,7 +410,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 template <int NT, int TEAMS>
 cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const FwdArgs& a, const MmaLayout& L,
                       unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = fwd_mma_kernel<NT, TEAMS>;
+    auto kern = a.res_P ? fwd_mma_kernel<NT, TEAMS, true> : fwd_mma_kernel<NT, TEAMS, false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_kernel(kern, dim3(grid), dim3(kWarps * 32 * TEAMS), smem, st, mk, mv, a, L);
@@ -382,12 +453,16 @@ struct Iv { int a, b; };
 
 // Merge relative row intervals (sorted by start), round each merged interval up
 // to whole 8-row TMA boxes and lay them out one after another in shared memory.
+// An interval that starts before the rounded end of the one before it joins it:
+// the rounded intervals then cover disjoint relative rows, so every relative
+// row has exactly one shared row and a slab is contiguous in shared memory.
 void layout_intervals(Iv* iv, int n, MmaLayout* L) {
     for (int i = 1; i < n; ++i)                   // insertion sort by start
         for (int j = i; j > 0 && iv[j].a < iv[j - 1].a; --j) { Iv t = iv[j]; iv[j] = iv[j - 1]; iv[j - 1] = t; }
     int m = 0;
     for (int i = 0; i < n; ++i) {
-        if (m > 0 && iv[i].a <= iv[m - 1].b) { if (iv[i].b > iv[m - 1].b) iv[m - 1].b = iv[i].b; }
+        const int end8 = m > 0 ? iv[m - 1].a + (((iv[m - 1].b - iv[m - 1].a) + 7) & ~7) : 0;
+        if (m > 0 && iv[i].a < end8) { if (iv[i].b > iv[m - 1].b) iv[m - 1].b = iv[i].b; }
         else iv[m++] = iv[i];
     }
     L->n_iv = m;

@@ -68,10 +68,10 @@ def test_rung_params_match_oracle(alpha, W):
 def _call_fwd(**kw):
     lib = B.lib()
     args = dict(q=16, k=16, v=16, out=16, lse=16, B=1, H=2, T=8, D=64, W=2, alpha=1.0,
-                K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0, rk=None)
+                K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0, rk=None, res=None, fk=0)
     args.update(kw)
     f = np.array([1, 2, 3] + [5] * 40, dtype=np.float32)
-    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, 0, 0, args["rk"])
+    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, args["fk"], 0, args["rk"], args["res"])
     rc = lib.fibattn_fwd(args["q"], args["k"], args["v"], args["out"], args["lse"], args["B"], args["H"],
                          args["T"], args["D"], args["W"], args["alpha"], B._fptr(f), args["K"], args["dtype"],
                          ctypes.byref(o), args["ws"], args["wsb"], None)
@@ -85,6 +85,10 @@ def _call_fwd(**kw):
     (dict(Hkv=3), 1), (dict(q=0), 1), (dict(lse=0), 1), (dict(ws=0), 1),
     (dict(q=17), 1), (dict(out=24), 1), (dict(wsb=10), 1), (dict(rope_base=-2.0), 1),
     (dict(rk=24), 1),
+    # forward residuals: 16-byte alignment; only the tensor-core forward (bf16
+    # I/O, fwd_kernel 0 or 3, W <= 16) writes them -- refused before any launch
+    (dict(res=24), 1), (dict(res=256, dtype=0), 2), (dict(res=256, dtype=1, W=40), 2),
+    (dict(res=256, dtype=1, fk=1), 2), (dict(res=256, dtype=1, fk=2), 2),
 ])
 def test_fwd_rejects_bad_arguments(kw, code):
     rc, msg = _call_fwd(**kw)
@@ -135,6 +139,33 @@ def test_workspace_queries():
     assert fa.bwd_workspace_bytes(16, 8, 1024, 8, 15, torch.bfloat16) > fa.fwd_workspace_bytes(16, 8, 1024, 8, 15,
                                                                                                  torch.bfloat16)
     assert B.lib().fibattn_fwd_workspace_bytes(1, 2, 8, 128, 2, 3, 0, None) == 0    # invalid -> 0
+
+
+def test_residual_bytes():
+    """The residual buffer holds rotated q (fp16 [B,H,T,64]), p per slot (fp32
+    [B,H,W+1+K,T]) and rung score differences (fp32 [B,H,K,T]), each array from
+    the next multiple of 256 bytes; fp32 I/O and invalid sizes give 0."""
+    import torch
+
+    def up(x):
+        return (x + 255) // 256 * 256
+    for (Bn, H, T, W, K) in ((2, 3, 100, 8, 15), (1, 1, 1, 0, 0), (16, 8, 1024, 8, 15), (1, 2, 77, 3, 7)):
+        n = Bn * H * T
+        want = up(n * 128) + up(n * (W + 1 + K) * 4) + up(n * K * 4)
+        assert B.lib().fibattn_residual_bytes(Bn, H, T, 64, W, K, 1) == want
+        assert fa.residual_bytes(Bn, H, T, W, K, torch.bfloat16) == want
+        assert B.lib().fibattn_residual_bytes(Bn, H, T, 64, W, K, 0) == 0
+        buf = torch.zeros(want, dtype=torch.uint8)
+        qt, P, sd = fa.residual_views(buf, Bn, H, T, W, K)
+        assert qt.shape == (Bn, H, T, 64) and P.shape == (Bn, H, W + 1 + K, T) and sd.shape == (Bn, H, K, T)
+        # the (non-empty) views tile the buffer in order without overlap
+        ends = [(t.data_ptr() - buf.data_ptr(), t.data_ptr() - buf.data_ptr() + t.numel() * t.element_size())
+                for t in (qt, P, sd) if t.numel()]
+        assert ends[0][0] == 0 and ends[-1][1] <= want
+        assert all(a[1] <= b[0] for a, b in zip(ends, ends[1:]))
+        assert all(a % 256 == 0 for a, _ in ends)
+    assert B.lib().fibattn_residual_bytes(1, 2, 8, 128, 2, 3, 1) == 0                # D != 64
+    assert B.lib().fibattn_residual_bytes(1, 2, 8, 64, 2, 33, 1) == 0                # K > 32
 
 
 def test_missing_library_fails_loudly(monkeypatch, tmp_path):

@@ -38,8 +38,12 @@ def test_wrapper_equals_abi_backward():
     out = fa.fib_attention(qc, kc, vc, theta, f, 8)
     out.backward(g)
     alpha = fa.alpha_of_theta(0.37)
-    o2, l2 = fa.fwd(qc.detach(), kc.detach(), vc.detach(), alpha, f, 8)
-    dq, dk, dv, dth, _ = fa.bwd(qc.detach(), kc.detach(), vc.detach(), l2, g, alpha, f, 8, out=o2)
+    # the wrapper (bf16) keeps the forward's rotated keys and residuals for its backward
+    rk = fa.rotated_k_like(kc)
+    res = fa.residuals_like(qc, 8, len(f))
+    o2, l2 = fa.fwd(qc.detach(), kc.detach(), vc.detach(), alpha, f, 8, rotated_k=rk, residuals=res)
+    dq, dk, dv, dth, _ = fa.bwd(qc.detach(), kc.detach(), vc.detach(), l2, g, alpha, f, 8, out=o2, rotated_k=rk,
+                                residuals=res)
     torch.cuda.synchronize()
     assert torch.equal(out.detach(), o2)
     for a, b in ((qc.grad, dq), (kc.grad, dk), (vc.grad, dv)):

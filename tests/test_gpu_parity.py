@@ -121,6 +121,10 @@ SMALL = [
     (1, 2, 2, 100, 5, 0.8, "fib", 0, True),
     (1, 2, 2, 64, 63, 1.0, "fib", 15, True),
     (1, 1, 1, 2100, 8, 1.5, "fib", 15, True),
+    # slabs that start inside the 8-row rounding of the interval before them
+    # (rung 11 at alpha 0.87, T 333; rung 11 at the alpha of a learned stack, T 1024)
+    (2, 4, 2, 333, 8, 0.87, "fib", 15, True),
+    (1, 2, 2, 1024, 8, 0.8801671, "fib", 15, True),
 ]
 
 
