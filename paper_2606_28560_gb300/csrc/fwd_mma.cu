@@ -280,6 +280,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     llo = quad_sum(llo);
     lhi = quad_sum(lhi);
 
+    float ilo = 0.f, ihi = 0.f;                   // SAVE: reciprocal row sums
+    float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;
     if constexpr (SAVE) {
         // ---- residuals need the row sums before the value product: rung p in
         // place of the scores (0 when masked) and its bf16 entries summed here,
@@ -296,9 +298,10 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             lhi += quad_sum(bf16_round(c0 * rs[k][1]) + bf16_round(c1 * rs[k][1]));
         }
         // ---- residual p = exp2(s - m) / l of every slot of rows 0..14 (0 where
-        // not attended, also for rungs no row of the warp attends)
-        const float ilo = 1.f / llo, ihi = 1.f / lhi;
-        float* Pg = a.res_P + (size_t)bh * a.S * s.T;
+        // not attended): the window here, the rungs in the value loop, 0 for the
+        // active rungs no row of the warp attends (the tail of the sorted list)
+        ilo = 1.f / llo;
+        ihi = 1.f / lhi;
 #pragma unroll
         for (int j = 0; j < NT; ++j)
 #pragma unroll
@@ -310,13 +313,12 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
                     Pg[(size_t)t * s.T + bw + r] = exp2f(sw[j][e] - (hi ? mhi : mlo)) * (hi ? ihi : ilo);
             }
         if (c4 == 0) {
-#pragma unroll
-            for (int k = 0; k < kMmaMaxRungs; ++k) {
-                if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
-                const bool use = a.r.d[k] <= (float)(bw + kRowsPerWarp - 1);
-                float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
-                if (vlo) row[qlo] = use ? rs[k][0] * ilo : 0.f;
-                if (vhi) row[qhi] = use ? rs[k][1] * ihi : 0.f;
+            int i = L.n_act;
+            while (i > 0 && L.act_d[i - 1] > (float)(bw + kRowsPerWarp - 1)) --i;
+            for (; i < L.n_act; ++i) {
+                float* row = Pg + (size_t)(s.W + 1 + L.act_k[i]) * s.T;
+                if (vlo) row[qlo] = 0.f;
+                if (vhi) row[qhi] = 0.f;
             }
         }
     }
@@ -371,6 +373,10 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         if constexpr (!SAVE) {
             llo += quad_sum(h00 + h01 + h20);
             lhi += quad_sum(h30 + h31);
+        } else if (c4 == 0) {                     // residual p of rung k
+            float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
+            if (vlo) row[qlo] = plo * ilo;
+            if (vhi) row[qhi] = phi * ihi;
         }
         const unsigned ahi[4] = {pack_bf16(h00, h01), 0u, pack_bf16(h20, 0.f), pack_bf16(h30, h31)};
         const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
