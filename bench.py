@@ -317,15 +317,17 @@ def run_gpu(args, rank, world, device):
     barrier()
     torch.cuda.synchronize(device)
     clocks.mark("t0")
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    e0.record(stream)
-    for _ in range(args.steps):
+    # an event between replays: the whole region and each step's time
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 1)]
+    evs[0].record(stream)
+    for i in range(args.steps):
         graph.replay()
-    e1.record(stream)
+        evs[i + 1].record(stream)
     torch.cuda.synchronize(device)
     clocks.mark("t1")
     barrier()
-    ms = e0.elapsed_time(e1)
+    ms = evs[0].elapsed_time(evs[-1])
+    step_ms = sorted(evs[i].elapsed_time(evs[i + 1]) for i in range(args.steps))
     clk = clocks.stop() if rank == 0 else None
     # per-kernel device times: the same step captured with the library's event
     # nodes, replayed after the timed region
@@ -429,7 +431,8 @@ def run_gpu(args, rank, world, device):
     stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
                 algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
-                stack=stack, integer=integer, gqa=gqa, recompute=recompute)
+                stack=stack, integer=integer, gqa=gqa, recompute=recompute,
+                median_ms=step_ms[len(step_ms) // 2], min_ms=step_ms[0], max_ms=step_ms[-1])
 
 
 def run_gqa_forward(wl, device, args, stream):
@@ -584,6 +587,60 @@ def oracle_sample(seconds_target=10.0, nthreads=None):
                       f"fp64 C oracle, {spent:.1f} s wall on {nthreads} threads"}
 
 
+def cpu_model() -> str:
+    """The host CPU's model line (lscpu, else /proc/cpuinfo, else the machine type)."""
+    import platform
+    import subprocess
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as fh:
+            for line in fh:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
+
+
+def oracle_per_config():
+    """The fp64 oracle, as it stands, on one full layer of each measured
+    configuration, single-threaded and on all host cores: config 2 forward
+    (B16 H8 T1024 W8, linear schedule, layer 7), config 3 forward (B4 H8 T4096
+    W10, coprime schedule, layer 1), config 4 forward + backward (B16 H8 T1024
+    W8, learned schedule, layer 0).  Seconds per layer and query-heads/s."""
+    import oracle as O
+    from paper_2606_28560_gb300 import inputs
+    nall = os.cpu_count() or 1
+    f = O.fib_base(K)
+    cases = [("config2_fwd_W8", 16, 1024, 8, float(O.alpha_schedule("linear", L)[7]), False, 1),
+             ("config3_fwd_W10", 4, 4096, 10, float(O.alpha_schedule("coprime", L, stride=7)[1]), False, 2),
+             ("config4_fwd_bwd_W8", 16, 1024, 8,
+              float(O.alpha_schedule("learned", L, theta=inputs.theta_learned(L, seed=SEED))[0]), True, SEED)]
+    out = {"cpu_model": cpu_model(), "host_threads": nall}
+    for name, Bc, Tc, Wc, alpha, bwd, seed in cases:
+        q, k, v = inputs.qkv(Bc, H, Tc, seed=seed, dtype=torch.bfloat16)
+        g = inputs.dout(Bc, H, Tc, seed=seed + 100, dtype=torch.bfloat16)
+        q, k, v, g = (x.double().numpy() for x in (q, k, v, g))
+        d = O.offsets_fp32(float(np.float32(alpha)), f)
+        O.forward(q, k, v, Wc, d, nthreads=nall)          # untimed: first-touch of the oracle's buffers
+        row = {}
+        for nt in sorted({1, nall}):
+            t0 = time.perf_counter()
+            O.forward(q, k, v, Wc, d, nthreads=nt)
+            if bwd:
+                O.backward(q, k, v, g, Wc, d, nthreads=nt)
+            dt = time.perf_counter() - t0
+            row[f"threads_{nt}"] = {"s_per_layer": round(dt, 3), "query_heads_per_s": round(Bc * H * Tc / dt, 1)}
+        out[name] = row
+    return out
+
+
 def run_reference(args, rank, world):
     """Reference arm: the fp64 CPU oracle, timed as it stands on the host
     cores; each step is a bounded sample (one layer fwd+bwd or part of one)."""
@@ -643,8 +700,8 @@ def ncu_case(which: str):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=30)
-    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--steps", type=int, default=50)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--ncu-case", choices=["fwd", "bwd"], default=None,
@@ -673,11 +730,16 @@ def main():
     r = run_gpu(args, rank, world, device)
     if rank == 0:
         cpu = None
+        cpu_configs = None
         if not args.no_cpu_baseline and world == 1:
             cpu = oracle_sample(seconds_target=10.0)
+            cpu_configs = oracle_per_config()
         line = {
             "metric": METRIC, "value": r["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": r["ms"] / args.steps, "higher_is_better": True,
+            "warmup": args.warmup, "ms_per_step": r["ms"] / args.steps,
+            "step_ms": {"median": round(r["median_ms"], 4), "min": round(r["min_ms"], 4),
+                        "max": round(r["max_ms"], 4), "median_per_layer_us": round(r["median_ms"] / L * 1e3, 2)},
+            "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic N(0,1), seeded",
             "config": workload_config(),
             "timing": "CUDA graph of one step (16 layers fwd+bwd, programmatic dependent launches) replayed; "
@@ -693,6 +755,7 @@ def main():
             "backward_recomputing_scores_16_layers": r["recompute"],
             "forward_gqa_16_layers": r["gqa"],
             "cpu_baseline": cpu,
+            "cpu_oracle_per_config": cpu_configs,
             "e2e": r["e2e"],
             "gpu_launches": r["launches"],
             "clocks": r["clk"],
