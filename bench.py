@@ -247,9 +247,9 @@ def algorithmic_bytes(residuals=True):
 # file of the kernel changes, the figure is reported as null until the next
 # capture.
 NCU_TRAFFIC = {
-    "bwd_query_mma": {"bytes_at_b32": 169047552 + 73504768,
+    "bwd_query_mma": {"bytes_at_b32": 164770304 + 35469312,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "1d0b53c2b14bffabbce8a4e0e9e9af35c77db54b53349cbfedd61397a0ad6a5e"},
+                      "sha256": "66e7e6496c9123f7f564ceea4bbb5cd95e7b6670066adcde2abc83748cf59488"},
 }
 
 
