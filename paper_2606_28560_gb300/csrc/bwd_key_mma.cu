@@ -51,24 +51,15 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
                                          bool vhi, unsigned long long* bar, unsigned parity, bool& ok,
                                          float (*rv)[16]) {
     const Shape& s = a.s;
-    // ---- rung values of the warp's 16 slab columns, all active rungs at once
-    // (the loads are independent, so their latencies overlap): rv[i][x] = p or
-    // dS of query bw + s0 + x for active rung i in increasing d (0 past the end
-    // of the sequence and for the padding entries)
+    // ---- the values this warp reads, every load issued before the first use
+    // (their latencies overlap, with each other and with the staging copies):
+    // the window band at this thread's fragment entries, and the rung values
+    // of the warp's 16 slab columns for all active rungs, rv[i][x] = p or dS of
+    // query bw + s0 + x for active rung i in increasing d (0 past the end of
+    // the sequence and for the padding entries)
+    float bv[NT][4];
 #pragma unroll
-    for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
-        const int u = lane + 32 * j;
-        const int i = u >> 4, x = u & 15;
-        const int q = bw + L.act_s0[i] + x;
-        const bool use = i < L.n_act && q < s.T;
-        rv[i][x] = use ? X[(size_t)(s.W + 1 + L.act_k[i]) * s.T + q] : 0.f;
-    }
-    __syncwarp();
-    // ---- window band values (loaded while the copies are in flight)
-    unsigned band[NT][2];
-#pragma unroll
-    for (int j = 0; j < NT; ++j) {
-        float v[4];
+    for (int j = 0; j < NT; ++j)
 #pragma unroll
         for (int e = 0; e < 4; ++e) {
             const bool hi = e >= 2;
@@ -77,10 +68,28 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
             const int t = x - r;                              // query - key
             const int q = bw + x;
             const bool use = (hi ? vhi : vlo) && t >= 0 && t <= s.W && q < s.T;
-            v[e] = use ? X[(size_t)t * s.T + q] : 0.f;
+            bv[j][e] = use ? X[(size_t)t * s.T + q] : 0.f;
         }
-        band[j][0] = pack2<F16>(v[0], v[1]);
-        band[j][1] = pack2<F16>(v[2], v[3]);
+    float rvv[kMmaMaxRungs * 16 / 32];
+#pragma unroll
+    for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
+        const int u = lane + 32 * j;
+        const int i = u >> 4, x = u & 15;
+        const int q = bw + L.act_s0[i] + x;
+        const bool use = i < L.n_act && q < s.T;
+        rvv[j] = use ? X[(size_t)(s.W + 1 + L.act_k[i]) * s.T + q] : 0.f;
+    }
+#pragma unroll
+    for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
+        const int u = lane + 32 * j;
+        rv[u >> 4][u & 15] = rvv[j];
+    }
+    __syncwarp();
+    unsigned band[NT][2];
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+        band[j][0] = pack2<F16>(bv[j][0], bv[j][1]);
+        band[j][1] = pack2<F16>(bv[j][2], bv[j][3]);
     }
     ok = mbar_wait(bar, parity) && ok;
 
