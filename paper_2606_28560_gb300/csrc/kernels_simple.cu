@@ -453,9 +453,23 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
     if (grid > 152 * 16) grid = 152 * 16;       // 16 resident 256-thread blocks on each of 152 SMs
     if (bf16) {
         const int heads = (int)(rows / T);
+        // one wave: as many blocks as are resident at once (a partial second
+        // wave would run on a nearly idle GPU); the grid-stride loop spreads
+        // the remainder over every SM
         const long long gitems = (long long)((heads + kRopeHeads - 1) / kRopeHeads) * T * 4;
+        static int wave = 0;
+        if (wave == 0) {
+            int dev = 0, sms = 0, per_sm = 0;
+            if (cudaGetDevice(&dev) == cudaSuccess &&
+                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
+                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rope_rows_bf16_kernel, 256, 0) == cudaSuccess &&
+                sms > 0 && per_sm > 0)
+                wave = sms * per_sm;
+            else
+                wave = 152 * 3;
+        }
         long long g2 = (gitems + 255) / 256;
-        if (g2 > 152 * 8) g2 = 152 * 8;
+        if (g2 > wave) g2 = wave;
         return launch_kernel(rope_rows_bf16_kernel, dim3((unsigned)g2), dim3(256), 0, st,
                              reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), heads, T,
                              rp);
