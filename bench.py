@@ -436,9 +436,10 @@ def run_gpu(args, rank, world, device):
 
 
 def run_gqa_forward(wl, device, args, stream):
-    """The forward of the 16 layers at the paper's head split (H = 8 query
-    heads, Hkv = 2 kv heads; groups of 4 share each CTA's staged keys and
-    values), same B, T, W and schedule as the step, graphed."""
+    """The 16 layers at the paper's head split (H = 8 query heads, Hkv = 2 kv
+    heads), same B, T, W and schedule as the step, graphed: the forward alone
+    (groups of 4 query heads share each CTA's staged keys and values) and the
+    whole forward + backward step with residuals."""
     import paper_2606_28560_gb300 as fa
     from paper_2606_28560_gb300 import inputs
     Hkv = 2
@@ -448,28 +449,52 @@ def run_gqa_forward(wl, device, args, stream):
         v = torch.empty((B, Hkv, T, D), dtype=torch.bfloat16, device=device)
         inputs.device_normal_(k, 5000 + 2 * l)
         inputs.device_normal_(v, 5001 + 2 * l)
-        kv.append((k, v, torch.empty((B, Hkv, T, D), dtype=torch.float16, device=device)))
+        kv.append({"k": k, "v": v, "rk": torch.empty((B, Hkv, T, D), dtype=torch.float16, device=device),
+                   "dk": torch.empty_like(k), "dv": torch.empty_like(v),
+                   "res": fa.residuals_like(wl.q[l], W, K)})
+    ws_f = torch.empty(fa.fwd_workspace_bytes(B, H, T, W, K, torch.bfloat16, Hkv=Hkv), dtype=torch.uint8,
+                       device=device)
+    ws_b = torch.empty(fa.bwd_workspace_bytes(B, H, T, W, K, torch.bfloat16, Hkv=Hkv), dtype=torch.uint8,
+                       device=device)
 
-    def fwd_all():
+    def fwd_all(res=False):
         for l in range(L):
-            k, v, rk = kv[l]
-            fa.fwd(wl.q[l], k, v, wl.alphas[l], wl.f, W, out=wl.out[l], lse=wl.lse[l], workspace=wl.ws_f,
-                   rotated_k=rk)
+            c = kv[l]
+            fa.fwd(wl.q[l], c["k"], c["v"], wl.alphas[l], wl.f, W, out=wl.out[l], lse=wl.lse[l], workspace=ws_f,
+                   rotated_k=c["rk"], residuals=c["res"] if res else None)
 
-    g = capture(fwd_all, device, profile=False)
-    for _ in range(2):
-        g.replay()
-    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    reps = max(3, args.steps // 3)
-    a0.record(stream)
-    for _ in range(reps):
-        g.replay()
-    a1.record(stream)
-    torch.cuda.synchronize(device)
-    layer_us = a0.elapsed_time(a1) / (reps * L) * 1e3
-    del g, kv
-    return {"B": B, "H": H, "Hkv": Hkv, "T": T, "W": W, "layer_us_incl_rope": round(layer_us, 2),
-            "query_heads_per_s": round(B * H * T / (layer_us * 1e-6), 1)}
+    def step():
+        fwd_all(True)
+        for l in reversed(range(L)):
+            c = kv[l]
+            fa.bwd(wl.q[l], c["k"], c["v"], wl.lse[l], wl.g[l], wl.alphas[l], wl.f, W, out=wl.out[l],
+                   dq=wl.dq[l], dk=c["dk"], dv=c["dv"], dtheta=wl.dth[l], dd=wl.dd[l], workspace=ws_b,
+                   rotated_k=c["rk"], residuals=c["res"])
+
+    out = {"B": B, "H": H, "Hkv": Hkv, "T": T, "W": W}
+    for name, fn in (("fwd", fwd_all), ("fwd_bwd", step)):
+        fn()
+        torch.cuda.synchronize(device)
+        g = capture(fn, device, profile=False)
+        for _ in range(2):
+            g.replay()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(3, args.steps // 3)
+        a0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        a1.record(stream)
+        torch.cuda.synchronize(device)
+        ms = a0.elapsed_time(a1) / reps
+        del g
+        if name == "fwd":
+            out["layer_us_incl_rope"] = round(ms / L * 1e3, 2)
+            out["query_heads_per_s"] = round(B * H * T * L / (ms * 1e-3), 1)
+        else:
+            out["fwd_bwd_ms_per_step"] = round(ms, 4)
+            out["fwd_bwd_query_heads_per_s"] = round(B * H * T * L / (ms * 1e-3), 1)
+    del kv
+    return out
 
 
 def run_autograd_stack(device, warm=2, reps=3):

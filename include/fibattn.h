@@ -129,6 +129,8 @@ int fibattn_fwd(const void* q, const void* k, const void* v,
  * dL/dalpha = sum_k f_k dd_k.  With both NULL (a fixed alpha schedule, alpha
  * not trained) the rung-distance gradient is not computed at all.
  * At an integer d_k the distance derivative is one-sided, from above.
+ * dq, dk, dv, dtheta and dd may not alias each other, an input, the
+ * residuals or the workspace.
  * ------------------------------------------------------------------------- */
 size_t fibattn_bwd_workspace_bytes(int B, int H, int T, int D, int W, int K,
                                    int dtype, const fibattn_opts* opts);

@@ -164,7 +164,13 @@ template <int NT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ RowMaps tmG, BwdArgs a,
                    MmaLayout L) {
-    grid_dependency_sync();
+    // The kernel before this one is the query pass of the same call.  With the
+    // forward residuals the first pass reads only p and dO, which it does not
+    // write, so the wait for it comes before the second pass (dS) and before
+    // block 0 sums the query pass's rung partials.
+    pdl_trigger();
+    const bool early = a.saved != 0;
+    if (!early) pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bar;
     __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
@@ -191,13 +197,17 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     __syncthreads();
-    if (blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
+    if (!early && blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
 
     unsigned parity = 0;
     bool ok = true;
     const size_t krow0 = (size_t)bhk * s.T;
 #pragma unroll 1
     for (int pass = 0; pass < 2; ++pass) {                // 0: dv from dO rows; 1: dk~ from q~ rows
+        if (pass == 1 && early) {
+            pdl_wait();
+            if (blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
+        }
         float acc[8][4];
 #pragma unroll
         for (int n = 0; n < 8; ++n) acc[n][0] = acc[n][1] = acc[n][2] = acc[n][3] = 0.f;

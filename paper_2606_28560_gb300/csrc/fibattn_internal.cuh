@@ -255,6 +255,12 @@ __device__ __forceinline__ void grid_dependency_sync() {
     asm volatile("griddepcontrol.wait;\n" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
 }
+// The two halves, for a kernel that knows which of its inputs the kernel
+// before it (launched by the same library call) does not write: it lets the
+// next launch be scheduled at once, reads those inputs, and waits only before
+// touching anything the previous kernel may produce.
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory"); }
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
 
 // Host: whether launches carry the programmatic-serialisation attribute
 // (environment FIBATTN_PDL=0 turns it off).

@@ -57,7 +57,11 @@ template <int NT, int TEAMS, bool SAVE>
 __global__ void __launch_bounds__(kWarps * 32 * TEAMS, TEAMS == 1 ? 2 : 1)
 fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
                FwdArgs a, MmaLayout L) {
-    grid_dependency_sync();
+    // The kernel before this one is the key rotation of the same call, which
+    // writes only the rotated keys: the query rows are loaded before waiting
+    // for it (TEAMS = 1; the grouped form waits at once).
+    pdl_trigger();
+    if (TEAMS == 2) pdl_wait();
     constexpr int Wp = NT * 8 - 16;               // window rows before the tile
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[2];
@@ -76,6 +80,25 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const int g4 = lane >> 2, c4 = lane & 3;
     const int wrel = warp * kRowsPerWarp;         // tile-relative first row of this warp
     const int bw = i0 + wrel;                     // absolute first row
+
+    // raw q words of this thread (rows g4, g4+8; dims 16kc + 2c4.. and 16kc + 8 + 2c4..)
+    unsigned qraw[2][4][2];
+    auto load_q = [&](int bhq) {
+        const __nv_bfloat16* Q = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)bhq * s.T) * kHeadDim;
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            const __nv_bfloat16* row = Q + (size_t)min(bw + g4 + 8 * half, s.T - 1) * kHeadDim;
+#pragma unroll
+            for (int kc = 0; kc < 4; ++kc) {
+                qraw[half][kc][0] = *reinterpret_cast<const unsigned*>(row + 16 * kc + 2 * c4);
+                qraw[half][kc][1] = *reinterpret_cast<const unsigned*>(row + 16 * kc + 8 + 2 * c4);
+            }
+        }
+    };
+    if (TEAMS == 1) {
+        load_q(unit);
+        pdl_wait();
+    }
 
     // ---- issue the key copies (and for TEAMS = 2 the value copies) (warp 0)
     if (tid == 0) {
@@ -98,7 +121,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     // Thread dims: 16kc + 2c4 + {0,1} and 16kc + 8 + 2c4 + {0,1} for kc = 0..3.
     unsigned qa[4][4];
     {
-        const __nv_bfloat16* Q = reinterpret_cast<const __nv_bfloat16*>(a.q) + ((size_t)bh * s.T) * kHeadDim;
+        if (TEAMS == 2) load_q(bh);
         // cos/sin of the 8 pairs at position bw+g4, then advanced by 8 positions
         // for row g4+8 with the host's fp64 cos/sin(8 theta_m)
         float cs[2][4], sn[2][4];
@@ -112,13 +135,11 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-            const int pos = min(pos0 + 8 * half, s.T - 1);
-            const __nv_bfloat16* row = Q + (size_t)pos * kHeadDim;
             float x[4][4];                        // [kc][j]: dims 16kc + {2c4, 2c4+1, 2c4+8, 2c4+9}
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
-                const unsigned u0 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 2 * c4);
-                const unsigned u1 = *reinterpret_cast<const unsigned*>(row + 16 * kc + 8 + 2 * c4);
+                const unsigned u0 = qraw[half][kc][0];
+                const unsigned u1 = qraw[half][kc][1];
                 x[kc][0] = __uint_as_float(u0 << 16); x[kc][1] = __uint_as_float(u0 & 0xffff0000u);
                 x[kc][2] = __uint_as_float(u1 << 16); x[kc][3] = __uint_as_float(u1 & 0xffff0000u);
             }
