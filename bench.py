@@ -247,9 +247,9 @@ def algorithmic_bytes(residuals=True):
 # file of the kernel changes, the figure is reported as null until the next
 # capture.
 NCU_TRAFFIC = {
-    "bwd_query_mma": {"bytes_at_b32": 164770304 + 35469312,
+    "bwd_query_mma": {"bytes_at_b32": 164776960 + 35540224,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "66e7e6496c9123f7f564ceea4bbb5cd95e7b6670066adcde2abc83748cf59488"},
+                      "sha256": "91c0baf805f1f7ad76e1b8a97b6bc3f03c79dce39fc014cfd8fb2a383b40c75b"},
 }
 
 
