@@ -298,8 +298,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         pa[j][0] = pack_bf16(p0, p1);
         pa[j][1] = pack_bf16(p2, p3);
     }
-    llo = quad_sum(llo);
-    lhi = quad_sum(lhi);
+    // (the row sums stay per-lane partials until every slot is in; one quad
+    // sum per row then completes them)
 
     float ilo = 0.f, ihi = 0.f;                   // SAVE: reciprocal row sums
     float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;
@@ -315,9 +315,11 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             rs[k][0] = exp2f(rs[k][0] - mlo);
             rs[k][1] = exp2f(rs[k][1] - mhi);
             const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-            llo += quad_sum(bf16_round(c0 * rs[k][0]) + bf16_round(c1 * rs[k][0]) + bf16_round(c7 * rs[k][0]));
-            lhi += quad_sum(bf16_round(c0 * rs[k][1]) + bf16_round(c1 * rs[k][1]));
+            llo += bf16_round(c0 * rs[k][0]) + bf16_round(c1 * rs[k][0]) + bf16_round(c7 * rs[k][0]);
+            lhi += bf16_round(c0 * rs[k][1]) + bf16_round(c1 * rs[k][1]);
         }
+        llo = quad_sum(llo);
+        lhi = quad_sum(lhi);
         // ---- residual p = exp2(s - m) / l of every slot of rows 0..14 (0 where
         // not attended): the window here, the rungs in the value loop, 0 for the
         // active rungs no row of the warp attends (the tail of the sorted list)
@@ -392,8 +394,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         const float h00 = bf16_round(c0 * plo), h01 = bf16_round(c1 * plo), h20 = bf16_round(c7 * plo);
         const float h30 = bf16_round(c0 * phi), h31 = bf16_round(c1 * phi);
         if constexpr (!SAVE) {
-            llo += quad_sum(h00 + h01 + h20);
-            lhi += quad_sum(h30 + h31);
+            llo += h00 + h01 + h20;
+            lhi += h30 + h31;
         } else if (c4 == 0) {                     // residual p of rung k
             float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
             if (vlo) row[qlo] = plo * ilo;
@@ -408,6 +410,11 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             mma_bf16_16816(o[n], ahi, b0, b1);
             mma_bf16_16816(o[n + 1], ahi, b2, b3);
         }
+    }
+
+    if constexpr (!SAVE) {
+        llo = quad_sum(llo);
+        lhi = quad_sum(lhi);
     }
 
     // ---- normalise and store rows 0..14 of the tile
