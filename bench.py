@@ -214,20 +214,22 @@ class Workload:
 def algorithmic_bytes(residuals=True):
     """Bytes each kernel must move once per launch (bf16 rows of 128 B,
     fp32 lse and fp32 P / dS slots).  S = W + 1 + K slots per query.  With
-    the forward residuals the forward also writes q~ (fp16 rows), p per slot
-    and the rung score differences, and the query pass reads those instead of
-    q, lse and the rotated keys' scores."""
+    the forward residuals the forward also writes q~ (fp16 rows), the
+    unnormalised weight per slot, the rung score differences and 1 / (weight
+    sum) per query, and the backward reads those instead of recomputing the
+    scores."""
     n = B * H * T
     S = W + 1 + K
     rows = n * ROW_BYTES
     if residuals:
         return {
-            # Q, K~, V read; O, q~ written; lse, p per slot, sd written
-            "fwd": 5 * rows + 4 * n + 4 * n * S + 4 * n * K,
+            # Q, K~, V read; O, q~ written; lse, weight per slot, sd, 1/l written
+            "fwd": 5 * rows + 2 * 4 * n + 4 * n * S + 4 * n * K,
             "rope_k": 2 * rows,
-            # dO, O, K~, V read; dQ written; p, sd read; dS written
-            "bwd_query_mma": 5 * rows + 2 * 4 * n * S + 4 * n * K,
-            "bwd_key_mma": 4 * rows + 2 * 4 * n * S,       # Q~ dO read, dK dV written, P/dS read
+            # dO, O, K~, V read; dQ written; weights, sd, 1/l read; dS written
+            "bwd_query_mma": 5 * rows + 2 * 4 * n * S + 4 * n * K + 4 * n,
+            # Q~ dO read, dK dV written, weights/dS and 1/l read
+            "bwd_key_mma": 4 * rows + 2 * 4 * n * S + 4 * n,
         }
     return {
         "fwd": 4 * rows + 4 * n,                           # Q, K~, V read; O written; lse

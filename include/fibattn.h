@@ -79,13 +79,16 @@ typedef struct {
                           16-byte aligned [NULL].  Given it, fibattn_fwd also writes
                           what the backward would otherwise recompute from q and k:
                           the RoPE-rotated queries (fp16 [B][H][T][D]), the
-                          softmax probability of every slot (fp32 [B][H][S][T],
-                          S = W + 1 + K: window distances 0..W, then rung k at
-                          W + 1 + k; 0 where not attended; rungs that are never
-                          read -- dropped by dedup or beyond T's reach -- are
-                          left unwritten) and the far-minus-floor raw score
-                          q~ . (k~_far - k~_floor) of every rung (fp32
-                          [B][H][K][T]); the three arrays follow one another in
+                          unnormalised softmax weight exp(s - max) of every
+                          slot (fp32 [B][H][S][T], S = W + 1 + K: window
+                          distances 0..W, then rung k at W + 1 + k; 0 where not
+                          attended; rungs that are never read -- dropped by
+                          dedup or beyond T's reach -- are left unwritten), the
+                          far-minus-floor raw score q~ . (k~_far - k~_floor) of
+                          every rung (fp32 [B][H][K][T]) and 1 / (sum of the
+                          weights) per query (fp32 [B][H][T]), so that the
+                          probability is weight / sum; the four arrays follow
+                          one another in
                           that order, each starting at the next multiple of 256
                           bytes.  Only the tensor-core forward writes them:
                           bf16 I/O, and fwd_kernel 0 or 3 with its layout applying;

@@ -119,19 +119,23 @@ def residuals_like(q: torch.Tensor, W: int, K: int) -> torch.Tensor:
 
 
 def residual_views(res: torch.Tensor, B, H, T, W, K):
-    """Views of a residual buffer: rotated q (fp16 [B,H,T,64]), p per slot
-    (fp32 [B,H,W+1+K,T]) and far-minus-floor rung scores (fp32 [B,H,K,T]);
-    the arrays follow one another, each from the next multiple of 256 bytes."""
+    """Views of a residual buffer: rotated q (fp16 [B,H,T,64]), the
+    unnormalised softmax weight exp(s - max) per slot (fp32 [B,H,W+1+K,T]),
+    far-minus-floor rung scores (fp32 [B,H,K,T]) and 1 / (sum of the weights)
+    per query (fp32 [B,H,T]; p = weight * that); the arrays follow one another,
+    each from the next multiple of 256 bytes."""
     def up(x):
         return (x + 255) // 256 * 256
     n = B * H * T
     S = W + 1 + K
     o_p = up(n * 64 * 2)
     o_sd = o_p + up(n * S * 4)
+    o_il = o_sd + up(n * K * 4)
     qt = res[:n * 128].view(torch.float16).view(B, H, T, 64)
     P = res[o_p:o_p + n * S * 4].view(torch.float32).view(B, H, S, T)
     sd = res[o_sd:o_sd + n * K * 4].view(torch.float32).view(B, H, K, T)
-    return qt, P, sd
+    il = res[o_il:o_il + n * 4].view(torch.float32).view(B, H, T)
+    return qt, P, sd, il
 
 
 def _check_residuals(res, q, W, K):

@@ -45,12 +45,27 @@ __device__ __forceinline__ void mma1688(float* d, unsigned a0, unsigned a1, unsi
 
 // One staged tensor of one query head: accumulate banded A x staged rows.
 // X: p or dS of this query head, slot-major [S][T]; F16: the operand type.
+// IL (p from the forward residuals, unnormalised): 1 / (row sum) per query
+// of this head; the warp copies the entries its values need into its rung
+// table and its band strip (wil, 32 floats) and scales each value.
 template <int NT, bool F16>
 __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, const BwdArgs& a, const MmaLayout& L,
                                          unsigned sbase, int bw, int wrel, int g4, int c4, int lane, bool vlo,
                                          bool vhi, unsigned long long* bar, unsigned parity, bool& ok,
-                                         float (*rv)[16]) {
+                                         float (*rv)[16], const float* IL = nullptr, float* wil = nullptr) {
     const Shape& s = a.s;
+    if (IL) {                                     // 1 / row sum of the queries the values below belong to
+#pragma unroll
+        for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
+            const int u = lane + 32 * j;
+            const int i = u >> 4, x = u & 15;
+            const int q = bw + L.act_s0[i] + x;
+            const bool use = i < L.n_act && q < s.T;
+            cp_async4(&rv[i][x], IL + (use ? q : 0), use);
+        }
+        cp_async4(wil + lane, IL + (bw + lane < s.T ? bw + lane : 0), bw + lane < s.T);
+        asm volatile("cp.async.commit_group;\n" ::: "memory");
+    }
     // ---- the values this warp reads, every load issued before the first use
     // (their latencies overlap, with each other and with the staging copies):
     // the window band at this thread's fragment entries, and the rung values
@@ -78,6 +93,20 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
         const int q = bw + L.act_s0[i] + x;
         const bool use = i < L.n_act && q < s.T;
         rvv[j] = use ? X[(size_t)(s.W + 1 + L.act_k[i]) * s.T + q] : 0.f;
+    }
+    if (IL) {
+        asm volatile("cp.async.wait_group 0;\n" ::: "memory");
+        __syncwarp();
+#pragma unroll
+        for (int j = 0; j < NT; ++j)
+#pragma unroll
+            for (int e = 0; e < 4; ++e) bv[j][e] *= wil[8 * j + 2 * c4 + (e & 1)];
+#pragma unroll
+        for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
+            const int u = lane + 32 * j;
+            rvv[j] *= rv[u >> 4][u & 15];
+        }
+        __syncwarp();                             // every lane has read its entries before the table is rewritten
     }
 #pragma unroll
     for (int j = 0; j < kMmaMaxRungs * 16 / 32; ++j) {
@@ -174,6 +203,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bar;
     __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
+    __shared__ float wils[kWarps][32];                    // per warp: 1 / row sum of its band queries
     __shared__ float red[kMmaMaxRungs];                   // block 0: dL/dd_k
     __shared__ long long red64[kWarps * kMmaMaxRungs];
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
@@ -221,7 +251,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
             }
             if (pass == 0)
                 key_pass<NT, false>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
-                                       rvals[warp]);
+                                       rvals[warp], early ? a.res_il + (size_t)qhead * s.T : nullptr, wils[warp]);
             else
                 key_pass<NT, true>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
                                       rvals[warp]);
@@ -293,8 +323,11 @@ cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, co
 }  // namespace
 
 size_t bwd_key_mma_static_smem() {
-    return sizeof(float) * (kWarps * kMmaMaxRungs * 16 + kMmaMaxRungs) + sizeof(long long) * kWarps * kMmaMaxRungs + 64;
+    return sizeof(float) * (kWarps * kMmaMaxRungs * 16 + kWarps * 32 + kMmaMaxRungs) +
+           sizeof(long long) * kWarps * kMmaMaxRungs + 64;
 }
+
+size_t bwd_key_mma_smem_bytes(const MmaLayout& L, bool) { return fwd_mma_smem_bytes(L); }
 
 int bwd_key_mma_blocks(const Shape& s) {
     const long long tiles = (s.T + kMmaTile - 1) / kMmaTile;
@@ -309,7 +342,7 @@ cudaError_t launch_bwd_key_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_
     if (!encode_row_maps(&mq, a.qt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
         !encode_row_maps(&mg, a.dout, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
         return cudaErrorInvalidValue;
-    const size_t smem = fwd_mma_smem_bytes(L);
+    const size_t smem = bwd_key_mma_smem_bytes(L, a.saved != 0);
     switch (L.nt) {
     case 2: return launch_nt<2>(mq, mg, a, L, (unsigned)grid, smem, st);
     case 3: return launch_nt<3>(mq, mg, a, L, (unsigned)grid, smem, st);

@@ -41,16 +41,11 @@ constexpr int kRowsPerWarp = 15;
 __device__ __forceinline__ float bf_lo(unsigned u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 0xffff0000u); }
 
-// 4-byte asynchronous copy global -> shared; zero-filled when !full.
-__device__ __forceinline__ void cp_async4(const float* dst, const float* src, bool full) {
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n"
-                 :: "r"(smem_u32(dst)), "l"(src), "r"(full ? 4 : 0) : "memory");
-}
-
 // DD: also the rung-distance gradient dL/dd_k (off when the caller asks for
 // neither dtheta nor dd, e.g. a fixed alpha schedule).
-// SV: p of every slot and the far-minus-floor rung scores come from the
-// forward's residuals (p and the rotated queries serve the key pass too), so
+// SV: p of every slot (stored unnormalised, with 1 / row sum per query) and
+// the far-minus-floor rung scores come from the forward's residuals (p and the
+// rotated queries serve the key pass too), so
 // the scores are not recomputed: dS = p (dp - Delta) is formed in the value
 // phase and the key phase only accumulates dq~.
 template <int NT, bool DD, bool SV>
@@ -115,11 +110,15 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     float* Pg = a.Ps + (size_t)bh * a.S * s.T;       // [slot][T] of this head
     float* DSg = a.DSs + (size_t)bh * a.S * s.T;
 
-    // SV: the residual p of the window band at this thread's accumulator
-    // entries (registers), and p and sd of the active rungs for the tile's
-    // rows (shared memory, 4-byte asynchronous copies by every thread)
+    // SV: the residual (unnormalised) p of the window band at this thread's
+    // accumulator entries and 1 / (row sum) of its rows (registers), and p
+    // and sd of the active rungs for the tile's rows (shared memory, 4-byte
+    // asynchronous copies by every thread); p = residual p / row sum
     float pb[NT][4];
+    float il_lo = 0.f, il_hi = 0.f;
     if constexpr (SV) {
+        il_lo = vlo ? a.res_il[rowbase + qlo] : 0.f;
+        il_hi = vhi ? a.res_il[rowbase + qhi] : 0.f;
 #pragma unroll
         for (int j = 0; j < NT; ++j)
 #pragma unroll
@@ -315,7 +314,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 const bool hi = e >= 2;
                 const int r = hi ? g4 + 8 : g4;
                 const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
-                dsv[e] = pb[j][e] * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
+                dsv[e] = pb[j][e] * (hi ? il_hi : il_lo) * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
                 if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) DSg[(size_t)t * s.T + bw + r] = dsv[e];
             }
             dsa[j][0] = pack_f16(dsv[0], dsv[1]);
@@ -386,7 +385,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
             const int row = wrel + g4 + (up ? 8 : 0);
             const bool rv = up ? vhi : vlo;
-            const float p = rv ? psd[0][i][row] : 0.f;
+            const float p = rv ? psd[0][i][row] * (up ? il_hi : il_lo) : 0.f;
             const float e = dp - (up ? dlt_hi : dlt_lo);
             const float ds = p * e;
             if constexpr (DD) {

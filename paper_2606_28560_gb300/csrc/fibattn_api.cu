@@ -131,10 +131,11 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
     return s;
 }
 
-// Forward residuals (fibattn_opts.residuals): rotated q (fp16), p per slot
-// (slot-major), far-minus-floor rung scores (rung-major).
+// Forward residuals (fibattn_opts.residuals): rotated q (fp16), unnormalised
+// p per slot (slot-major), far-minus-floor rung scores (rung-major), 1 / (row
+// sum) per query.
 struct ResLayout {
-    size_t qt, P, sd, total;
+    size_t qt, P, sd, il, total;
 };
 
 ResLayout res_layout(int B, int H, int T, int W, int K) {
@@ -143,7 +144,8 @@ ResLayout res_layout(int B, int H, int T, int W, int K) {
     L.qt = 0;
     L.P = align256(n * kHeadDim * 2);
     L.sd = L.P + align256(n * ((size_t)W + 1 + K) * 4);
-    L.total = L.sd + align256(n * (size_t)K * 4);
+    L.il = L.sd + align256(n * (size_t)K * 4);
+    L.total = L.il + align256(n * 4);
     return L;
 }
 
@@ -388,6 +390,7 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
         a.res_qt = rb + R.qt;
         a.res_P = reinterpret_cast<float*>(rb + R.P);
         a.res_sd = reinterpret_cast<float*>(rb + R.sd);
+        a.res_il = reinterpret_cast<float*>(rb + R.il);
     }
     a.S = W + 1 + K;
     if ((rc = bind_context())) return rc;
@@ -463,13 +466,15 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         return fail(FIBATTN_ERR_UNSUPPORTED, "tensor-core backward needs bf16, out, W <= 16, K <= 16 and a staged row "
                                              "union that fits shared memory");
     if (mma_ok) a.nblk_q = bwd_mma_blocks(a.s);
-    if (mma_ok && o.residuals) {                 // p, sd and q~ from the forward
+    if (mma_ok && o.residuals &&                 // p, sd and q~ from the forward
+        bwd_key_mma_smem_bytes(KL, true) + bwd_key_mma_static_smem() <= 227 * 1024) {
         const ResLayout R = res_layout(B, H, T, W, K);
         char* rb = reinterpret_cast<char*>(o.residuals);
         a.saved = 1;
         a.qt = rb + R.qt;
         a.Ps = reinterpret_cast<float*>(rb + R.P);
         a.res_sd = reinterpret_cast<const float*>(rb + R.sd);
+        a.res_il = reinterpret_cast<const float*>(rb + R.il);
     }
     cudaError_t e;
     if ((rc = bind_context())) return rc;

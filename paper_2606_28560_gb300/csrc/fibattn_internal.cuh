@@ -47,12 +47,13 @@ struct FwdArgs {
     void* out;                // [B,H,T,D]
     float* lse;               // [B,H,T]
     // Optional residuals for the backward (tensor-core forward only; all
-    // nullptr when not asked for): the rotated queries, the probability of
-    // every slot (0 where not attended) and the far-minus-floor raw score of
-    // every rung row.
+    // nullptr when not asked for): the rotated queries, the unnormalised
+    // probability exp(s - max) of every slot (0 where not attended), the
+    // far-minus-floor raw score of every rung row and 1 / (row sum) per query.
     void* res_qt;             // fp16 [B,H,T,D]
     float* res_P;             // slot-major [B,H,S,T], S = W + 1 + K
     float* res_sd;            // rung-major [B,H,K,T]
+    float* res_il;            // [B,H,T]
     int S;
     Shape s;
     RungParams r;
@@ -81,9 +82,10 @@ struct BwdArgs {
     float* Ps;                // tensor-core path, slot-major [B,H,S,T]: p      (P region)
     float* DSs;               //                                      dS = p (dp - Delta)  (DP region)
     long long* rpart;         // per query-pass block dL/dd_k partials, 2^-32 fixed point [kMaxRungs][nblk_q]
+    const float* res_il;      // forward residual 1 / (row sum) [B,H,T] (p = Ps[slot] * res_il)
     const float* res_sd;      // forward residual far-minus-floor rung scores [B,H,K,T], or nullptr;
                               // when the forward residuals are used, Ps and qt point into them
-    int saved;                // tensor-core passes read p (Ps), sd and q~ (qt) from the forward residuals
+    int saved;                // tensor-core passes read p (Ps, unnormalised), sd and q~ (qt) from the forward residuals
     int nblk_q;               // query-pass blocks
     int S;                    // slots per query = W + 1 + K
     float alpha;

@@ -51,8 +51,9 @@ constexpr int kRowsPerWarp = 15;                 // useful query rows of a 16-ro
 // two buffers, and each team of 8 warps loops over its share of the group's
 // query heads (team t takes heads t, t + 2, ...).
 // SAVE: also write the residuals the tensor-core backward reads instead of
-// recomputing the scores -- the rotated queries, p of every slot (normalised,
-// fp32; 0 where not attended) and the far-minus-floor raw score of every rung.
+// recomputing the scores, each where it is formed -- the rotated queries, the
+// unnormalised p = exp(s - max) of every slot (fp32, 0 where not attended),
+// the far-minus-floor raw score of every rung and 1 / (row sum) per query.
 template <int NT, int TEAMS, bool SAVE>
 __global__ void __launch_bounds__(kWarps * 32 * TEAMS, TEAMS == 1 ? 2 : 1)
 fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowMaps tmV,
@@ -289,52 +290,34 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     if (mhi == -INFINITY) mhi = 0.f;
     float llo = 0.f, lhi = 0.f;
     unsigned pa[NT][2];                           // window band P as bf16 A fragments
+    float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;   // residual exp(s - max) per slot
 #pragma unroll
     for (int j = 0; j < NT; ++j) {
-        const float p0 = bf16_round(exp2f(sw[j][0] - mlo)), p1 = bf16_round(exp2f(sw[j][1] - mlo));
-        const float p2 = bf16_round(exp2f(sw[j][2] - mhi)), p3 = bf16_round(exp2f(sw[j][3] - mhi));
+        const float e0 = exp2f(sw[j][0] - mlo), e1 = exp2f(sw[j][1] - mlo);
+        const float e2 = exp2f(sw[j][2] - mhi), e3 = exp2f(sw[j][3] - mhi);
+        const float p0 = bf16_round(e0), p1 = bf16_round(e1), p2 = bf16_round(e2), p3 = bf16_round(e3);
         llo += p0 + p1;
         lhi += p2 + p3;
         pa[j][0] = pack_bf16(p0, p1);
         pa[j][1] = pack_bf16(p2, p3);
-    }
-    // (the row sums stay per-lane partials until every slot is in; one quad
-    // sum per row then completes them)
-
-    float ilo = 0.f, ihi = 0.f;                   // SAVE: reciprocal row sums
-    float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;
-    if constexpr (SAVE) {
-        // ---- residuals need the row sums before the value product: rung p in
-        // place of the scores (0 when masked) and its bf16 entries summed here,
-        // in the order the value loop would take them
-#pragma unroll
-        for (int k = 0; k < kMmaMaxRungs; ++k) {
-            if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
-            if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
-            const float w = a.r.w[k], w1 = 1.f - w;
-            rs[k][0] = exp2f(rs[k][0] - mlo);
-            rs[k][1] = exp2f(rs[k][1] - mhi);
-            const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-            llo += bf16_round(c0 * rs[k][0]) + bf16_round(c1 * rs[k][0]) + bf16_round(c7 * rs[k][0]);
-            lhi += bf16_round(c0 * rs[k][1]) + bf16_round(c1 * rs[k][1]);
-        }
-        llo = quad_sum(llo);
-        lhi = quad_sum(lhi);
-        // ---- residual p = exp2(s - m) / l of every slot of rows 0..14 (0 where
-        // not attended): the window here, the rungs in the value loop, 0 for the
-        // active rungs no row of the warp attends (the tail of the sorted list)
-        ilo = 1.f / llo;
-        ihi = 1.f / lhi;
-#pragma unroll
-        for (int j = 0; j < NT; ++j)
+        if constexpr (SAVE) {                     // window slot t of rows 0..14 (0 before position 0)
+            const float ev[4] = {e0, e1, e2, e3};
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const bool hi = e >= 2;
                 const int r = hi ? g4 + 8 : g4;
                 const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
-                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W)
-                    Pg[(size_t)t * s.T + bw + r] = exp2f(sw[j][e] - (hi ? mhi : mlo)) * (hi ? ihi : ilo);
+                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) Pg[(size_t)t * s.T + bw + r] = ev[e];
             }
+        }
+    }
+    // (the row sums stay per-lane partials until every slot is in; one quad
+    // sum per row then completes them)
+
+
+    if constexpr (SAVE) {
+        // ---- residual p of the active rungs no row of the warp attends (the
+        // tail of the list sorted by d): 0
         if (c4 == 0) {
             int i = L.n_act;
             while (i > 0 && L.act_d[i - 1] > (float)(bw + kRowsPerWarp - 1)) --i;
@@ -386,20 +369,20 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
         if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
         const float w = a.r.w[k], w1 = 1.f - w;
-        // p, 0 when masked (SAVE: already formed, and the row sums taken)
-        const float plo = SAVE ? rs[k][0] : exp2f(rs[k][0] - mlo), phi = SAVE ? rs[k][1] : exp2f(rs[k][1] - mhi);
+        const float plo = exp2f(rs[k][0] - mlo), phi = exp2f(rs[k][1] - mhi);   // 0 when masked
         // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
         // take the same rounded entries, as for the window band
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
         const float h00 = bf16_round(c0 * plo), h01 = bf16_round(c1 * plo), h20 = bf16_round(c7 * plo);
         const float h30 = bf16_round(c0 * phi), h31 = bf16_round(c1 * phi);
-        if constexpr (!SAVE) {
-            llo += h00 + h01 + h20;
-            lhi += h30 + h31;
-        } else if (c4 == 0) {                     // residual p of rung k
-            float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
-            if (vlo) row[qlo] = plo * ilo;
-            if (vhi) row[qhi] = phi * ihi;
+        llo += h00 + h01 + h20;
+        lhi += h30 + h31;
+        if constexpr (SAVE) {
+            if (c4 == 0) {                        // residual p of rung k
+                float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
+                if (vlo) row[qlo] = plo;
+                if (vhi) row[qhi] = phi;
+            }
         }
         const unsigned ahi[4] = {pack_bf16(h00, h01), 0u, pack_bf16(h20, 0.f), pack_bf16(h30, h31)};
         const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
@@ -412,10 +395,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         }
     }
 
-    if constexpr (!SAVE) {
-        llo = quad_sum(llo);
-        lhi = quad_sum(lhi);
-    }
+    llo = quad_sum(llo);
+    lhi = quad_sum(lhi);
 
     // ---- normalise and store rows 0..14 of the tile
     const bool ok = ok_k && ok_v;
@@ -427,14 +408,20 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
         for (int n = 0; n < 8; ++n)
             *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][0] * inv_lo, o[n][1] * inv_lo);
-        if (c4 == 0) a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
+        if (c4 == 0) {
+            a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
+            if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qlo] = 1.f / llo;
+        }
     }
     if (vhi && wrel + g4 + 8 < kMmaTile) {
         __nv_bfloat16* row = O + (size_t)qhi * kHeadDim;
 #pragma unroll
         for (int n = 0; n < 8; ++n)
             *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][2] * inv_hi, o[n][3] * inv_hi);
-        if (c4 == 0) a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
+        if (c4 == 0) {
+            a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
+            if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qhi] = 1.f / lhi;
+        }
     }
     }                                             // query heads of the group
 }

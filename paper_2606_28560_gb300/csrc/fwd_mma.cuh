@@ -81,6 +81,8 @@ cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStrea
 // Tensor-core key-centric backward: dv and dk from the {p, dS} pairs of the
 // tensor-core query pass, staging q~ and dO rows of the layout above.
 int bwd_key_mma_blocks(const Shape& s);
+// Dynamic shared memory of the key pass (the staged rows).
+size_t bwd_key_mma_smem_bytes(const MmaLayout& L, bool saved);
 size_t bwd_key_mma_static_smem();
 cudaError_t launch_bwd_key_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_t st);
 

@@ -16,6 +16,12 @@ constexpr unsigned kWaitLimit = 1u << 26;        // mbarrier polls before giving
 
 __device__ __forceinline__ unsigned smem_u32(const void* p) { return (unsigned)__cvta_generic_to_shared(p); }
 
+// 4-byte asynchronous copy global -> shared; zero-filled when !full.
+__device__ __forceinline__ void cp_async4(const float* dst, const float* src, bool full) {
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;\n"
+                 :: "r"(smem_u32(dst)), "l"(src), "r"(full ? 4 : 0) : "memory");
+}
+
 __device__ __forceinline__ void mbar_init(unsigned long long* bar, unsigned count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;\n" :: "r"(smem_u32(bar)), "r"(count));
 }

@@ -142,8 +142,9 @@ def test_workspace_queries():
 
 
 def test_residual_bytes():
-    """The residual buffer holds rotated q (fp16 [B,H,T,64]), p per slot (fp32
-    [B,H,W+1+K,T]) and rung score differences (fp32 [B,H,K,T]), each array from
+    """The residual buffer holds rotated q (fp16 [B,H,T,64]), the unnormalised
+    weight per slot (fp32 [B,H,W+1+K,T]), rung score differences (fp32
+    [B,H,K,T]) and 1 / (weight sum) per query (fp32 [B,H,T]), each array from
     the next multiple of 256 bytes; fp32 I/O and invalid sizes give 0."""
     import torch
 
@@ -151,16 +152,17 @@ def test_residual_bytes():
         return (x + 255) // 256 * 256
     for (Bn, H, T, W, K) in ((2, 3, 100, 8, 15), (1, 1, 1, 0, 0), (16, 8, 1024, 8, 15), (1, 2, 77, 3, 7)):
         n = Bn * H * T
-        want = up(n * 128) + up(n * (W + 1 + K) * 4) + up(n * K * 4)
+        want = up(n * 128) + up(n * (W + 1 + K) * 4) + up(n * K * 4) + up(n * 4)
         assert B.lib().fibattn_residual_bytes(Bn, H, T, 64, W, K, 1) == want
         assert fa.residual_bytes(Bn, H, T, W, K, torch.bfloat16) == want
         assert B.lib().fibattn_residual_bytes(Bn, H, T, 64, W, K, 0) == 0
         buf = torch.zeros(want, dtype=torch.uint8)
-        qt, P, sd = fa.residual_views(buf, Bn, H, T, W, K)
+        qt, P, sd, il = fa.residual_views(buf, Bn, H, T, W, K)
         assert qt.shape == (Bn, H, T, 64) and P.shape == (Bn, H, W + 1 + K, T) and sd.shape == (Bn, H, K, T)
+        assert il.shape == (Bn, H, T)
         # the (non-empty) views tile the buffer in order without overlap
         ends = [(t.data_ptr() - buf.data_ptr(), t.data_ptr() - buf.data_ptr() + t.numel() * t.element_size())
-                for t in (qt, P, sd) if t.numel()]
+                for t in (qt, P, sd, il) if t.numel()]
         assert ends[0][0] == 0 and ends[-1][1] <= want
         assert all(a[1] <= b[0] for a, b in zip(ends, ends[1:]))
         assert all(a % 256 == 0 for a, _ in ends)

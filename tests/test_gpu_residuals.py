@@ -7,8 +7,9 @@ Bars:
   without them (the same arithmetic; the residuals are extra stores).
 - rotated q (fp16): |q~ - ref| <= 2^-11 |ref| + 1e-5 -- fp16 round-to-nearest
   of a value whose fp32 rotation is accurate to ~1e-6 relative.
-- p per slot: |p - ref| <= 1e-2, the bf16 output bar (p is in [0, 1]; the
-  scores come from fp16 operands).
+- p per slot, the stored weight times the stored 1 / (weight sum):
+  |p - ref| <= 1e-2, the bf16 output bar (p is in [0, 1]; the scores come
+  from fp16 operands); the row's weights sum to 1 / that within 1e-5.
 - sd: |sd - ref| <= 2^-10 sum_e |q~_e| (|k~far_e| + |k~floor_e|) + 1e-4 --
   each fp16 factor carries at most 2^-11 relative rounding, accumulation fp32.
 - gradients: the bf16 bars of the tensor-core backward against the oracle.
@@ -51,7 +52,7 @@ def test_residuals_of_the_forward(case):
             pytest.skip(str(e))
         raise
     assert torch.equal(out_r, out) and torch.equal(lse_r, lse)
-    qt, P, sd = (x.cpu() for x in fa.residual_views(res, Bn, H, T, W, K))
+    qt, P, sd, il = (x.cpu() for x in fa.residual_views(res, Bn, H, T, W, K))
     qf, kf = _f64(q), _f64(k)
     G = H // Hkv
     a32 = float(np.float32(alpha))
@@ -82,8 +83,11 @@ def test_residuals_of_the_forward(case):
                 want = np.zeros(W + 1 + K, dtype=bool)
                 want[:W + 1] = True
                 want[W + 1:] = p["active"] & (p["d"] <= T - 1)     # rungs within reach of the sequence
-                gp = P[b, h, :, i].to(torch.float64).numpy()
+                gp = P[b, h, :, i].to(torch.float64).numpy() * float(il[b, h, i])
                 assert np.all(np.abs(gp[want] - ref[want]) <= 1e-2), (b, h, i, gp[want], ref[want])
+                # the weights of the attended slots sum to 1 / il (every attended slot is
+                # stored, the others hold 0)
+                assert abs(float(gp[want].sum()) - 1.0) <= 1e-2
 
 
 def _check_bwd_residuals(q, k, v, dout, alpha, f, W, dedup=True, rung_grads=True):
