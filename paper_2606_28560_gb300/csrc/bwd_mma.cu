@@ -344,70 +344,145 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     };
 
     // ---- rung dp (interpolated) and ddp = dp_far - dp_floor, to shared memory
+    if constexpr (SV) {
+        // Two rungs per iteration (their MMA and reduction chains are
+        // independent); with an odd count the last pair repeats its first rung,
+        // whose second copy reads and writes the same values.
 #pragma unroll 1
-    for (int i = 0; i < n_use; ++i) {
-        release_above(L.act_iv[i]);
-        const float w = L.act_w[i], w1 = 1.f - w;
-        need_rows(L.act_smem[i] + wrel);
-        float dt[2][4];
+        for (int i = 0; i < n_use; i += 2) {
+            const int ib[2] = {i, i + 1 < n_use ? i + 1 : i};
+            release_above(L.act_iv[i]);
+            need_rows(L.act_smem[ib[0]] + wrel);
+            need_rows(L.act_smem[ib[1]] + wrel);
+            float dt[2][2][4];
 #pragma unroll
-        for (int t = 0; t < 2; ++t) {
-            dt[t][0] = dt[t][1] = dt[t][2] = dt[t][3] = 0.f;
-            const int krow = L.act_smem[i] + wrel + 8 * t + (lane & 7);
+            for (int u = 0; u < 2; ++u)
 #pragma unroll
-            for (int kc = 0; kc < 4; kc += 2) {
-                unsigned b0, b1, b2, b3;
-                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
-                mma_bf16_16816(dt[t], da[kc], b0, b1);
-                mma_bf16_16816(dt[t], da[kc + 1], b2, b3);
-            }
-        }
-        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-        // this lane's shares of dp and ddp for rows g4 and g4+8
-        const float x0 = fmaf(c0, dt[0][0], fmaf(c1, dt[0][1], c7 * dt[1][0]));
-        const float x2 = fmaf(c0, dt[1][2], c1 * dt[1][3]);
-        float x1 = 0.f, x3 = 0.f;
-        if constexpr (DD) {
-            x1 = fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0]));
-            x3 = fmaf(df0, dt[1][2], df1 * dt[1][3]);
-        }
-        if constexpr (SV) {
-            // reduce-scatter over the quad: lanes c4 = 0, 1 end with dp, ddp of
-            // row g4, lanes 2, 3 with those of row g4+8; lanes 0 and 2 then form
-            // their row's dS (from the residual p) and dL/dd_k term, the terms
-            // summed over the warp's rows in a fixed order; dS replaces p in
-            // shared memory for the key phase
+                for (int t = 0; t < 2; ++t) {
+                    dt[u][t][0] = dt[u][t][1] = dt[u][t][2] = dt[u][t][3] = 0.f;
+                    const int krow = L.act_smem[ib[u]] + wrel + 8 * t + (lane & 7);
+#pragma unroll
+                    for (int kc = 0; kc < 4; kc += 2) {
+                        unsigned b0, b1, b2, b3;
+                        ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                        mma_bf16_16816(dt[u][t], da[kc], b0, b1);
+                        mma_bf16_16816(dt[u][t], da[kc + 1], b2, b3);
+                    }
+                }
+            // per rung: this lane's shares of dp and ddp for rows g4 and g4+8,
+            // reduce-scattered over the quad (lanes c4 = 0, 1 end with row g4,
+            // lanes 2, 3 with row g4+8); lanes 0 and 2 then form their row's dS
+            // (from the residual p) and dL/dd_k term, the terms summed over the
+            // warp's rows in a fixed order; dS replaces p in shared memory for
+            // the key phase
             const bool up = c4 >= 2;
-            float dp = up ? x2 : x0, ddp = up ? x3 : x1;
-            dp += __shfl_xor_sync(0xffffffffu, up ? x0 : x2, 2);
-            if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, up ? x1 : x3, 2);
-            dp += __shfl_xor_sync(0xffffffffu, dp, 1);
-            if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
             const int row = wrel + g4 + (up ? 8 : 0);
             const bool rv = up ? vhi : vlo;
-            const float p = rv ? psd[0][i][row] * (up ? il_hi : il_lo) : 0.f;
-            const float e = dp - (up ? dlt_hi : dlt_lo);
-            const float ds = p * e;
-            if constexpr (DD) {
-                const float sd = rv ? psd[1][i][row] : 0.f;
-                float g = (c4 & 1) == 0 ? p * fmaf(s.scale * sd, e, ddp) : 0.f;
-                g += __shfl_xor_sync(0xffffffffu, g, 2);
-                g += __shfl_xor_sync(0xffffffffu, g, 4);
-                g += __shfl_xor_sync(0xffffffffu, g, 8);
-                g += __shfl_xor_sync(0xffffffffu, g, 16);
-                if (lane == 0) gsm[warp][L.act_k[i]] = g;
+            float ds[2];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const float w = L.act_w[ib[u]], w1 = 1.f - w;
+                const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+                const float x0 = fmaf(c0, dt[u][0][0], fmaf(c1, dt[u][0][1], c7 * dt[u][1][0]));
+                const float x2 = fmaf(c0, dt[u][1][2], c1 * dt[u][1][3]);
+                float x1 = 0.f, x3 = 0.f;
+                if constexpr (DD) {
+                    x1 = fmaf(df0, dt[u][0][0], fmaf(df1, dt[u][0][1], -m7 * dt[u][1][0]));
+                    x3 = fmaf(df0, dt[u][1][2], df1 * dt[u][1][3]);
+                }
+                float dp = up ? x2 : x0, ddp = up ? x3 : x1;
+                dp += __shfl_xor_sync(0xffffffffu, up ? x0 : x2, 2);
+                if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, up ? x1 : x3, 2);
+                dp += __shfl_xor_sync(0xffffffffu, dp, 1);
+                if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
+                const float p = rv ? psd[0][ib[u]][row] * (up ? il_hi : il_lo) : 0.f;
+                const float e = dp - (up ? dlt_hi : dlt_lo);
+                ds[u] = p * e;
+                if constexpr (DD) {
+                    const float sd = rv ? psd[1][ib[u]][row] : 0.f;
+                    float g = (c4 & 1) == 0 ? p * fmaf(s.scale * sd, e, ddp) : 0.f;
+                    g += __shfl_xor_sync(0xffffffffu, g, 2);
+                    g += __shfl_xor_sync(0xffffffffu, g, 4);
+                    g += __shfl_xor_sync(0xffffffffu, g, 8);
+                    g += __shfl_xor_sync(0xffffffffu, g, 16);
+                    if (lane == 0) gsm[warp][L.act_k[ib[u]]] = g;
+                }
             }
             __syncwarp();                         // the quad has read p before it is replaced
             if ((c4 & 1) == 0 && rv) {
-                psd[0][i][row] = ds;
-                DSg[(size_t)(s.W + 1 + L.act_k[i]) * s.T + bw + g4 + (up ? 8 : 0)] = ds;
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    psd[0][ib[u]][row] = ds[u];
+                    DSg[(size_t)(s.W + 1 + L.act_k[ib[u]]) * s.T + bw + g4 + (up ? 8 : 0)] = ds[u];
+                }
             }
-        } else {
-            const float dp_lo = quad_sum(x0), dp_hi = quad_sum(x2);
-            const float ddp_lo = DD ? quad_sum(x1) : 0.f, ddp_hi = DD ? quad_sum(x3) : 0.f;
-            if (c4 == 0) {
-                *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
-                *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
+        }
+    } else {
+    #pragma unroll 1
+        for (int i = 0; i < n_use; ++i) {
+            release_above(L.act_iv[i]);
+            const float w = L.act_w[i], w1 = 1.f - w;
+            need_rows(L.act_smem[i] + wrel);
+            float dt[2][4];
+    #pragma unroll
+            for (int t = 0; t < 2; ++t) {
+                dt[t][0] = dt[t][1] = dt[t][2] = dt[t][3] = 0.f;
+                const int krow = L.act_smem[i] + wrel + 8 * t + (lane & 7);
+    #pragma unroll
+                for (int kc = 0; kc < 4; kc += 2) {
+                    unsigned b0, b1, b2, b3;
+                    ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
+                    mma_bf16_16816(dt[t], da[kc], b0, b1);
+                    mma_bf16_16816(dt[t], da[kc + 1], b2, b3);
+                }
+            }
+            const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+            // this lane's shares of dp and ddp for rows g4 and g4+8
+            const float x0 = fmaf(c0, dt[0][0], fmaf(c1, dt[0][1], c7 * dt[1][0]));
+            const float x2 = fmaf(c0, dt[1][2], c1 * dt[1][3]);
+            float x1 = 0.f, x3 = 0.f;
+            if constexpr (DD) {
+                x1 = fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0]));
+                x3 = fmaf(df0, dt[1][2], df1 * dt[1][3]);
+            }
+            if constexpr (SV) {
+                // reduce-scatter over the quad: lanes c4 = 0, 1 end with dp, ddp of
+                // row g4, lanes 2, 3 with those of row g4+8; lanes 0 and 2 then form
+                // their row's dS (from the residual p) and dL/dd_k term, the terms
+                // summed over the warp's rows in a fixed order; dS replaces p in
+                // shared memory for the key phase
+                const bool up = c4 >= 2;
+                float dp = up ? x2 : x0, ddp = up ? x3 : x1;
+                dp += __shfl_xor_sync(0xffffffffu, up ? x0 : x2, 2);
+                if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, up ? x1 : x3, 2);
+                dp += __shfl_xor_sync(0xffffffffu, dp, 1);
+                if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
+                const int row = wrel + g4 + (up ? 8 : 0);
+                const bool rv = up ? vhi : vlo;
+                const float p = rv ? psd[0][i][row] * (up ? il_hi : il_lo) : 0.f;
+                const float e = dp - (up ? dlt_hi : dlt_lo);
+                const float ds = p * e;
+                if constexpr (DD) {
+                    const float sd = rv ? psd[1][i][row] : 0.f;
+                    float g = (c4 & 1) == 0 ? p * fmaf(s.scale * sd, e, ddp) : 0.f;
+                    g += __shfl_xor_sync(0xffffffffu, g, 2);
+                    g += __shfl_xor_sync(0xffffffffu, g, 4);
+                    g += __shfl_xor_sync(0xffffffffu, g, 8);
+                    g += __shfl_xor_sync(0xffffffffu, g, 16);
+                    if (lane == 0) gsm[warp][L.act_k[i]] = g;
+                }
+                __syncwarp();                         // the quad has read p before it is replaced
+                if ((c4 & 1) == 0 && rv) {
+                    psd[0][i][row] = ds;
+                    DSg[(size_t)(s.W + 1 + L.act_k[i]) * s.T + bw + g4 + (up ? 8 : 0)] = ds;
+                }
+            } else {
+                const float dp_lo = quad_sum(x0), dp_hi = quad_sum(x2);
+                const float ddp_lo = DD ? quad_sum(x1) : 0.f, ddp_hi = DD ? quad_sum(x3) : 0.f;
+                if (c4 == 0) {
+                    *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
+                    *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
+                }
             }
         }
     }
