@@ -1,6 +1,7 @@
-"""GPU parity of the forward residuals (rotated queries, p of every slot,
-far-minus-floor rung scores) and of the backward that reads them instead of
-recomputing the scores.
+"""GPU parity of the forward residuals (rotated queries, the unnormalised
+softmax weight of every slot with 1 / (weight sum) per query, far-minus-floor
+rung scores) and of the backward that reads them instead of recomputing the
+scores.
 
 Bars:
 - out, lse of a forward that writes residuals: bit-identical to the forward
@@ -9,7 +10,9 @@ Bars:
   of a value whose fp32 rotation is accurate to ~1e-6 relative.
 - p per slot, the stored weight times the stored 1 / (weight sum):
   |p - ref| <= 1e-2, the bf16 output bar (p is in [0, 1]; the scores come
-  from fp16 operands); the row's weights sum to 1 / that within 1e-5.
+  from fp16 operands); the row's p sum to 1 within 1e-2 (the forward's sum
+  adds the bf16-rounded weights its value product uses, the stored weights
+  are unrounded: a relative difference up to 2^-9).
 - sd: |sd - ref| <= 2^-10 sum_e |q~_e| (|k~far_e| + |k~floor_e|) + 1e-4 --
   each fp16 factor carries at most 2^-11 relative rounding, accumulation fp32.
 - gradients: the bf16 bars of the tensor-core backward against the oracle.
