@@ -584,9 +584,44 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         if (lane == 0) gsm[warp][L.act_k[i]] = 0.f;
     }
     // ---- rungs: scores, p, dS, dL/dd_k (SV: dS from the value phase);
-    // dq~ += dShat_k K~_slab
+    // dq~ += dShat_k K~_slab.  SV: two rungs per iteration (the second's dS
+    // loads and fragments overlap the first's products); the odd last rung
+    // goes through the loop below.
+    int i_first = 0;
+    if constexpr (SV) {
 #pragma unroll 1
-    for (int i = 0; i < n_use; ++i) {
+        for (; i_first + 1 < n_use; i_first += 2) {
+            need_keys(L.act_iv[i_first]);
+            need_keys(L.act_iv[i_first + 1]);
+            unsigned afr2[2][4];
+#pragma unroll
+            for (int u = 0; u < 2; ++u) {
+                const int ii = i_first + u;
+                const float w = L.act_w[ii], w1 = 1.f - w;
+                const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
+                const float dsl = vlo ? psd[0][ii][wrel + g4] : 0.f;
+                const float dsh = vhi ? psd[0][ii][wrel + g4 + 8] : 0.f;
+                afr2[u][0] = pack_f16(c0 * dsl, c1 * dsl);
+                afr2[u][1] = 0u;
+                afr2[u][2] = pack_f16(c7 * dsl, 0.f);
+                afr2[u][3] = pack_f16(c0 * dsh, c1 * dsh);
+            }
+            const int krow0 = L.act_smem[i_first] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+            const int krow1 = L.act_smem[i_first + 1] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+#pragma unroll
+            for (int n = 0; n < 8; n += 2) {
+                unsigned b0, b1, b2, b3, e0, e1, e2, e3;
+                ldsm_x4_t(row_chunk(sbase, krow0, n + (lane >> 4)), b0, b1, b2, b3);
+                ldsm_x4_t(row_chunk(sbase, krow1, n + (lane >> 4)), e0, e1, e2, e3);
+                mma_f16_16816(dq[n], afr2[0], b0, b1);
+                mma_f16_16816(dq[n + 1], afr2[0], b2, b3);
+                mma_f16_16816(dq[n], afr2[1], e0, e1);
+                mma_f16_16816(dq[n + 1], afr2[1], e2, e3);
+            }
+        }
+    }
+#pragma unroll 1
+    for (int i = i_first; i < n_use; ++i) {
         need_keys(L.act_iv[i]);
         const float w = L.act_w[i], w1 = 1.f - w;
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
