@@ -375,7 +375,8 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     const size_t smem_limit = 227 * 1024;
     MmaLayout ML;
     StageLayout L;
-    const bool mma_ok = bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 3) && build_mma_layout(a.s, a.r, o.rope_base, smem_limit, &ML);
+    const bool mma_ok = bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 3) &&
+                        build_mma_layout(a.s, a.r, o.rope_base, smem_limit - fwd_mma_static_smem(), &ML);
     const bool staged_ok = !mma_ok && bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 2) &&
                            build_stage_layout(a.s, a.r, o.rope_base, smem_limit, &L);
     if ((o.fwd_kernel == 3 && !mma_ok) || (o.fwd_kernel == 2 && !staged_ok))

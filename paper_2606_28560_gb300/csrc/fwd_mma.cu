@@ -466,7 +466,10 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.buf_rows * 128 + 1024; }
 
-size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - 64; }
+// the two barriers of a CTA, rounded up
+size_t fwd_mma_static_smem() { return 64; }
+
+size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - fwd_mma_static_smem(); }
 
 namespace {
 

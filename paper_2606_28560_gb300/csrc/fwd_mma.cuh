@@ -54,6 +54,8 @@ bool build_mma_layout(const Shape& s, const RungParams& r, double rope_base, siz
 // the first key of a tile (win_smem: relative row 0; rung_smem[k]: row s0_k).
 bool build_key_layout(const Shape& s, const RungParams& r, double rope_base, size_t smem_limit, MmaLayout* L);
 size_t fwd_mma_smem_bytes(const MmaLayout& L);
+// Static shared memory of a forward CTA of one team (8 warps).
+size_t fwd_mma_static_smem();
 // Dynamic shared memory a grouped-query forward CTA may use (keys and values
 // both resident).
 size_t fwd_mma_gqa_smem_limit();
