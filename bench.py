@@ -249,9 +249,9 @@ def algorithmic_bytes(residuals=True):
 # file of the kernel changes, the figure is reported as null until the next
 # capture.
 NCU_TRAFFIC = {
-    "bwd_query_mma": {"bytes_at_b32": 164776960 + 35540224,
+    "bwd_query_mma": {"bytes_at_b32": 165859328 + 35686912,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "91c0baf805f1f7ad76e1b8a97b6bc3f03c79dce39fc014cfd8fb2a383b40c75b"},
+                      "sha256": "4fd42fdcbaa8cf9348964e096d6ebe658f007bc18f3f5ca757c0f9b474d30aab"},
 }
 
 
