@@ -546,7 +546,11 @@ def run_e2e(args, wl, device, dist):
     memory, inside the timed region.  The copies run on two copy streams and
     overlap the compute: a layer's forward waits only for its own q, k, v,
     its backward for its own dout, and each result goes back as soon as the
-    layer that produced it is done."""
+    layer that produced it is done.  The device inputs are double-buffered by
+    step, as a prefetching loader would: step s + 1's inputs stream in while
+    step s's gradients stream out, so both directions of the link stay busy.
+    Every buffer is reused only after the work that last read or wrote it
+    (per-layer events)."""
     fa = wl.fa
     n_in = 4 * L
     host_in = [torch.empty((B, H, T, D), dtype=torch.bfloat16, pin_memory=True) for _ in range(n_in)]
@@ -555,58 +559,78 @@ def run_e2e(args, wl, device, dist):
         h.copy_(src)
     host_out = [torch.empty((B, H, T, D), dtype=torch.bfloat16, pin_memory=True) for _ in range(4 * L)]
     host_th = torch.empty((L, 4), dtype=torch.float32, pin_memory=True)
+    # input sets by step parity: the workload's own buffers and a second copy
+    sets = [(wl.q, wl.k, wl.v, wl.g),
+            tuple([torch.empty_like(x) for x in t] for t in (wl.q, wl.k, wl.v, wl.g))]
     # compute on a stream of its own: work on the legacy default stream would
     # serialise with the copy streams
     comp, s_in, s_out = torch.cuda.Stream(device), torch.cuda.Stream(device), torch.cuda.Stream(device)
-    ev_in = [torch.cuda.Event() for _ in range(L)]          # q, k, v of layer l on the device
-    ev_g = [torch.cuda.Event() for _ in range(L)]           # dout of layer l on the device
-    ev_f = [torch.cuda.Event() for _ in range(L)]           # forward of layer l done
-    ev_b = [torch.cuda.Event() for _ in range(L)]           # backward of layer l done
+    ev_in = [[torch.cuda.Event() for _ in range(L)] for _ in range(2)]    # q, k, v of layer l on the device
+    ev_g = [[torch.cuda.Event() for _ in range(L)] for _ in range(2)]     # dout of layer l on the device
+    ev_b = [[torch.cuda.Event() for _ in range(L)] for _ in range(2)]     # backward of layer l done (set free)
+    ev_f = [torch.cuda.Event() for _ in range(L)]            # forward of layer l done
+    ev_bo = [torch.cuda.Event() for _ in range(L)]           # backward of layer l done (outputs ready)
+    ev_oc = [torch.cuda.Event() for _ in range(L)]           # out of layer l read back
+    ev_gc = [torch.cuda.Event() for _ in range(L)]           # dq, dk, dv of layer l read back
+    ev_th = torch.cuda.Event()                               # dtheta read back
     steps = max(2, min(args.steps, 10))
+    state = {"step": 0}
 
     def one():
-        # the previous step's kernels and result copies are done with the buffers
-        s_in.wait_stream(comp)
-        comp.wait_stream(s_out)
+        p = state["step"] % 2
+        state["step"] += 1
+        q, k, v, g = sets[p]
         with torch.cuda.stream(s_in):
             for l in range(L):
-                for j, dst in enumerate((wl.q, wl.k, wl.v)):
+                s_in.wait_event(ev_b[p][l])      # the step before last is done with this set
+                for j, dst in enumerate((q, k, v)):
                     dst[l].copy_(host_in[4 * l + j], non_blocking=True)
-                ev_in[l].record(s_in)
+                ev_in[p][l].record(s_in)
             for l in reversed(range(L)):
-                wl.g[l].copy_(host_in[4 * l + 3], non_blocking=True)
-                ev_g[l].record(s_in)
+                g[l].copy_(host_in[4 * l + 3], non_blocking=True)
+                ev_g[p][l].record(s_in)
         for l in range(L):
-            comp.wait_event(ev_in[l])
-            fa.fwd(wl.q[l], wl.k[l], wl.v[l], wl.alphas[l], wl.f, W, out=wl.out[l], lse=wl.lse[l],
+            comp.wait_event(ev_in[p][l])
+            comp.wait_event(ev_oc[l])            # the previous step's out of this layer is on the host
+            fa.fwd(q[l], k[l], v[l], wl.alphas[l], wl.f, W, out=wl.out[l], lse=wl.lse[l],
                    workspace=wl.ws_f, rotated_k=wl.rk[l], residuals=wl.res[l], stream=comp)
             ev_f[l].record(comp)
             s_out.wait_event(ev_f[l])
             with torch.cuda.stream(s_out):
                 host_out[4 * l].copy_(wl.out[l], non_blocking=True)
+                ev_oc[l].record(s_out)
+        comp.wait_event(ev_th)                   # the previous step's dtheta is on the host
         for l in reversed(range(L)):
-            comp.wait_event(ev_g[l])
-            fa.bwd(wl.q[l], wl.k[l], wl.v[l], wl.lse[l], wl.g[l], wl.alphas[l], wl.f, W, out=wl.out[l],
+            comp.wait_event(ev_g[p][l])
+            comp.wait_event(ev_gc[l])            # the previous step's gradients of this layer are on the host
+            fa.bwd(q[l], k[l], v[l], wl.lse[l], g[l], wl.alphas[l], wl.f, W, out=wl.out[l],
                    dq=wl.dq[l], dk=wl.dk[l], dv=wl.dv[l], dtheta=wl.dth[l], dd=wl.dd[l], workspace=wl.ws_b,
                    rotated_k=wl.rk[l], residuals=wl.res[l], stream=comp)
-            ev_b[l].record(comp)
-            s_out.wait_event(ev_b[l])
+            ev_b[p][l].record(comp)
+            ev_bo[l].record(comp)
+            s_out.wait_event(ev_bo[l])
             with torch.cuda.stream(s_out):
                 for j, src in enumerate((wl.dq, wl.dk, wl.dv)):
                     host_out[4 * l + 1 + j].copy_(src[l], non_blocking=True)
+                ev_gc[l].record(s_out)
         with torch.cuda.stream(s_out):
             host_th.copy_(wl.dth, non_blocking=True)
-        comp.wait_stream(s_out)                  # the step ends when its results are on the host
+            ev_th.record(s_out)
 
     with torch.cuda.stream(comp):
+        one()
         one()
         torch.cuda.synchronize(device)
         if dist:
             torch.distributed.barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(comp)
+        s_in.wait_stream(comp)                   # the first timed copies start after e0
+        s_out.wait_stream(comp)
         for _ in range(steps):
             one()
+        comp.wait_stream(s_out)                  # the last step ends when its results are on the host
+        comp.wait_stream(s_in)
         e1.record(comp)
         torch.cuda.synchronize(device)
     ms = max_over_ranks(e0.elapsed_time(e1), device)
@@ -614,9 +638,11 @@ def run_e2e(args, wl, device, dist):
     value = job_throughput(world, steps, ms)
     bi = n_in * B * H * T * ROW_BYTES
     bo = 4 * L * B * H * T * ROW_BYTES + L * 4 * 4
+    ok = all(torch.equal(host_out[4 * l + 1].to(device), wl.dq[l]) for l in (0, L - 1))
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,
-            "ms_per_step": round(ms / steps, 4),
-            "copies": "two copy streams overlapping the compute; per-layer events"}
+            "ms_per_step": round(ms / steps, 4), "results_on_host_match": ok,
+            "copies": "two copy streams overlapping the compute; device inputs double-buffered by step "
+                      "(the next step's inputs stream in while this step's gradients stream out); per-layer events"}
 
 
 # ------------------------------------------------------------- CPU oracle --
