@@ -251,7 +251,7 @@ def algorithmic_bytes(residuals=True):
 NCU_TRAFFIC = {
     "bwd_query_mma": {"bytes_at_b32": 165859328 + 35686912,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "4fd42fdcbaa8cf9348964e096d6ebe658f007bc18f3f5ca757c0f9b474d30aab"},
+                      "sha256": "c6aaa7b76693a7c57d07d9a1f5b35a29b60580b7b86101a0f829cf0d6ddda1af"},
 }
 
 

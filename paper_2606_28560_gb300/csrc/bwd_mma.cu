@@ -445,44 +445,11 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 x1 = fmaf(df0, dt[0][0], fmaf(df1, dt[0][1], -m7 * dt[1][0]));
                 x3 = fmaf(df0, dt[1][2], df1 * dt[1][3]);
             }
-            if constexpr (SV) {
-                // reduce-scatter over the quad: lanes c4 = 0, 1 end with dp, ddp of
-                // row g4, lanes 2, 3 with those of row g4+8; lanes 0 and 2 then form
-                // their row's dS (from the residual p) and dL/dd_k term, the terms
-                // summed over the warp's rows in a fixed order; dS replaces p in
-                // shared memory for the key phase
-                const bool up = c4 >= 2;
-                float dp = up ? x2 : x0, ddp = up ? x3 : x1;
-                dp += __shfl_xor_sync(0xffffffffu, up ? x0 : x2, 2);
-                if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, up ? x1 : x3, 2);
-                dp += __shfl_xor_sync(0xffffffffu, dp, 1);
-                if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
-                const int row = wrel + g4 + (up ? 8 : 0);
-                const bool rv = up ? vhi : vlo;
-                const float p = rv ? psd[0][i][row] * (up ? il_hi : il_lo) : 0.f;
-                const float e = dp - (up ? dlt_hi : dlt_lo);
-                const float ds = p * e;
-                if constexpr (DD) {
-                    const float sd = rv ? psd[1][i][row] : 0.f;
-                    float g = (c4 & 1) == 0 ? p * fmaf(s.scale * sd, e, ddp) : 0.f;
-                    g += __shfl_xor_sync(0xffffffffu, g, 2);
-                    g += __shfl_xor_sync(0xffffffffu, g, 4);
-                    g += __shfl_xor_sync(0xffffffffu, g, 8);
-                    g += __shfl_xor_sync(0xffffffffu, g, 16);
-                    if (lane == 0) gsm[warp][L.act_k[i]] = g;
-                }
-                __syncwarp();                         // the quad has read p before it is replaced
-                if ((c4 & 1) == 0 && rv) {
-                    psd[0][i][row] = ds;
-                    DSg[(size_t)(s.W + 1 + L.act_k[i]) * s.T + bw + g4 + (up ? 8 : 0)] = ds;
-                }
-            } else {
-                const float dp_lo = quad_sum(x0), dp_hi = quad_sum(x2);
-                const float ddp_lo = DD ? quad_sum(x1) : 0.f, ddp_hi = DD ? quad_sum(x3) : 0.f;
-                if (c4 == 0) {
-                    *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
-                    *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
-                }
+            const float dp_lo = quad_sum(x0), dp_hi = quad_sum(x2);
+            const float ddp_lo = DD ? quad_sum(x1) : 0.f, ddp_hi = DD ? quad_sum(x3) : 0.f;
+            if (c4 == 0) {
+                *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
+                *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
             }
         }
     }
