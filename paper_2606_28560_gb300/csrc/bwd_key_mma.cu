@@ -189,17 +189,26 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
     }
 }
 
-template <int NT>
+// SPLIT: blocks [0, units) take pass 0 (dv) and blocks [units, 2 units) pass
+// 1 (dk~) of the same key tiles, for grids too small to fill the GPU with one
+// block per tile (grouped-query heads, small batches); else a block runs both
+// passes of its tile.
+template <int NT, bool SPLIT>
 __global__ void __launch_bounds__(kWarps * 32, 2)
 bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ RowMaps tmG, BwdArgs a,
                    MmaLayout L) {
     // The kernel before this one is the query pass of the same call.  With the
-    // forward residuals the first pass reads only p and dO, which it does not
-    // write, so the wait for it comes before the second pass (dS) and before
-    // block 0 sums the query pass's rung partials.
+    // forward residuals pass 0 reads only p and dO, which it does not write,
+    // so the wait for it comes before pass 1 (dS), whose first block then sums
+    // the query pass's rung partials.
     pdl_trigger();
-    const bool early = a.saved != 0;
-    if (!early) pdl_wait();
+    const int tiles = (a.s.T + kMmaTile - 1) / kMmaTile;
+    const int units = tiles * a.s.B * a.s.Hkv;
+    const int pass_first = SPLIT && (int)blockIdx.x >= units ? 1 : 0;
+    const int pass_end = SPLIT ? pass_first + 1 : 2;
+    const int blk = (int)blockIdx.x - pass_first * units;
+    bool waited = a.saved == 0;
+    if (waited) pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bar;
     __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
@@ -210,9 +219,8 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     const unsigned sbase = smem_u32(buf);
 
     const Shape s = a.s;
-    const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
-    const int bhk = blockIdx.x / tiles;                   // b * Hkv + hk
-    const int j0 = (blockIdx.x % tiles) * kMmaTile;
+    const int bhk = blk / tiles;                          // b * Hkv + hk
+    const int j0 = (blk % tiles) * kMmaTile;
     const int b = bhk / s.Hkv, hk = bhk % s.Hkv;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int g4 = lane >> 2, c4 = lane & 3;
@@ -227,16 +235,16 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
     __syncthreads();
-    if (!early && blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
 
     unsigned parity = 0;
     bool ok = true;
     const size_t krow0 = (size_t)bhk * s.T;
 #pragma unroll 1
-    for (int pass = 0; pass < 2; ++pass) {                // 0: dv from dO rows; 1: dk~ from q~ rows
-        if (pass == 1 && early) {
-            pdl_wait();
-            if (blockIdx.x == 0 && a.want_dd) convert_rung_sums(a, red, red64);
+    for (int pass = pass_first; pass < pass_end; ++pass) {  // 0: dv from dO rows; 1: dk~ from q~ rows
+        if (pass == 1) {
+            if (!waited) pdl_wait();
+            waited = true;
+            if (blk == 0 && a.want_dd) convert_rung_sums(a, red, red64);
         }
         float acc[8][4];
 #pragma unroll
@@ -251,7 +259,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
             }
             if (pass == 0)
                 key_pass<NT, false>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
-                                       rvals[warp], early ? a.res_il + (size_t)qhead * s.T : nullptr, wils[warp]);
+                                       rvals[warp], a.saved ? a.res_il + (size_t)qhead * s.T : nullptr, wils[warp]);
             else
                 key_pass<NT, true>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
                                       rvals[warp]);
@@ -314,7 +322,17 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
 template <int NT>
 cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, const MmaLayout& L,
                       unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = bwd_key_mma_kernel<NT>;
+    // one block per tile unless that leaves the GPU under two waves of blocks
+    static int slots = 0;
+    if (slots == 0) {
+        int dev = 0, sms = 0;
+        slots = cudaGetDevice(&dev) == cudaSuccess &&
+                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && sms > 0
+                    ? 2 * sms : 2 * 152;
+    }
+    const bool split = (long long)grid < 2LL * slots;
+    auto kern = split ? bwd_key_mma_kernel<NT, true> : bwd_key_mma_kernel<NT, false>;
+    if (split) grid *= 2;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_kernel(kern, dim3(grid), dim3(kWarps * 32), smem, st, mq, mg, a, L);
