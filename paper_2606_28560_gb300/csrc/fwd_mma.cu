@@ -431,7 +431,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 template <int NT, int TEAMS>
 cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const FwdArgs& a, const MmaLayout& L,
                       unsigned grid, size_t smem, cudaStream_t st) {
-    auto kern = a.res_P ? fwd_mma_kernel<NT, TEAMS, true> : fwd_mma_kernel<NT, TEAMS, false>;
+    // (the grouped form runs only without residuals)
+    auto kern = a.res_P ? fwd_mma_kernel<NT, TEAMS, TEAMS == 1> : fwd_mma_kernel<NT, TEAMS, false>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_kernel(kern, dim3(grid), dim3(kWarps * 32 * TEAMS), smem, st, mk, mv, a, L);
@@ -630,9 +631,11 @@ cudaError_t launch_fwd_mma(const FwdArgs& a, const MmaLayout& L, cudaStream_t st
         !encode_row_maps(&mv, a.v, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
         return cudaErrorInvalidValue;
     // Grouped-query attention: one CTA per kv head's tile with both staged
-    // tensors resident, when they fit.
+    // tensors resident, when they fit and no residuals are written (with the
+    // residual stores, one CTA per query head's tile with two CTAs per SM
+    // measured faster; L2 then serves the group's repeated row reads).
     const size_t smem2 = 2 * (size_t)L.rows * 128 + 1024;
-    if (a.s.G >= 2 && smem2 <= fwd_mma_gqa_smem_limit()) {
+    if (a.s.G >= 2 && smem2 <= fwd_mma_gqa_smem_limit() && !a.res_P) {
         const unsigned grid = (unsigned)(tiles * heads);
         switch (L.nt) {
         case 2: return launch_nt<2, 2>(mk, mv, a, L, grid, smem2, st);
