@@ -9,7 +9,9 @@ k again, and with bf16 I/O also its residuals (the rotated queries, p of every
 attended slot and the rung score differences), so the backward does not
 recompute the scores.  alpha is a host value of the C ABI -- the kernels' shared-memory
 layout depends on the rung distances -- so a theta held on the GPU is read
-once per call.
+once per call (a device-to-host copy that waits for the queued work), unless
+the caller passes alpha: `attention_stack` reads the thetas of all its layers
+in one copy.
 """
 from __future__ import annotations
 
@@ -31,8 +33,9 @@ class FibAttentionFunction(torch.autograd.Function):
     (a 0-dim tensor); offsets, W and the options are constants."""
 
     @staticmethod
-    def forward(ctx, q, k, v, theta, offsets, W, rope_base, scale, dedup):
-        alpha = alpha_of_theta(float(theta))
+    def forward(ctx, q, k, v, theta, offsets, W, rope_base, scale, dedup, alpha=None):
+        if alpha is None:
+            alpha = alpha_of_theta(float(theta))
         rk = B.rotated_k_like(k)
         kw = dict(rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk)
         res = None
@@ -61,19 +64,22 @@ class FibAttentionFunction(torch.autograd.Function):
                                    rope_base=rope_base, scale=scale, dedup=dedup, rotated_k=rk,
                                    residuals=res if res.numel() else None)
         dtheta = dth.reshape(()).to(device=tdev, dtype=tdtype)
-        return dq, dk, dv, dtheta, None, None, None, None, None
+        return dq, dk, dv, dtheta, None, None, None, None, None, None
 
 
 def fib_attention(q, k, v, theta, offsets=None, W: int = 8, *, rope_base: float = 1e4, scale=None,
-                  dedup: bool = True):
+                  dedup: bool = True, alpha=None):
     """Functional form.  q [B,H,T,64]; k, v [B,Hkv,T,64] (bf16 or fp32, CUDA,
     contiguous); theta a 0-dim tensor (requires_grad for the learned
-    schedule); offsets the base sequence (default: Fibonacci, K = 15)."""
+    schedule); offsets the base sequence (default: Fibonacci, K = 15).
+    ``alpha``: the host value 0.5 + sigmoid(theta), when the caller has it
+    (skips reading theta)."""
     if offsets is None:
         offsets = B.base("fib", 15)
     if not torch.is_tensor(theta):
         theta = torch.tensor(float(theta))
-    return FibAttentionFunction.apply(q, k, v, theta, offsets, W, rope_base, scale, dedup)
+    return FibAttentionFunction.apply(q, k, v, theta, offsets, W, rope_base, scale, dedup,
+                                      None if alpha is None else float(alpha))
 
 
 class FibAttention(torch.nn.Module):
@@ -95,9 +101,11 @@ class FibAttention(torch.nn.Module):
     def alpha(self) -> float:
         return alpha_of_theta(float(self.theta))
 
-    def forward(self, q, k, v):
+    def forward(self, q, k, v, alpha=None):
+        """``alpha``: the host value of 0.5 + sigmoid(theta), when the caller
+        has read it (skips the per-call read of a theta on the GPU)."""
         return FibAttentionFunction.apply(q, k, v, self.theta, self.offsets, self.W, self.rope_base, self.scale,
-                                          self.dedup)
+                                          self.dedup, None if alpha is None else float(alpha))
 
 
 def theta_of_alpha(alpha: float) -> float:
@@ -109,7 +117,13 @@ def theta_of_alpha(alpha: float) -> float:
 
 def attention_stack(x: torch.Tensor, layers) -> torch.Tensor:
     """A stack of attention layers without projections: each layer attends
-    with q = k = v = the previous layer's output (the first takes x)."""
-    for layer in layers:
-        x = layer(x, x, x)
+    with q = k = v = the previous layer's output (the first takes x).  The
+    layers' thetas are read to the host in one copy before the first layer."""
+    layers = list(layers)
+    if not layers:
+        return x
+    dev = layers[0].theta.device
+    thetas = torch.stack([layer.theta.detach().to(device=dev, dtype=torch.float64) for layer in layers]).tolist()
+    for layer, th in zip(layers, thetas):
+        x = layer(x, x, x, alpha=alpha_of_theta(th))
     return x

@@ -8,6 +8,7 @@ a call returns a non-OK status -- there is no fallback.
 from __future__ import annotations
 
 import ctypes
+import functools
 import os
 import threading
 
@@ -56,11 +57,11 @@ def lib():
             op = ctypes.POINTER(Opts)
             L.fibattn_fwd_workspace_bytes.argtypes = [ci] * 7 + [op]
             L.fibattn_fwd_workspace_bytes.restype = sz
-            L.fibattn_fwd.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, fp, ci, ci, op, vp, sz, vp]
+            L.fibattn_fwd.argtypes = [vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, vp, ci, ci, op, vp, sz, vp]
             L.fibattn_fwd.restype = ci
             L.fibattn_bwd_workspace_bytes.argtypes = [ci] * 7 + [op]
             L.fibattn_bwd_workspace_bytes.restype = sz
-            L.fibattn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, fp, ci, ci,
+            L.fibattn_bwd.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, ci, ci, ci, ci, ci, cf, vp, ci, ci,
                                       op, vp, sz, vp]
             L.fibattn_bwd.restype = ci
             L.fibattn_last_error.argtypes = []
@@ -102,10 +103,14 @@ def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto", bw
                 residuals.data_ptr() if residuals is not None else None)
 
 
+@functools.lru_cache(maxsize=256)
+def _residual_bytes(B, H, T, W, K, bf16, D) -> int:
+    return int(lib().fibattn_residual_bytes(B, H, T, D, W, K, FIBATTN_BF16 if bf16 else FIBATTN_F32))
+
+
 def residual_bytes(B, H, T, W, K, dtype=torch.bfloat16, D=64) -> int:
     """Size of the forward residuals (``residuals=``); 0 for fp32 I/O."""
-    code = FIBATTN_BF16 if dtype == torch.bfloat16 else FIBATTN_F32
-    return int(lib().fibattn_residual_bytes(B, H, T, D, W, K, code))
+    return _residual_bytes(int(B), int(H), int(T), int(W), int(K), dtype == torch.bfloat16, int(D))
 
 
 def residuals_like(q: torch.Tensor, W: int, K: int) -> torch.Tensor:
@@ -175,6 +180,8 @@ def _stream_ptr(stream) -> int:
 
 
 def _offsets(offsets) -> np.ndarray:
+    if isinstance(offsets, np.ndarray) and offsets.dtype == np.float32 and offsets.flags.c_contiguous:
+        return offsets
     return np.ascontiguousarray(np.asarray(offsets, dtype=np.float32))
 
 
@@ -278,11 +285,11 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
         out = torch.empty_like(q)
     if lse is None:
         lse = torch.empty((B, H, T), dtype=torch.float32, device=q.device)
-    need = int(lib().fibattn_fwd_workspace_bytes(B, H, T, D, W, len(f), code, ctypes.byref(o)))
-    if workspace is None:
+    if workspace is None:                        # (a given workspace's size is checked by the library)
+        need = int(lib().fibattn_fwd_workspace_bytes(B, H, T, D, W, len(f), code, ctypes.byref(o)))
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
     _check(lib().fibattn_fwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr(), lse.data_ptr(),
-                             B, H, T, D, int(W), float(alpha), _fptr(f), len(f), code, ctypes.byref(o),
+                             B, H, T, D, int(W), float(alpha), f.ctypes.data, len(f), code, ctypes.byref(o),
                              workspace.data_ptr(), workspace.numel(), _stream_ptr(stream)))
     return out, lse
 
@@ -315,15 +322,15 @@ def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_bas
     if rung_grads:
         dtheta = torch.empty(4, dtype=torch.float32, device=q.device) if dtheta is None else dtheta
         dd = torch.empty(max(K, 1), dtype=torch.float32, device=q.device) if dd is None else dd
-    need = int(lib().fibattn_bwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
-    if workspace is None:
+    if workspace is None:                        # (a given workspace's size is checked by the library)
+        need = int(lib().fibattn_bwd_workspace_bytes(B, H, T, D, W, K, code, ctypes.byref(o)))
         workspace = torch.empty(max(need, 256), dtype=torch.uint8, device=q.device)
     _check(lib().fibattn_bwd(q.data_ptr(), k.data_ptr(), v.data_ptr(), out.data_ptr() if out is not None else None,
                              lse.data_ptr(), dout.data_ptr(),
                              dq.data_ptr(), dk.data_ptr(), dv.data_ptr(),
                              dtheta.data_ptr() if dtheta is not None else None,
                              dd.data_ptr() if dd is not None else None,
-                             B, H, T, D, int(W), float(alpha), _fptr(f), K, code, ctypes.byref(o),
+                             B, H, T, D, int(W), float(alpha), f.ctypes.data, K, code, ctypes.byref(o),
                              workspace.data_ptr(), workspace.numel(), _stream_ptr(stream)))
     if dtheta is None and dd is None:
         return dq, dk, dv, None, None

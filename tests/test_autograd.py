@@ -112,3 +112,32 @@ def test_sixteen_layer_stack_runs_all_schedules():
         x.grad = None
         if kind == "learned":
             assert all(torch.isfinite(l.theta.grad) for l in layers)
+
+
+@pytest.mark.gpu
+def test_stack_reads_thetas_once_with_identical_results():
+    """attention_stack passes each layer the host alpha it read for all layers
+    in one copy; the result and the gradients equal those of layers that each
+    read their own theta."""
+    torch.manual_seed(2)
+    x = torch.randn(1, 4, 300, 64, device="cuda").to(torch.bfloat16)
+    gout = torch.randn_like(x)
+    f = fa.base("fib", 15)
+    thetas = [0.3, -1.1, 0.9]
+
+    def run(stacked):
+        xi = x.clone().requires_grad_(True)
+        layers = [fa.FibAttention(W=8, offsets=f, theta=t, learned=True).cuda() for t in thetas]
+        if stacked:
+            out = fa.attention_stack(xi, layers)
+        else:
+            out = xi
+            for layer in layers:
+                out = layer(out, out, out)
+        (out.float() * gout.float()).sum().backward()
+        return out.detach(), xi.grad, [l.theta.grad.clone() for l in layers]
+
+    o1, g1, t1 = run(True)
+    o2, g2, t2 = run(False)
+    assert torch.equal(o1, o2) and torch.equal(g1, g2)
+    assert all(torch.equal(a, b) for a, b in zip(t1, t2))
