@@ -215,3 +215,46 @@ def test_calls_from_a_fresh_host_thread():
         for a, b in zip(main[name][:3], got[name][:3]):
             assert torch.equal(a, b)
     assert torch.equal(got["fwd"][0], out)
+
+
+def _random_cases(n=16, seed=2606):
+    """Seeded shapes across the launch paths: grouped-query heads (G = 1, 2, 4),
+    lengths from 1 to 700 (ragged last tiles), W = 0..16, fractional alpha
+    over [0.5, 1.5], both bases, K = 0..15, dedup on and off."""
+    rng = np.random.default_rng(seed)
+    cases = []
+    for _ in range(n):
+        Hkv = int(rng.integers(1, 3))
+        G = int(rng.choice([1, 2, 4]))
+        base = str(rng.choice(["fib", "pow2"]))
+        K = int(rng.integers(0, 16 if base == "fib" else 11))
+        cases.append((int(rng.integers(1, 3)), Hkv * G, Hkv, int(rng.integers(1, 701)), int(rng.integers(0, 17)),
+                      float(np.float32(rng.uniform(0.5, 1.5))), base, K, bool(rng.integers(0, 2))))
+    return cases
+
+
+RANDOM = _random_cases()
+
+
+@pytest.mark.parametrize("case", RANDOM, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]:.4f}{c[6]}{c[7]}d{int(c[8])}"
+                                              for c in RANDOM])
+def test_random_shapes_forward_and_backward_from_residuals(case):
+    """The residual forward's output and the backward from its residuals
+    against the oracle on seeded random shapes."""
+    from tests.test_gpu_parity import bf16_out_tol
+    Bn, H, Hkv, T, W, alpha, base, K, dedup = case
+    q, k, v = inputs.qkv(Bn, H, T, seed=T * 31 + W, dtype=torch.bfloat16, Hkv=Hkv)
+    g = inputs.dout(Bn, H, T, seed=T * 31 + W + 1, dtype=torch.bfloat16)
+    f = fa.base(base, K)
+    try:
+        res = fa.residuals_like(q.cuda(), W, K)
+        out, _ = fa.fwd(q.cuda(), k.cuda(), v.cuda(), alpha, f, W, dedup=dedup, residuals=res)
+    except fa.FibattnError as e:
+        if e.status == 2:
+            pytest.skip(str(e))
+        raise
+    torch.cuda.synchronize()
+    d = O.offsets_fp32(float(np.float32(alpha)), f.astype(np.float64))
+    ro, _ = O.forward(_f64(q), _f64(k), _f64(v), W, d, dedup=dedup, nthreads=NTHREADS)
+    assert not (np.abs(_f64(out) - ro) > bf16_out_tol(ro)).any()
+    _check_bwd_residuals(q, k, v, g, alpha, f, W, dedup)
