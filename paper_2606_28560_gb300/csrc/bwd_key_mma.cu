@@ -12,7 +12,7 @@
 // are products of a banded matrix with staged query rows:
 //   window band  acc += P_band^T  X[b, b+16+Wp)       P_band^T[r][x] = p(b+x, t = x-r)
 //   rung k       acc += Phat_k^T  X[b+s0, b+s0+16)    Phat_k^T[r][r] = (1-w) p, [r][r+1] = w p
-// with X = dO rows (bf16, pass 1: dv) and then X = q~ rows (fp16, pass 2:
+// with X = dO rows (bf16, pass 0: dv) and then X = q~ rows (fp16, pass 1:
 // dk~, dS in place of p).  The CTA stages the union of the query rows its
 // warps read, one tensor (and query head) at a time, in one buffer.
 // A-operand values: p as bf16, dS as fp16; accumulation fp32.
