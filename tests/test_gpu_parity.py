@@ -128,6 +128,22 @@ SMALL = [
 ]
 
 
+def _random_cases(n=16, seed=2606):
+    """Seeded shapes across the launch paths: grouped-query heads (G = 1, 2, 4),
+    lengths from 1 to 700 (ragged last tiles), W = 0..16, fractional alpha
+    over [0.5, 1.5], both bases, K = 0..15, dedup on and off."""
+    rng = np.random.default_rng(seed)
+    cases = []
+    for _ in range(n):
+        Hkv = int(rng.integers(1, 3))
+        G = int(rng.choice([1, 2, 4]))
+        base = str(rng.choice(["fib", "pow2"]))
+        K = int(rng.integers(0, 16 if base == "fib" else 11))
+        cases.append((int(rng.integers(1, 3)), Hkv * G, Hkv, int(rng.integers(1, 701)), int(rng.integers(0, 17)),
+                      float(np.float32(rng.uniform(0.5, 1.5))), base, K, bool(rng.integers(0, 2))))
+    return cases
+
+
 FWD_KERNELS = [(torch.float32, "auto"), (torch.bfloat16, "gather"), (torch.bfloat16, "staged"),
                (torch.bfloat16, "mma")]
 
@@ -297,3 +313,37 @@ def test_config5_bf16_long_stress(base, K):
         g = inputs.dout(2, 8, 16384, seed=s, dtype=torch.bfloat16)
         check_fwd(q, k, v, float(alphas[layer]), f, 12)
         check_bwd(q, k, v, g, float(alphas[layer]), f, 12)
+
+
+RANDOM = _random_cases(n=8, seed=1404)
+
+
+@pytest.mark.parametrize("dtype,kernel", FWD_KERNELS, ids=["f32", "bf16-gather", "bf16-staged", "bf16-mma"])
+@pytest.mark.parametrize("case", RANDOM, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]:.4f}{c[6]}{c[7]}d{int(c[8])}"
+                                              for c in RANDOM])
+def test_forward_random_shapes(case, dtype, kernel):
+    """Every forward kernel on seeded random shapes (see _random_cases)."""
+    Bn, H, Hkv, T, W, alpha, base, K, dedup = case
+    q, k, v = inputs.qkv(Bn, H, T, seed=T * 17 + W, dtype=dtype, Hkv=Hkv)
+    try:
+        check_fwd(q, k, v, alpha, _offsets(base, K), W, dedup, kernel)
+    except fa.FibattnError as e:
+        if e.status == 2:
+            pytest.skip(str(e))
+        raise
+
+
+@pytest.mark.parametrize("dtype,kernel", BWD_KERNELS, ids=["f32", "bf16-gather", "bf16-mma"])
+@pytest.mark.parametrize("case", RANDOM, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]:.4f}{c[6]}{c[7]}d{int(c[8])}"
+                                              for c in RANDOM])
+def test_backward_random_shapes(case, dtype, kernel):
+    """Every backward query pass on seeded random shapes (see _random_cases)."""
+    Bn, H, Hkv, T, W, alpha, base, K, dedup = case
+    q, k, v = inputs.qkv(Bn, H, T, seed=T * 17 + W + 1, dtype=dtype, Hkv=Hkv)
+    g = inputs.dout(Bn, H, T, seed=T * 17 + W + 2, dtype=dtype)
+    try:
+        check_bwd(q, k, v, g, alpha, _offsets(base, K), W, dedup, kernel)
+    except fa.FibattnError as e:
+        if e.status == 2:
+            pytest.skip(str(e))
+        raise

@@ -27,7 +27,7 @@ import oracle as O
 import paper_2606_28560_gb300 as fa
 from paper_2606_28560_gb300 import inputs
 from tests.independent_forms import rope_complex_np
-from tests.test_gpu_parity import NTHREADS, SMALL, TOL, _f64, _rel
+from tests.test_gpu_parity import NTHREADS, SMALL, TOL, _f64, _random_cases, _rel
 
 pytestmark = pytest.mark.gpu
 
@@ -215,22 +215,6 @@ def test_calls_from_a_fresh_host_thread():
         for a, b in zip(main[name][:3], got[name][:3]):
             assert torch.equal(a, b)
     assert torch.equal(got["fwd"][0], out)
-
-
-def _random_cases(n=16, seed=2606):
-    """Seeded shapes across the launch paths: grouped-query heads (G = 1, 2, 4),
-    lengths from 1 to 700 (ragged last tiles), W = 0..16, fractional alpha
-    over [0.5, 1.5], both bases, K = 0..15, dedup on and off."""
-    rng = np.random.default_rng(seed)
-    cases = []
-    for _ in range(n):
-        Hkv = int(rng.integers(1, 3))
-        G = int(rng.choice([1, 2, 4]))
-        base = str(rng.choice(["fib", "pow2"]))
-        K = int(rng.integers(0, 16 if base == "fib" else 11))
-        cases.append((int(rng.integers(1, 3)), Hkv * G, Hkv, int(rng.integers(1, 701)), int(rng.integers(0, 17)),
-                      float(np.float32(rng.uniform(0.5, 1.5))), base, K, bool(rng.integers(0, 2))))
-    return cases
 
 
 RANDOM = _random_cases()
