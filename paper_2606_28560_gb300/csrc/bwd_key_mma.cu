@@ -211,7 +211,8 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     if (waited) pdl_wait();
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bar;
-    __shared__ float rvals[kWarps][kMmaMaxRungs][16];     // per warp: rung values of its slab columns
+    // per warp: rung values of its slab columns; after a pass, its output rows
+    __shared__ __align__(16) float rvals[kWarps][kMmaMaxRungs][16];
     __shared__ float wils[kWarps][32];                    // per warp: 1 / row sum of its band queries
     __shared__ float red[kMmaMaxRungs];                   // block 0: dL/dd_k
     __shared__ long long red64[kWarps * kMmaMaxRungs];
@@ -279,6 +280,12 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
 #pragma unroll
                 for (int u = 0; u < 2; ++u) rope_cs(a.rope, 8 * n + 2 * c4 + u, klo, ec[n][u], es[n][u]);
         }
+        // Rows g4 (half 0) and g4 + 8 (half 1) leave through this warp's table,
+        // 8 rows of 128 bytes at a time (16-byte chunk c of row r at chunk
+        // c ^ r), and go out as runs of consecutive rows: a warp's stores then
+        // cover 512 contiguous bytes instead of 8 rows' 16-byte pieces.
+        unsigned* stage = reinterpret_cast<unsigned*>(&rvals[warp][0][0]);
+        __syncwarp();                             // the pass's reads of the table are done
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
             if (pass && half == 1) {
@@ -293,8 +300,6 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
                         ec[n][u] = cn;
                     }
             }
-            if (!(half ? vhi : vlo)) continue;
-            const int key = half ? khi : klo;
 #pragma unroll
             for (int n = 0; n < 8; ++n) {
                 acc[n][2 * half] *= sc;
@@ -311,10 +316,22 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
                     }
                 }
             }
-            __nv_bfloat16* row = dst + (size_t)key * kHeadDim;
 #pragma unroll
             for (int n = 0; n < 8; ++n)
-                *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(acc[n][2 * half], acc[n][2 * half + 1]);
+                stage[g4 * 32 + ((n ^ g4) << 2) + c4] = pack_bf16(acc[n][2 * half], acc[n][2 * half + 1]);
+            __syncwarp();
+            // rows bw + 8 half + r, r < 8 (7 in the second half: row 15 of the
+            // tile is the next warp's), below T
+            const int nrow = min(half ? kRowsPerWarp - 8 : 8, s.T - (bw + 8 * half));
+#pragma unroll
+            for (int c = lane; c < 64; c += 32) {
+                const int r = c >> 3, ch = c & 7;
+                if (r < nrow) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(stage + r * 32 + ((ch ^ r) << 2));
+                    *reinterpret_cast<uint4*>(dst + (size_t)(bw + 8 * half + r) * kHeadDim + 8 * ch) = v;
+                }
+            }
+            __syncwarp();                         // the table is read before it is rewritten
         }
     }
 }
