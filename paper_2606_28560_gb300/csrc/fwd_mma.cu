@@ -66,6 +66,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     constexpr int Wp = NT * 8 - 16;               // window rows before the tile
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[2];
+    __shared__ __align__(16) unsigned ostage[kWarps * TEAMS][256];   // per warp: 8 output rows on their way out
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* vbuf = TEAMS == 1 ? buf : buf + (size_t)L.rows * 128;
     const unsigned sbase = smem_u32(buf), vbase = smem_u32(vbuf);
@@ -402,26 +403,38 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const bool ok = ok_k && ok_v;
     const float inv_lo = ok ? 1.f / llo : __int_as_float(0x7fc00000);
     const float inv_hi = ok ? 1.f / lhi : __int_as_float(0x7fc00000);
+    // Rows g4 (half 0) and g4 + 8 (half 1) leave through this warp's stage, 8
+    // rows of 128 bytes at a time (16-byte chunk c of row r at chunk c ^ r), and
+    // go out as runs of consecutive rows: 512 contiguous bytes per warp store.
     __nv_bfloat16* O = reinterpret_cast<__nv_bfloat16*>(a.out) + rowbase * kHeadDim;
-    if (vlo && wrel + g4 < kMmaTile) {
-        __nv_bfloat16* row = O + (size_t)qlo * kHeadDim;
+    unsigned* stage = ostage[team * kWarps + warp];
+#pragma unroll
+    for (int half = 0; half < 2; ++half) {
+        const float inv = half ? inv_hi : inv_lo;
 #pragma unroll
         for (int n = 0; n < 8; ++n)
-            *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][0] * inv_lo, o[n][1] * inv_lo);
-        if (c4 == 0) {
-            a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
-            if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qlo] = 1.f / llo;
+            stage[g4 * 32 + ((n ^ g4) << 2) + c4] = pack_bf16(o[n][2 * half] * inv, o[n][2 * half + 1] * inv);
+        __syncwarp();
+        // rows bw + 8 half + r, r < 8 (7 in the second half: row 15 of the
+        // tile is the next warp's), below T
+        const int nrow = min(half ? kRowsPerWarp - 8 : 8, s.T - (bw + 8 * half));
+#pragma unroll
+        for (int c = lane; c < 64; c += 32) {
+            const int r = c >> 3, ch = c & 7;
+            if (r < nrow) {
+                const uint4 v = *reinterpret_cast<const uint4*>(stage + r * 32 + ((ch ^ r) << 2));
+                *reinterpret_cast<uint4*>(O + (size_t)(bw + 8 * half + r) * kHeadDim + 8 * ch) = v;
+            }
         }
+        __syncwarp();                             // the stage is read before it is rewritten
     }
-    if (vhi && wrel + g4 + 8 < kMmaTile) {
-        __nv_bfloat16* row = O + (size_t)qhi * kHeadDim;
-#pragma unroll
-        for (int n = 0; n < 8; ++n)
-            *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(o[n][2] * inv_hi, o[n][3] * inv_hi);
-        if (c4 == 0) {
-            a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
-            if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qhi] = 1.f / lhi;
-        }
+    if (c4 == 0 && vlo) {
+        a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
+        if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qlo] = 1.f / llo;
+    }
+    if (c4 == 0 && vhi) {
+        a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
+        if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qhi] = 1.f / lhi;
     }
     }                                             // query heads of the group
 }
@@ -467,10 +480,10 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.buf_rows * 128 + 1024; }
 
-// the two barriers of a CTA, rounded up
-size_t fwd_mma_static_smem() { return 64; }
+// the two barriers of a CTA (rounded up) and its warps' output stages
+size_t fwd_mma_static_smem() { return 64 + kWarps * 1024; }
 
-size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - fwd_mma_static_smem(); }
+size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - 64 - 2 * kWarps * 1024; }
 
 namespace {
 
