@@ -573,7 +573,7 @@ def run_e2e(args, wl, device, dist):
     ev_oc = [torch.cuda.Event() for _ in range(L)]           # out of layer l read back
     ev_gc = [torch.cuda.Event() for _ in range(L)]           # dq, dk, dv of layer l read back
     ev_th = torch.cuda.Event()                               # dtheta read back
-    steps = max(2, min(args.steps, 10))
+    steps = max(2, min(args.steps, 20))
     state = {"step": 0}
 
     def one():
@@ -627,13 +627,17 @@ def run_e2e(args, wl, device, dist):
         e0.record(comp)
         s_in.wait_stream(comp)                   # the first timed copies start after e0
         s_out.wait_stream(comp)
-        for _ in range(steps):
+        # per step: when its last result (dtheta) is on the host
+        done = [torch.cuda.Event(enable_timing=True) for _ in range(steps)]
+        for i in range(steps):
             one()
+            done[i].record(s_out)
         comp.wait_stream(s_out)                  # the last step ends when its results are on the host
         comp.wait_stream(s_in)
         e1.record(comp)
         torch.cuda.synchronize(device)
     ms = max_over_ranks(e0.elapsed_time(e1), device)
+    gaps = sorted(done[i].elapsed_time(done[i + 1]) for i in range(steps - 1))
     world = torch.distributed.get_world_size() if dist else 1
     value = job_throughput(world, steps, ms)
     bi = n_in * B * H * T * ROW_BYTES
@@ -641,6 +645,8 @@ def run_e2e(args, wl, device, dist):
     ok = all(torch.equal(host_out[4 * l + 1].to(device), wl.dq[l]) for l in (0, L - 1))
     return {"value": value, "unit": UNIT, "h2d_bytes_per_step": bi, "d2h_bytes_per_step": bo,
             "ms_per_step": round(ms / steps, 4), "results_on_host_match": ok,
+            "step_gap_ms": {"min": round(gaps[0], 4), "median": round(gaps[len(gaps) // 2], 4),
+                            "max": round(gaps[-1], 4)},
             "copies": "two copy streams overlapping the compute; device inputs double-buffered by step "
                       "(the next step's inputs stream in while this step's gradients stream out); per-layer events"}
 

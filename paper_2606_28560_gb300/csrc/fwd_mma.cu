@@ -66,7 +66,10 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     constexpr int Wp = NT * 8 - 16;               // window rows before the tile
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[2];
-    __shared__ __align__(16) unsigned ostage[kWarps * TEAMS][256];   // per warp: 8 output rows on their way out
+    // TEAMS = 1, per warp: 8 output rows on their way out (the grouped form,
+    // one 16-warp CTA per SM, stores directly: the stage's shared memory costs
+    // it more L1 than the scattered stores do)
+    __shared__ __align__(16) unsigned ostage[TEAMS == 1 ? kWarps : 1][256];
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     unsigned char* vbuf = TEAMS == 1 ? buf : buf + (size_t)L.rows * 128;
     const unsigned sbase = smem_u32(buf), vbase = smem_u32(vbuf);
@@ -407,26 +410,39 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     // rows of 128 bytes at a time (16-byte chunk c of row r at chunk c ^ r), and
     // go out as runs of consecutive rows: 512 contiguous bytes per warp store.
     __nv_bfloat16* O = reinterpret_cast<__nv_bfloat16*>(a.out) + rowbase * kHeadDim;
-    unsigned* stage = ostage[team * kWarps + warp];
+    if constexpr (TEAMS == 1) {
+        unsigned* stage = ostage[warp];
 #pragma unroll
-    for (int half = 0; half < 2; ++half) {
-        const float inv = half ? inv_hi : inv_lo;
+        for (int half = 0; half < 2; ++half) {
+            const float inv = half ? inv_hi : inv_lo;
 #pragma unroll
-        for (int n = 0; n < 8; ++n)
-            stage[g4 * 32 + ((n ^ g4) << 2) + c4] = pack_bf16(o[n][2 * half] * inv, o[n][2 * half + 1] * inv);
-        __syncwarp();
-        // rows bw + 8 half + r, r < 8 (7 in the second half: row 15 of the
-        // tile is the next warp's), below T
-        const int nrow = min(half ? kRowsPerWarp - 8 : 8, s.T - (bw + 8 * half));
+            for (int n = 0; n < 8; ++n)
+                stage[g4 * 32 + ((n ^ g4) << 2) + c4] = pack_bf16(o[n][2 * half] * inv, o[n][2 * half + 1] * inv);
+            __syncwarp();
+            // rows bw + 8 half + r, r < 8 (7 in the second half: row 15 of the
+            // tile is the next warp's), below T
+            const int nrow = min(half ? kRowsPerWarp - 8 : 8, s.T - (bw + 8 * half));
 #pragma unroll
-        for (int c = lane; c < 64; c += 32) {
-            const int r = c >> 3, ch = c & 7;
-            if (r < nrow) {
-                const uint4 v = *reinterpret_cast<const uint4*>(stage + r * 32 + ((ch ^ r) << 2));
-                *reinterpret_cast<uint4*>(O + (size_t)(bw + 8 * half + r) * kHeadDim + 8 * ch) = v;
+            for (int c = lane; c < 64; c += 32) {
+                const int r = c >> 3, ch = c & 7;
+                if (r < nrow) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(stage + r * 32 + ((ch ^ r) << 2));
+                    *reinterpret_cast<uint4*>(O + (size_t)(bw + 8 * half + r) * kHeadDim + 8 * ch) = v;
+                }
             }
+            __syncwarp();                             // the stage is read before it is rewritten
         }
-        __syncwarp();                             // the stage is read before it is rewritten
+    } else {
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+            if (!(half ? vhi : vlo)) continue;
+            const float inv = half ? inv_hi : inv_lo;
+            __nv_bfloat16* row = O + (size_t)(half ? qhi : qlo) * kHeadDim;
+#pragma unroll
+            for (int n = 0; n < 8; ++n)
+                *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) =
+                    pack_bf16(o[n][2 * half] * inv, o[n][2 * half + 1] * inv);
+        }
     }
     if (c4 == 0 && vlo) {
         a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
@@ -483,7 +499,7 @@ size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.buf_rows * 128 
 // the two barriers of a CTA (rounded up) and its warps' output stages
 size_t fwd_mma_static_smem() { return 64 + kWarps * 1024; }
 
-size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - 64 - 2 * kWarps * 1024; }
+size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - 64 - 1024; }
 
 namespace {
 
