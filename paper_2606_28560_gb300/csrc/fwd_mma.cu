@@ -181,16 +181,30 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
     const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
     const size_t rowbase = (size_t)bh * s.T;
-    if constexpr (SAVE) {                         // rotated query rows 0..14 of the warp's tile
+    if constexpr (SAVE) {
+        // rotated query rows 0..14 of the warp's tile, through the warp's stage
+        // (16-byte chunk c of row r at chunk c ^ r) and out as runs of rows
+        static_assert(TEAMS == 1, "the residuals are written by the one-head form");
+        unsigned* stage = ostage[warp];
+        __half* QT = reinterpret_cast<__half*>(a.res_qt) + rowbase * kHeadDim;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-            if (!(half ? vhi : vlo)) continue;
-            __half* row = reinterpret_cast<__half*>(a.res_qt) + (rowbase + (half ? qhi : qlo)) * kHeadDim;
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
-                *reinterpret_cast<unsigned*>(row + 16 * kc + 2 * c4) = qa[kc][half];
-                *reinterpret_cast<unsigned*>(row + 16 * kc + 8 + 2 * c4) = qa[kc][2 + half];
+                stage[g4 * 32 + (((2 * kc) ^ g4) << 2) + c4] = qa[kc][half];
+                stage[g4 * 32 + (((2 * kc + 1) ^ g4) << 2) + c4] = qa[kc][2 + half];
             }
+            __syncwarp();
+            const int nrow = min(half ? kRowsPerWarp - 8 : 8, s.T - (bw + 8 * half));
+#pragma unroll
+            for (int c = lane; c < 64; c += 32) {
+                const int r = c >> 3, ch = c & 7;
+                if (r < nrow) {
+                    const uint4 v = *reinterpret_cast<const uint4*>(stage + r * 32 + ((ch ^ r) << 2));
+                    *reinterpret_cast<uint4*>(QT + (size_t)(bw + 8 * half + r) * kHeadDim + 8 * ch) = v;
+                }
+            }
+            __syncwarp();                         // the stage is read before it is rewritten
         }
     }
 
