@@ -170,6 +170,17 @@ def test_residual_bytes():
     assert B.lib().fibattn_residual_bytes(1, 2, 8, 64, 2, 33, 1) == 0                # K > 32
 
 
+def test_offsets_marshalling():
+    """Offsets reach the C ABI as a contiguous fp32 host array: one that is
+    already so is passed as it is, anything else (a list, fp64, a strided
+    view) is copied into one with the same values."""
+    f = fa.base("fib", 15)
+    assert B._offsets(f) is f
+    for other in (list(map(float, f)), f.astype(np.float64), np.repeat(f, 2)[::2]):
+        g = B._offsets(other)
+        assert g.dtype == np.float32 and g.flags.c_contiguous and np.array_equal(g, f)
+
+
 def test_missing_library_fails_loudly(monkeypatch, tmp_path):
     monkeypatch.setattr(build_mod, "LIB", str(tmp_path / "nope.so"))
     monkeypatch.setattr(B, "_lib", None)
