@@ -24,8 +24,10 @@
 //
 // Staging: the CTA's union of key rows (rotated keys, fp16) and then of value
 // rows (bf16, same buffer) is copied by TMA (3-D tensor maps [heads][T][64],
-// 8-row boxes, 128-byte swizzle, rows outside [0, T) zero-filled) under an
-// mbarrier with a bounded wait.
+// 64-row boxes with 8-row tails, 128-byte swizzle, rows outside [0, T)
+// zero-filled) under an mbarrier with a bounded wait.  The one-head form
+// writes its output rows (and the rotated query rows it keeps) through a
+// 1 KB stage per warp, as 16-byte pieces of runs of consecutive rows.
 #include <cmath>
 
 #include <cuda.h>
