@@ -15,7 +15,8 @@
 // with X = dO rows (bf16, pass 0: dv) and then X = q~ rows (fp16, pass 1:
 // dk~, dS in place of p).  The CTA stages the union of the query rows its
 // warps read, one tensor (and query head) at a time, in one buffer.
-// A-operand values: p as bf16, dS as fp16; accumulation fp32.
+// A-operand values: p as bf16, dS as fp16; accumulation fp32.  A warp's dv
+// and dk rows leave through its rung table as runs of consecutive rows.
 #include <cmath>
 
 #include "fibattn_internal.cuh"
