@@ -204,6 +204,19 @@ class Workload:
                    dtheta=self.dth[l] if rung_grads else None, dd=self.dd[l] if rung_grads else None,
                    workspace=self.ws_b, rotated_k=self.rk[l], rung_grads=rung_grads, residuals=self._res(l))
 
+    def step_static(self, alphas, round_offsets: bool):
+        """The same step under a static schedule (no dL/dtheta): rung
+        distances interpolated, or rounded to integers (the paper's
+        integer-offset variants)."""
+        fa = self.fa
+        for l in range(self.L):
+            fa.fwd(self.q[l], self.k[l], self.v[l], float(alphas[l]), self.f, W, out=self.out[l], lse=self.lse[l],
+                   workspace=self.ws_f, rotated_k=self.rk[l], residuals=self._res(l), round_offsets=round_offsets)
+        for l in reversed(range(self.L)):
+            fa.bwd(self.q[l], self.k[l], self.v[l], self.lse[l], self.g[l], float(alphas[l]), self.f, W,
+                   out=self.out[l], dq=self.dq[l], dk=self.dk[l], dv=self.dv[l], workspace=self.ws_b,
+                   rotated_k=self.rk[l], rung_grads=False, residuals=self._res(l), round_offsets=round_offsets)
+
     def fwd_only(self, W_):
         fa = self.fa
         for l in range(self.L):
@@ -211,35 +224,41 @@ class Workload:
                    workspace=self.ws_f, rotated_k=self.rk[l])
 
 
-def algorithmic_bytes(residuals=True):
-    """Bytes each kernel must move once per launch (bf16 rows of 128 B,
-    fp32 lse and fp32 P / dS slots).  S = W + 1 + K slots per query.  With
-    the forward residuals the forward also writes q~ (fp16 rows), the
-    unnormalised weight per slot, the rung score differences and 1 / (weight
-    sum) per query, and the backward reads those instead of recomputing the
-    scores."""
+def method_bytes():
+    """Bytes the method itself must move per launch of each kernel (the
+    compulsory traffic of the attention, bf16 rows of 128 B, fp32 lse): the
+    forward reads Q, K (rotated), V and writes O and lse; the query pass reads
+    q, k, v, dO, O and lse and writes dQ; the key pass reads q and dO and
+    writes dK and dV.  The RoPE prologue moves no method bytes of its own (its
+    key read is the forward's K, counted there)."""
+    n = B * H * T
+    rows = n * ROW_BYTES
+    return {"fwd": 4 * rows + 4 * n, "rope_k": 0,
+            "bwd_query_mma": 6 * rows + 4 * n,
+            "bwd_key_mma": 4 * rows}
+
+
+def overhead_bytes():
+    """Traffic the design adds on top of the method bytes, per launch: the
+    rotated keys written by the prologue and read in place of K; the forward
+    residuals (rotated q as bf16 rows, the unnormalised weight of each of the S
+    slots, the rung score differences, 1 / row sum) written by the forward and
+    read by the backward; dS per slot written by the query pass and, with the
+    weights, read by the key pass."""
     n = B * H * T
     S = W + 1 + K
     rows = n * ROW_BYTES
-    if residuals:
-        return {
-            # Q, K~, V read; O, q~ written; lse, weight per slot, sd, 1/l written
-            "fwd": 5 * rows + 2 * 4 * n + 4 * n * S + 4 * n * K,
-            "rope_k": 2 * rows,
-            # dO, O, K~, V read; dQ written; weights, sd, 1/l read; dS written
-            "bwd_query_mma": 5 * rows + 2 * 4 * n * S + 4 * n * K + 4 * n,
-            # Q~ dO read, dK dV written, weights/dS and 1/l read
-            "bwd_key_mma": 4 * rows + 2 * 4 * n * S + 4 * n,
-        }
-    return {
-        "fwd": 4 * rows + 4 * n,                           # Q, K~, V read; O written; lse
-        "rope_k": 2 * rows, "rope_q": 2 * rows,            # read, write rotated
-        "bwd_query": 5 * rows + 4 * n + 2 * 4 * n * S,     # Q~ K~ V dO read, dQ written, lse, P/dS written
-        # Q, dO, O, K~, V read; dQ, Q~ written; lse read; P/dS written
-        "bwd_query_mma": 7 * rows + 4 * n + 2 * 4 * n * S,
-        "bwd_key": 4 * rows + 2 * 4 * n * S,               # Q~ dO read, dK dV written, P/dS read
-        "bwd_key_mma": 4 * rows + 2 * 4 * n * S,
-    }
+    return {"rope_k": 2 * rows,
+            "fwd": rows + 4 * n * S + 4 * n * K + 4 * n,
+            "bwd_query_mma": 4 * n * S + 4 * n * K + 4 * n + 4 * n * S,
+            "bwd_key_mma": 2 * 4 * n * S + 4 * n}
+
+
+def step_method_bytes():
+    """Per step (16 layers of forward and backward): each tensor once, 512 B
+    forward (Q, K, V, O) and 1024 B backward (Q, K, V, O, dO read; dQ, dK, dV
+    written) per query-head."""
+    return L * B * H * T * (4 + 8) * ROW_BYTES
 
 
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch,
@@ -345,17 +364,27 @@ def run_gpu(args, rank, world, device):
     ms_max = max_over_ranks(ms, device)
     value = job_throughput(world, args.steps, ms_max)
 
-    # roofline of the dominant kernel (largest share of device time)
+    # roofline of the dominant kernel (largest share of device time), on the
+    # method's bytes; the design's extra traffic is reported beside it
     hbm, peak_kind = peaks()
-    algo = algorithmic_bytes()
+    algo = method_bytes()
+    over = overhead_bytes()
     tot = sum(v[0] for v in prof.values()) or 1.0
     dom = max(prof.items(), key=lambda kv: kv[1][0])[0] if prof else "fwd"
     dms, dcnt = prof.get(dom, (0.0, 1))
     avg_s = dms / max(dcnt, 1) / 1e3
     achieved = algo.get(dom, 0) / avg_s / 1e9 if avg_s > 0 else 0.0
+
+    def per_launch_s(v):
+        return v[0] / max(v[1], 1) / 1e3
+
     kernels = {k: {"ms_per_step": round(v[0], 4), "launches_per_step": v[1], "share": round(v[0] / tot, 4),
                    "us_per_launch": round(v[0] / max(v[1], 1) * 1e3, 2),
-                   "algo_GBps": round(algo.get(k, 0) / (v[0] / max(v[1], 1) / 1e3) / 1e9, 1) if v[0] > 0 else None}
+                   "method_bytes_per_launch": algo.get(k, 0), "overhead_bytes_per_launch": over.get(k, 0),
+                   "method_GBps": round(algo.get(k, 0) / per_launch_s(v) / 1e9, 1) if v[0] > 0 else None,
+                   "method_frac_of_hbm": round(algo.get(k, 0) / per_launch_s(v) / 1e9 / hbm, 4) if v[0] > 0 else None,
+                   "with_overhead_GBps": round((algo.get(k, 0) + over.get(k, 0)) / per_launch_s(v) / 1e9, 1)
+                   if v[0] > 0 else None}
                for k, v in prof.items()}
 
     # forward only at the same shape (W sweep): layer time from a graph without
@@ -406,6 +435,22 @@ def run_gpu(args, rank, world, device):
         torch.cuda.synchronize(device)
         integer[name] = {"ms_per_step": round(a0.elapsed_time(a1) / reps, 4)}
         del gi
+    lin = wl.fa.alpha_schedule("linear", L)
+    for name, rnd in (("linear_rounded_no_dtheta", True), ("linear_interpolated_no_dtheta", False)):
+        gi = capture(lambda: wl.step_static(lin, rnd), device, profile=False)
+        for _ in range(2):
+            gi.replay()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        reps = max(3, args.steps // 3)
+        a0.record(stream)
+        for _ in range(reps):
+            gi.replay()
+        a1.record(stream)
+        torch.cuda.synchronize(device)
+        integer[name] = {"ms_per_step": round(a0.elapsed_time(a1) / reps, 4)}
+        del gi
+    integer["linear_interpolated_over_rounded"] = round(integer["linear_interpolated_no_dtheta"]["ms_per_step"] /
+                                                        integer["linear_rounded_no_dtheta"]["ms_per_step"], 3)
     integer["learned_alpha_ms_per_step"] = round(ms_max / args.steps, 4)
     integer["interpolated_over_integer"] = round(integer["learned_alpha_ms_per_step"] /
                                                  integer["alpha1_with_dtheta"]["ms_per_step"], 3)
@@ -432,7 +477,7 @@ def run_gpu(args, rank, world, device):
     e2e = run_e2e(args, wl, device, dist)
     stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
-                algo=algo, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
+                algo=algo, over=over, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
                 stack=stack, integer=integer, gqa=gqa, recompute=recompute,
                 median_ms=step_ms[len(step_ms) // 2], min_ms=step_ms[0], max_ms=step_ms[-1])
 
@@ -841,7 +886,12 @@ def main():
             "roofline": {"bound": "hbm", "kernel": r["dom"], "achieved": round(r["achieved"], 1),
                          "peak": r["hbm"], "unit": "GB/s", "frac": round(r["achieved"] / r["hbm"], 4),
                          "traffic": ncu_traffic(r["dom"]), "peak_source": r["peak_kind"],
-                         "algorithmic_bytes_per_launch": r["algo"].get(r["dom"])},
+                         "algorithmic_bytes_per_launch": r["algo"].get(r["dom"]),
+                         "overhead_bytes_per_launch": r["over"].get(r["dom"]),
+                         "step": {"method_bytes": step_method_bytes(),
+                                  "achieved": round(step_method_bytes() / (r["ms"] / args.steps / 1e3) / 1e9, 1),
+                                  "frac": round(step_method_bytes() / (r["ms"] / args.steps / 1e3) / 1e9 / r["hbm"],
+                                                4)}},
             "kernels": r["kernels"],
             "forward_only_B16H8T1024": r["fwd_sweep"],
             "autograd_stack_16_layers": r["stack"],

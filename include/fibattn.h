@@ -48,7 +48,11 @@ typedef enum {
     FIBATTN_ERR_INVALID_ARG = 1,   /* bad shape, pointer, alignment, alpha, ...   */
     FIBATTN_ERR_UNSUPPORTED = 2,   /* valid but not built (e.g. D != 64)           */
     FIBATTN_ERR_CUDA = 3,          /* a CUDA runtime call or launch failed         */
-    FIBATTN_ERR_INTERNAL = 4       /* an internal consistency check failed         */
+    FIBATTN_ERR_INTERNAL = 4,      /* an internal consistency check failed, or a
+                                      kernel gave up a bounded wait (see
+                                      fibattn_check_status)                        */
+    FIBATTN_ERR_RANGE = 5          /* an operand left the range of the library's
+                                      16-bit rotated rows (fibattn_check_status)   */
 } fibattn_status;
 
 typedef enum { FIBATTN_F32 = 0, FIBATTN_BF16 = 1 } fibattn_dtype;
@@ -59,10 +63,10 @@ typedef struct {
     float scale;       /* score scale; <= 0 means 1/sqrt(D)                            */
     int   Hkv;         /* key/value heads (GQA); 0 means Hkv = H                       */
     int   no_dedup;    /* 0: drop rungs with d_k <= W [default]; 1: keep them          */
-    int   fwd_kernel;  /* forward kernel: 0 automatic [default]; 1 row-gather kernel;
-                          2 shared-memory staged CUDA-core kernel; 3 tensor-core
-                          kernel (2 and 3: bf16 I/O only; 3: W <= 16, K <= 16;
-                          FIBATTN_ERR_UNSUPPORTED when the choice does not apply) */
+    int   fwd_kernel;  /* forward kernel: 0 automatic [default]; 1 row-gather kernel
+                          (any W and K, fp32 or bf16); 3 tensor-core kernel (bf16
+                          I/O, W <= 16, K <= 16); 2 is not built.
+                          FIBATTN_ERR_UNSUPPORTED when the choice does not apply. */
     int   bwd_kernel;  /* backward query pass: 0 automatic [default]; 1 row-gather
                           single sweep (Delta accumulated from the slots, `out`
                           unused); 2 tensor-core kernel (bf16 I/O, `out` given,
@@ -78,7 +82,7 @@ typedef struct {
     void* residuals;   /* optional device buffer of fibattn_residual_bytes(...) bytes,
                           16-byte aligned [NULL].  Given it, fibattn_fwd also writes
                           what the backward would otherwise recompute from q and k:
-                          the RoPE-rotated queries (fp16 [B][H][T][D]), the
+                          the RoPE-rotated queries (bf16 [B][H][T][D]), the
                           unnormalised softmax weight exp(s - max) of every
                           slot (fp32 [B][H][S][T], S = W + 1 + K: window
                           distances 0..W, then rung k at W + 1 + k; 0 where not
@@ -98,6 +102,14 @@ typedef struct {
                           in its tensor-core passes instead of recomputing the
                           scores; when its tensor-core passes do not apply it
                           ignores the buffer. */
+    int   round_offsets; /* 0: continuous distances d_k = fl32(alpha f_k), rungs
+                          interpolated [default]; 1: the integer-offset variants
+                          (Section 2, "Implementation note", the fused
+                          boolean-mask path): d_k rounded to the nearest integer,
+                          ties to even, after the fp32 product; every rung then
+                          reads one row.  fibattn_bwd then requires dtheta and dd
+                          to be NULL (the rounded distances do not vary with
+                          alpha). */
 } fibattn_opts;
 
 /* ---------------------------------------------------------------------------
@@ -154,13 +166,38 @@ size_t fibattn_residual_bytes(int B, int H, int T, int D, int W, int K, int dtyp
 const char* fibattn_last_error(void);
 
 /* ---------------------------------------------------------------------------
+ * Device status (no counterpart in the paper).  Kernels report two conditions
+ * that no argument check can catch before launch into a per-device status
+ * word, without stopping:
+ *   bit 0 -- a kernel gave up waiting for one of its own shared-memory staging
+ *            copies (each wait is bounded to 1 s of the GPU's global timer);
+ *            the affected tiles' outputs (out, lse, gradients) are NaN.
+ *   bit 1 -- a RoPE-rotated q or k entry reached 65520 in magnitude: the bf16
+ *            path keeps rotated rows in fp16 (for score precision), which
+ *            cannot hold it.
+ * fibattn_check_status synchronises `stream`, reads the calling thread's
+ * current device's word into *flags (may be NULL) and clears it.  Returns
+ * FIBATTN_ERR_INTERNAL if bit 0 was set, else FIBATTN_ERR_RANGE if bit 1 was
+ * set, else FIBATTN_OK.  Compute calls never synchronise to look at it.
+ * ------------------------------------------------------------------------- */
+int fibattn_check_status(void* stream, unsigned* flags);
+
+/* Test hook for the bounded wait: launches one warp on `stream` that waits on
+ * a shared-memory barrier no copy will complete, with a bound of timeout_us
+ * microseconds (1 .. 1e7); the wait runs out and sets status bit 0, which a
+ * following fibattn_check_status reports.  The kernel touches no memory but
+ * its own shared barrier and the status word. */
+int fibattn_test_wait_timeout(unsigned timeout_us, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Host-side parameter prep (no GPU needed).
  * ------------------------------------------------------------------------- */
 
-/* Rung prep (Section 2): d[k] = fl32(alpha * f[k]); s0[k] = floor(d[k]);
+/* Rung prep (Section 2): d[k] = fl32(alpha * f[k]) (with round_offsets then
+ * rounded to the nearest integer, ties to even); s0[k] = floor(d[k]);
  * w[k] = d[k] - s0[k]; active[k] = 1 unless dedup drops it (d[k] <= W).
  * Any output pointer may be NULL.  Host pointers. */
-int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup,
+int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup, int round_offsets,
                         float* d, int* s0, float* w, int* active);
 
 /* Base sequences (Section 2): kind 0 = Fibonacci 1,2,3,5,... ; kind 1 =
@@ -173,6 +210,11 @@ int fibattn_base(int kind, int K, float* f);
  * linear multiset, layer l takes linear index (stride*l mod L).
  * theta is read only for kind 1.  Host arrays. */
 int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, float* alpha);
+
+/* Inverse of the learned map on [0.5, 1.5]: theta[l] = log((alpha[l] - 0.5) /
+ * (1.5 - alpha[l])), the ends (theta = -/+ infinity) clamped to -/+ 30; used to
+ * start a learned theta at a static schedule's alpha.  Host arrays. */
+int fibattn_theta_of_alpha(int L, const float* alpha, float* theta);
 
 /* ---------------------------------------------------------------------------
  * Coverage of a layer stack (Section 4.2, "Why staggering widens coverage"):

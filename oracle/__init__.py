@@ -153,6 +153,14 @@ def offsets_fp32(alpha: float, f) -> np.ndarray:
     return out
 
 
+def offsets_rounded(alpha: float, f) -> np.ndarray:
+    """The integer-offset variants evaluated through the paper's fused
+    boolean-mask path (Section 2, "Implementation note"): d_k = fl32(alpha f_k)
+    rounded to the nearest integer, ties to even, so that every rung reads one
+    whole row (interpolation weight 0)."""
+    return np.rint(offsets_fp32(alpha, f))
+
+
 def coverage(alphas, f, W: int, T: int, dedup: bool = True) -> dict:
     """Distinct key distances a query reads in a stack of layers (Section 4.2,
     "Why staggering widens coverage"), as plain sets.  Layer l reads the window

@@ -15,7 +15,6 @@ in one copy.
 """
 from __future__ import annotations
 
-import math
 
 import torch
 
@@ -23,8 +22,9 @@ from . import binding as B
 
 
 def alpha_of_theta(theta: float) -> float:
-    """alpha = 0.5 + sigmoid(theta) (Section 2, "The per-layer scalar")."""
-    return 0.5 + 1.0 / (1.0 + math.exp(-theta))
+    """alpha = 0.5 + sigmoid(theta) (Section 2, "The per-layer scalar"), as the
+    library computes it (fibattn_alpha_schedule, learned kind)."""
+    return float(B.alpha_schedule("learned", 1, theta=[float(theta)])[0])
 
 
 class FibAttentionFunction(torch.autograd.Function):
@@ -109,10 +109,9 @@ class FibAttention(torch.nn.Module):
 
 
 def theta_of_alpha(alpha: float) -> float:
-    """Inverse of alpha_of_theta on (0.5, 1.5); the ends map to -/+ infinity,
-    clamped to +-30 (alpha within 1e-13 of the end)."""
-    a = min(max(alpha, 0.5 + 1e-13), 1.5 - 1e-13)
-    return max(-30.0, min(30.0, math.log((a - 0.5) / (1.5 - a))))
+    """Inverse of alpha_of_theta on [0.5, 1.5] (fibattn_theta_of_alpha); the
+    ends map to -/+ infinity, clamped to -/+ 30."""
+    return float(B.theta_of_alpha_array([float(alpha)])[0])
 
 
 def attention_stack(x: torch.Tensor, layers) -> torch.Tensor:
@@ -123,7 +122,8 @@ def attention_stack(x: torch.Tensor, layers) -> torch.Tensor:
     if not layers:
         return x
     dev = layers[0].theta.device
-    thetas = torch.stack([layer.theta.detach().to(device=dev, dtype=torch.float64) for layer in layers]).tolist()
-    for layer, th in zip(layers, thetas):
-        x = layer(x, x, x, alpha=alpha_of_theta(th))
+    thetas = torch.stack([layer.theta.detach().to(device=dev, dtype=torch.float32) for layer in layers]).tolist()
+    alphas = B.alpha_schedule("learned", len(layers), theta=thetas)
+    for layer, a in zip(layers, alphas):
+        x = layer(x, x, x, alpha=float(a))
     return x

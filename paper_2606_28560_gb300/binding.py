@@ -35,7 +35,8 @@ class FibattnError(RuntimeError):
 class Opts(ctypes.Structure):
     _fields_ = [("rope_base", ctypes.c_float), ("scale", ctypes.c_float),
                 ("Hkv", ctypes.c_int), ("no_dedup", ctypes.c_int), ("fwd_kernel", ctypes.c_int),
-                ("bwd_kernel", ctypes.c_int), ("rotated_k", ctypes.c_void_p), ("residuals", ctypes.c_void_p)]
+                ("bwd_kernel", ctypes.c_int), ("rotated_k", ctypes.c_void_p), ("residuals", ctypes.c_void_p),
+                ("round_offsets", ctypes.c_int)]
 
 
 def library_path() -> str:
@@ -66,14 +67,20 @@ def lib():
             L.fibattn_bwd.restype = ci
             L.fibattn_last_error.argtypes = []
             L.fibattn_last_error.restype = ctypes.c_char_p
-            L.fibattn_rung_params.argtypes = [cf, fp, ci, ci, ci, fp, ip, fp, ip]
+            L.fibattn_rung_params.argtypes = [cf, fp, ci, ci, ci, ci, fp, ip, fp, ip]
             L.fibattn_rung_params.restype = ci
             L.fibattn_base.argtypes = [ci, ci, fp]
             L.fibattn_base.restype = ci
             L.fibattn_alpha_schedule.argtypes = [ci, ci, fp, ci, fp]
             L.fibattn_alpha_schedule.restype = ci
+            L.fibattn_theta_of_alpha.argtypes = [ci, fp, fp]
+            L.fibattn_theta_of_alpha.restype = ci
             L.fibattn_residual_bytes.argtypes = [ci] * 7
             L.fibattn_residual_bytes.restype = sz
+            L.fibattn_check_status.argtypes = [vp, ctypes.POINTER(ctypes.c_uint)]
+            L.fibattn_check_status.restype = ci
+            L.fibattn_test_wait_timeout.argtypes = [ctypes.c_uint, vp]
+            L.fibattn_test_wait_timeout.restype = ci
             _lib = L
     return _lib
 
@@ -91,16 +98,16 @@ def _iptr(a: np.ndarray):
     return a.ctypes.data_as(ctypes.POINTER(ctypes.c_int))
 
 
-FWD_KERNELS = {"auto": 0, "gather": 1, "staged": 2, "mma": 3}
+FWD_KERNELS = {"auto": 0, "gather": 1, "mma": 3}
 BWD_KERNELS = {"auto": 0, "gather": 1, "mma": 2}
 
 
 def _opts(rope_base=1e4, scale=None, Hkv=None, dedup=True, fwd_kernel="auto", bwd_kernel="auto",
-          rotated_k=None, residuals=None) -> Opts:
+          rotated_k=None, residuals=None, round_offsets=False) -> Opts:
     return Opts(float(rope_base), float(scale) if scale else 0.0, int(Hkv or 0), 0 if dedup else 1,
                 FWD_KERNELS[fwd_kernel], BWD_KERNELS[bwd_kernel],
                 rotated_k.data_ptr() if rotated_k is not None else None,
-                residuals.data_ptr() if residuals is not None else None)
+                residuals.data_ptr() if residuals is not None else None, 1 if round_offsets else 0)
 
 
 @functools.lru_cache(maxsize=256)
@@ -124,7 +131,7 @@ def residuals_like(q: torch.Tensor, W: int, K: int) -> torch.Tensor:
 
 
 def residual_views(res: torch.Tensor, B, H, T, W, K):
-    """Views of a residual buffer: rotated q (fp16 [B,H,T,64]), the
+    """Views of a residual buffer: rotated q (bf16 [B,H,T,64]), the
     unnormalised softmax weight exp(s - max) per slot (fp32 [B,H,W+1+K,T]),
     far-minus-floor rung scores (fp32 [B,H,K,T]) and 1 / (sum of the weights)
     per query (fp32 [B,H,T]; p = weight * that); the arrays follow one another,
@@ -136,7 +143,7 @@ def residual_views(res: torch.Tensor, B, H, T, W, K):
     o_p = up(n * 64 * 2)
     o_sd = o_p + up(n * S * 4)
     o_il = o_sd + up(n * K * 4)
-    qt = res[:n * 128].view(torch.float16).view(B, H, T, 64)
+    qt = res[:n * 128].view(torch.bfloat16).view(B, H, T, 64)
     P = res[o_p:o_p + n * S * 4].view(torch.float32).view(B, H, S, T)
     sd = res[o_sd:o_sd + n * K * 4].view(torch.float32).view(B, H, K, T)
     il = res[o_il:o_il + n * 4].view(torch.float32).view(B, H, T)
@@ -201,6 +208,14 @@ def alpha_schedule(kind: str, L: int = 16, theta=None, stride: int = 7) -> np.nd
     return out
 
 
+def theta_of_alpha_array(alpha) -> np.ndarray:
+    """theta with 0.5 + sigmoid(theta) = alpha, per entry (fibattn_theta_of_alpha)."""
+    a = np.ascontiguousarray(np.atleast_1d(np.asarray(alpha, dtype=np.float32)))
+    out = np.zeros(len(a), dtype=np.float32)
+    _check(lib().fibattn_theta_of_alpha(len(a), _fptr(a), _fptr(out)))
+    return out
+
+
 def coverage(alphas, offsets, W: int, T: int, dedup: bool = True) -> dict:
     """Distinct key distances of a layer stack (see fibattn_coverage)."""
     al = np.ascontiguousarray(np.asarray(alphas, dtype=np.float32))
@@ -238,12 +253,12 @@ def staging_layout(kind: str, T: int, W: int, alpha: float, offsets, dedup: bool
     return dict(start=st[:m].copy(), len=ln[:m].copy(), smem=sm[:m].copy(), slab_row=slab[:K].copy())
 
 
-def rung_params(alpha: float, offsets, W: int, dedup: bool = True):
+def rung_params(alpha: float, offsets, W: int, dedup: bool = True, round_offsets: bool = False):
     f = _offsets(offsets)
     K = len(f)
     d = np.zeros(K, np.float32); w = np.zeros(K, np.float32)
     s0 = np.zeros(K, np.int32); act = np.zeros(K, np.int32)
-    _check(lib().fibattn_rung_params(float(alpha), _fptr(f), K, int(W), 0 if dedup else 1,
+    _check(lib().fibattn_rung_params(float(alpha), _fptr(f), K, int(W), 0 if dedup else 1, 1 if round_offsets else 0,
                                      _fptr(d), _iptr(s0), _fptr(w), _iptr(act)))
     return dict(d=d, s0=s0, w=w, active=act.astype(bool))
 
@@ -263,9 +278,11 @@ def bwd_workspace_bytes(B, H, T, W, K, dtype, Hkv=None, D=64) -> int:
 
 
 def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, dedup=True,
-        out=None, lse=None, workspace=None, stream=None, kernel="auto", rotated_k=None, residuals=None):
+        out=None, lse=None, workspace=None, stream=None, kernel="auto", rotated_k=None, residuals=None,
+        round_offsets=False):
     """Forward pass.  q [B,H,T,64]; k, v [B,Hkv,T,64] (fp32 or bf16, CUDA,
-    contiguous).  ``kernel``: "auto", "gather", "staged" or "mma".
+    contiguous).  ``kernel``: "auto", "gather" or "mma".  ``round_offsets``:
+    the integer-offset variants (rung distances rounded to integers).
     ``rotated_k``: optional buffer (``rotated_k_like(k)``) that receives the
     rotated keys for a later ``bwd(..., rotated_k=...)``.  ``residuals``:
     optional buffer (``residuals_like(q, W, K)``) that receives the rotated
@@ -276,7 +293,8 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
     f = _offsets(offsets)
     _check_rotated(rotated_k, k)
     _check_residuals(residuals, q, W, len(f))
-    o = _opts(rope_base, scale, Hkv, dedup, kernel, rotated_k=rotated_k, residuals=residuals)
+    o = _opts(rope_base, scale, Hkv, dedup, kernel, rotated_k=rotated_k, residuals=residuals,
+              round_offsets=round_offsets)
     code = _dtype_code(q)
     for t in (q, k, v):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
@@ -296,22 +314,24 @@ def fwd(q, k, v, alpha: float, offsets, W: int, *, rope_base=1e4, scale=None, de
 
 def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_base=1e4, scale=None, dedup=True,
         dq=None, dk=None, dv=None, dtheta=None, dd=None, workspace=None, stream=None, kernel="auto",
-        rotated_k=None, rung_grads=True, residuals=None):
+        rotated_k=None, rung_grads=True, residuals=None, round_offsets=False):
     """Backward pass.  ``out``: the forward output (optional; enables the
     tensor-core query pass).  ``kernel``: "auto", "gather" or "mma".
     ``rotated_k``: the buffer the forward of the same k filled (skips rotating
     k again).  ``residuals``: the buffer the forward of the same inputs filled
     (the tensor-core passes then read p, the rung score differences and the
     rotated queries instead of recomputing them).  ``rung_grads=False`` skips
-    dL/dtheta and dL/dd_k (a fixed schedule).  Returns (dq, dk, dv, dtheta [1],
-    dd [K]) on the device (dtheta, dd None without rung_grads)."""
+    dL/dtheta and dL/dd_k (a fixed schedule; required with ``round_offsets``).
+    Returns (dq, dk, dv, dtheta [1], dd [K]) on the device (dtheta, dd None
+    without rung_grads)."""
     B, H, T, D = q.shape
     Hkv = k.shape[1]
     f = _offsets(offsets)
     K = len(f)
     _check_rotated(rotated_k, k)
     _check_residuals(residuals, q, W, K)
-    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel, rotated_k=rotated_k, residuals=residuals)
+    o = _opts(rope_base, scale, Hkv, dedup, bwd_kernel=kernel, rotated_k=rotated_k, residuals=residuals,
+              round_offsets=round_offsets)
     code = _dtype_code(q)
     for t in (q, k, v, dout) + ((out,) if out is not None else ()):
         if not (t.is_cuda and t.is_contiguous() and t.dtype == q.dtype):
@@ -335,6 +355,27 @@ def bwd(q, k, v, lse, dout, alpha: float, offsets, W: int, *, out=None, rope_bas
     if dtheta is None and dd is None:
         return dq, dk, dv, None, None
     return dq, dk, dv, (dtheta[:1] if dtheta is not None else None), (dd[:K] if dd is not None else None)
+
+
+# ---------------------------------------------------------- device status ----
+
+def check_status(stream=None):
+    """Synchronise ``stream`` and read and clear the device status word
+    (fibattn_check_status).  Returns the flags; raises FibattnError when a
+    kernel gave up a bounded wait (status 4) or a rotated row overflowed fp16
+    (status 5)."""
+    flags = ctypes.c_uint(0)
+    rc = lib().fibattn_check_status(_stream_ptr(stream), ctypes.byref(flags))
+    if rc != 0:
+        e = FibattnError(rc, lib().fibattn_last_error().decode(errors="replace"))
+        e.flags = flags.value
+        raise e
+    return flags.value
+
+
+def test_wait_timeout(timeout_us: int, stream=None):
+    """Launch the library's bounded-wait probe (a wait that no copy completes)."""
+    _check(lib().fibattn_test_wait_timeout(int(timeout_us), _stream_ptr(stream)))
 
 
 # ------------------------------------------------------------- profiling ----

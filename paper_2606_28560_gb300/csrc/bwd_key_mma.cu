@@ -12,10 +12,12 @@
 // are products of a banded matrix with staged query rows:
 //   window band  acc += P_band^T  X[b, b+16+Wp)       P_band^T[r][x] = p(b+x, t = x-r)
 //   rung k       acc += Phat_k^T  X[b+s0, b+s0+16)    Phat_k^T[r][r] = (1-w) p, [r][r+1] = w p
-// with X = dO rows (bf16, pass 0: dv) and then X = q~ rows (fp16, pass 1:
+// with X = dO rows (bf16, pass 0: dv) and then X = q~ rows (bf16, pass 1:
 // dk~, dS in place of p).  The CTA stages the union of the query rows its
 // warps read, one tensor (and query head) at a time, in one buffer.
-// A-operand values: p as bf16, dS as fp16; accumulation fp32.  A warp's dv
+// A-operand values: p and dS as bf16 (the exponent range of fp32: no score
+// gradient underflows, however small the upstream gradient); accumulation
+// fp32.  A warp's dv
 // and dk rows leave through its rung table as runs of consecutive rows.
 #include <cmath>
 
@@ -31,25 +33,12 @@ using namespace mma;
 constexpr int kWarps = kMmaWarps;
 constexpr int kRowsPerWarp = 15;
 
-template <bool F16>
-__device__ __forceinline__ unsigned pack2(float lo, float hi) {
-    return F16 ? pack_f16(lo, hi) : pack_bf16(lo, hi);
-}
-template <bool F16>
-__device__ __forceinline__ void mma16816(float* d, const unsigned* a, unsigned b0, unsigned b1) {
-    if constexpr (F16) mma_f16_16816(d, a, b0, b1); else mma_bf16_16816(d, a, b0, b1);
-}
-template <bool F16>
-__device__ __forceinline__ void mma1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
-    if constexpr (F16) mma_f16_1688(d, a0, a1, b0); else mma_bf16_1688(d, a0, a1, b0);
-}
-
 // One staged tensor of one query head: accumulate banded A x staged rows.
-// X: p or dS of this query head, slot-major [S][T]; F16: the operand type.
+// X: p or dS of this query head, slot-major [S][T]; operands bf16.
 // IL (p from the forward residuals, unnormalised): 1 / (row sum) per query
 // of this head; the warp copies the entries its values need into its rung
 // table and its band strip (wil, 32 floats) and scales each value.
-template <int NT, bool F16>
+template <int NT>
 __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, const BwdArgs& a, const MmaLayout& L,
                                          unsigned sbase, int bw, int wrel, int g4, int c4, int lane, bool vlo,
                                          bool vhi, unsigned long long* bar, unsigned parity, bool& ok,
@@ -118,8 +107,8 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
     unsigned band[NT][2];
 #pragma unroll
     for (int j = 0; j < NT; ++j) {
-        band[j][0] = pack2<F16>(bv[j][0], bv[j][1]);
-        band[j][1] = pack2<F16>(bv[j][2], bv[j][3]);
+        band[j][0] = pack_bf16(bv[j][0], bv[j][1]);
+        band[j][1] = pack_bf16(bv[j][2], bv[j][3]);
     }
     ok = mbar_wait(bar, parity) && ok;
 
@@ -131,8 +120,8 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
             ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
-            mma16816<F16>(acc[n], afr, b0, b1);
-            mma16816<F16>(acc[n + 1], afr, b2, b3);
+            mma_bf16_16816(acc[n], afr, b0, b1);
+            mma_bf16_16816(acc[n + 1], afr, b2, b3);
         }
     }
     if constexpr (NT & 1) {
@@ -142,10 +131,10 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
         for (int n = 0; n < 8; n += 4) {
             unsigned b0, b1, b2, b3;
             ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 3)), b0, b1, b2, b3);
-            mma1688<F16>(acc[n], band[kk][0], band[kk][1], b0);
-            mma1688<F16>(acc[n + 1], band[kk][0], band[kk][1], b1);
-            mma1688<F16>(acc[n + 2], band[kk][0], band[kk][1], b2);
-            mma1688<F16>(acc[n + 3], band[kk][0], band[kk][1], b3);
+            mma_bf16_1688(acc[n], band[kk][0], band[kk][1], b0);
+            mma_bf16_1688(acc[n + 1], band[kk][0], band[kk][1], b1);
+            mma_bf16_1688(acc[n + 2], band[kk][0], band[kk][1], b2);
+            mma_bf16_1688(acc[n + 3], band[kk][0], band[kk][1], b3);
         }
     }
 
@@ -176,15 +165,15 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
             const float clo = fmaf(blo, w, alo), chi = fmaf(bhi, w, ahi);
             const float2 v0 = *reinterpret_cast<const float2*>(&rv[ii][2 * c4]);
             const float2 v8 = *reinterpret_cast<const float2*>(&rv[ii][2 * c4 + 8]);
-            const unsigned afr[4] = {pack2<F16>(clo * v0.x, chi * v0.y), 0u,
-                                     pack2<F16>(m2 * w * v8.x, 0.f), pack2<F16>(clo * v8.x, chi * v8.y)};
+            const unsigned afr[4] = {pack_bf16(clo * v0.x, chi * v0.y), 0u,
+                                     pack_bf16(m2 * w * v8.x, 0.f), pack_bf16(clo * v8.x, chi * v8.y)};
             const int xrow = L.act_smem[ii] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
             for (int n = 0; n < 8; n += 2) {
                 unsigned b0, b1, b2, b3;
                 ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
-                mma16816<F16>(acc[n], afr, b0, b1);
-                mma16816<F16>(acc[n + 1], afr, b2, b3);
+                mma_bf16_16816(acc[n], afr, b0, b1);
+                mma_bf16_16816(acc[n + 1], afr, b2, b3);
             }
         }
     }
@@ -260,16 +249,17 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
                 issue_rows(buf, &m.m64, &m.m8, L, j0, qhead, &bar, lane);
             }
             if (pass == 0)
-                key_pass<NT, false>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
-                                       rvals[warp], a.saved ? a.res_il + (size_t)qhead * s.T : nullptr, wils[warp]);
+                key_pass<NT>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
+                                 rvals[warp], a.saved ? a.res_il + (size_t)qhead * s.T : nullptr, wils[warp]);
             else
-                key_pass<NT, true>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
-                                      rvals[warp]);
+                key_pass<NT>(acc, X, a, L, sbase, bw, wrel, g4, c4, lane, vlo, vhi, &bar, parity, ok,
+                                 rvals[warp]);
             parity ^= 1u;
             // every warp is done with the staged rows before the buffer is refilled
             asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
             __syncthreads();
         }
+        if (!ok) raise_status(a.status, kStatusWaitTimeout);
         const float sc = ok ? (pass ? s.scale : 1.f) : __int_as_float(0x7fc00000);
         __nv_bfloat16* dst = reinterpret_cast<__nv_bfloat16*>(pass ? a.dk : a.dv) + krow0 * kHeadDim;
         // dk = R(-theta key) dk~: cos, sin of pair m = 8n + 2c4 + u (m + 32 in
@@ -375,7 +365,7 @@ cudaError_t launch_bwd_key_mma(const BwdArgs& a, const MmaLayout& L, cudaStream_
     if (grid <= 0) return cudaSuccess;
     RowMaps mq, mg;
     const int heads = a.s.B * a.s.H;
-    if (!encode_row_maps(&mq, a.qt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, heads) ||
+    if (!encode_row_maps(&mq, a.qt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads) ||
         !encode_row_maps(&mg, a.dout, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, heads))
         return cudaErrorInvalidValue;
     const size_t smem = bwd_key_mma_smem_bytes(L, a.saved != 0);

@@ -21,8 +21,17 @@
 // with s1, s0 the raw far and floor dot products.  p and dS per slot (zero
 // where not attended; slot-major arrays [head][slot][T], so that the key pass
 // reads runs of consecutive queries), Delta and the rotated queries go to the
-// workspace for the key-centric pass.  dS enters the dq MMAs as fp16 (11-bit significand);
-// accumulation is fp32.
+// workspace for the key-centric pass (the rotated queries as bf16).
+//
+// Range: dS enters the dq MMAs as fp16 (11-bit significand, the type of the
+// staged rotated keys), whose normal range (6.1e-5 .. 65504) is far narrower
+// than bf16's.  Each query row's dS is therefore multiplied by a power of two
+// c before the rounding, chosen from the row's largest |dp - Delta| (a bound
+// on |dS|, p <= 1) so that the scaled values reach [2^14, 2^15); the row's
+// dq~ is divided by c at the end (exact, a power of two).  So no row's score
+// gradients underflow or overflow fp16 whatever the magnitude of dO (a
+// bf16-autocast training step passes upstream gradients of 1e-5 .. 1e-8).
+// Accumulation is fp32.
 #include <cmath>
 
 #include "fibattn_internal.cuh"
@@ -40,6 +49,15 @@ constexpr int kRowsPerWarp = 15;
 
 __device__ __forceinline__ float bf_lo(unsigned u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf_hi(unsigned u) { return __uint_as_float(u & 0xffff0000u); }
+
+// Biased fp32 exponent of the power of two c with m c in [2^14, 2^15), for
+// m = a row's largest |dp - Delta| (c = 1 for m = 0 or subnormal; clamped so
+// that both c and 1 / c are normal).
+__device__ __forceinline__ int ds_scale_exp(float m) {
+    const int e = (__float_as_int(m) >> 23) & 0xff;
+    return e == 0 ? 127 : min(253, max(1, 268 - e));
+}
+__device__ __forceinline__ float exp_to_f(int ce) { return __int_as_float(ce << 23); }
 
 // DD: also the rung-distance gradient dL/dd_k (off when the caller asks for
 // neither dtheta nor dd, e.g. a fixed alpha schedule).
@@ -171,9 +189,11 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         dlt_hi = quad_sum(part[1]);
     }
 
-    // ---- q~ as fp16 A fragments (RoPE pairs m, m+32 in the same thread)
-    unsigned qa[4][4];
+    // ---- q~ as fp16 A fragments (RoPE pairs m, m+32 in the same thread), and
+    // as bf16 for the key pass (qs)
+    unsigned qa[4][4], qs[SV ? 1 : 4][4];
     if constexpr (!SV) {
+        float qmax = 0.f;                         // largest |q~| of the thread: fp16 holds < 65520
         unsigned qr[4][4];
         tile_frags(0, qr);
         float cs[2][4], sn[2][4];
@@ -212,14 +232,18 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                     const float xa = x[kc][j], xb = x[kc + 2][j];
                     x[kc][j] = xa * cs[kc][j] - xb * sn[kc][j];
                     x[kc + 2][j] = xb * cs[kc][j] + xa * sn[kc][j];
+                    qmax = fmaxf(qmax, fmaxf(fabsf(x[kc][j]), fabsf(x[kc + 2][j])));
                 }
             }
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
                 qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);
                 qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);
+                qs[kc][half] = pack_bf16(x[kc][0], x[kc][1]);
+                qs[kc][2 + half] = pack_bf16(x[kc][2], x[kc][3]);
             }
         }
+        if (qmax >= 65520.f) raise_status(a.status, kStatusRange);
     }
     // ---- q~ rows to the workspace (for the key pass): written in place of the
     // staged q rows, then stored by TMA (rows past T are clipped); the value
@@ -237,9 +261,9 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             const int row = wrel + g4 + 8 * half;
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
-                asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc) + 4 * c4), "r"(qa[kc][half]));
+                asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc) + 4 * c4), "r"(qs[kc][half]));
                 asm volatile("st.shared.b32 [%0], %1;\n" :: "r"(row_chunk(sbase, row, 2 * kc + 1) + 4 * c4),
-                             "r"(qa[kc][2 + half]));
+                             "r"(qs[kc][2 + half]));
             }
         }
         asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
@@ -302,23 +326,32 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             mma_bf16_16816(dpw[j], da[kc + 1], b2, b3);
         }
     }
-    // window band dS = p (dp - Delta) as fp16 A fragments (SV: here; else in
-    // the key phase, once the scores are known); dS per slot to the workspace
+    // the rows' largest |dp - Delta| over the band (rung terms join below):
+    // the bound on |dS| that sets the rows' fp16 scale
+    float emax_lo = 0.f, emax_hi = 0.f;
+#pragma unroll
+    for (int j = 0; j < NT; ++j) {
+        emax_lo = fmaxf(emax_lo, fmaxf(fabsf(dpw[j][0] - dlt_lo), fabsf(dpw[j][1] - dlt_lo)));
+        emax_hi = fmaxf(emax_hi, fmaxf(fabsf(dpw[j][2] - dlt_hi), fabsf(dpw[j][3] - dlt_hi)));
+    }
+    emax_lo = quad_max(emax_lo);
+    emax_hi = quad_max(emax_hi);
+    // window band dS = p (dp - Delta) (SV: here, kept in fp32 until the rows'
+    // scale is known; else in the key phase, once the scores are known); dS
+    // per slot to the workspace
     unsigned dsa[NT][2];
+    float dsb[SV ? NT : 1][4];
     if constexpr (SV) {
 #pragma unroll
         for (int j = 0; j < NT; ++j) {
-            float dsv[4];
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const bool hi = e >= 2;
                 const int r = hi ? g4 + 8 : g4;
                 const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
-                dsv[e] = pb[j][e] * (hi ? il_hi : il_lo) * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
-                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) DSg[(size_t)t * s.T + bw + r] = dsv[e];
+                dsb[j][e] = pb[j][e] * (hi ? il_hi : il_lo) * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
+                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) DSg[(size_t)t * s.T + bw + r] = dsb[j][e];
             }
-            dsa[j][0] = pack_f16(dsv[0], dsv[1]);
-            dsa[j][1] = pack_f16(dsv[2], dsv[3]);
         }
     }
     // Rungs in increasing d; those masked for every row of the warp's tile
@@ -347,7 +380,9 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     if constexpr (SV) {
         // Two rungs per iteration (their MMA and reduction chains are
         // independent); with an odd count the last pair repeats its first rung,
-        // whose second copy reads and writes the same values.
+        // whose second copy reads and writes the same values.  Each lane tracks
+        // its row's largest |dp - Delta| (lanes c4 < 2: row g4, else g4 + 8).
+        float emax_row = 0.f;
 #pragma unroll 1
         for (int i = 0; i < n_use; i += 2) {
             const int ib[2] = {i, i + 1 < n_use ? i + 1 : i};
@@ -397,6 +432,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
                 const float p = rv ? psd[0][ib[u]][row] * (up ? il_hi : il_lo) : 0.f;
                 const float e = dp - (up ? dlt_hi : dlt_lo);
+                emax_row = fmaxf(emax_row, fabsf(e));
                 ds[u] = p * e;
                 if constexpr (DD) {
                     const float sd = rv ? psd[1][ib[u]][row] : 0.f;
@@ -417,6 +453,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 }
             }
         }
+        emax_lo = fmaxf(emax_lo, __shfl_sync(0xffffffffu, emax_row, lane & ~3));
+        emax_hi = fmaxf(emax_hi, __shfl_sync(0xffffffffu, emax_row, (lane & ~3) | 2));
     } else {
     #pragma unroll 1
         for (int i = 0; i < n_use; ++i) {
@@ -447,6 +485,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             }
             const float dp_lo = quad_sum(x0), dp_hi = quad_sum(x2);
             const float ddp_lo = DD ? quad_sum(x1) : 0.f, ddp_hi = DD ? quad_sum(x3) : 0.f;
+            emax_lo = fmaxf(emax_lo, fabsf(dp_lo - dlt_lo));
+            emax_hi = fmaxf(emax_hi, fabsf(dp_hi - dlt_hi));
             if (c4 == 0) {
                 *reinterpret_cast<float2*>(dps[warp][i][g4]) = make_float2(dp_lo, ddp_lo);
                 *reinterpret_cast<float2*>(dps[warp][i][g4 + 8]) = make_float2(dp_hi, ddp_hi);
@@ -454,6 +494,17 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         }
     }
     release_above(-1);
+
+    // the rows' fp16 scale c (a power of two) and 1 / c
+    const int ce_lo = ds_scale_exp(emax_lo), ce_hi = ds_scale_exp(emax_hi);
+    const float cs_lo = exp_to_f(ce_lo), cs_hi = exp_to_f(ce_hi);
+    if constexpr (SV) {
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+            dsa[j][0] = pack_f16(dsb[j][0] * cs_lo, dsb[j][1] * cs_lo);
+            dsa[j][1] = pack_f16(dsb[j][2] * cs_hi, dsb[j][3] * cs_hi);
+        }
+    }
 
     // key rows of an interval: waited for before its first use
     bool ok_k = true;
@@ -509,8 +560,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                     DSg[(size_t)t * s.T + bw + r] = dsv[e];
                 }
             }
-            dsa[j][0] = pack_f16(dsv[0], dsv[1]);
-            dsa[j][1] = pack_f16(dsv[2], dsv[3]);
+            dsa[j][0] = pack_f16(dsv[0] * cs_lo, dsv[1] * cs_lo);
+            dsa[j][1] = pack_f16(dsv[2] * cs_hi, dsv[3] * cs_hi);
         }
     }
     {
@@ -566,8 +617,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 const int ii = i_first + u;
                 const float w = L.act_w[ii], w1 = 1.f - w;
                 const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-                const float dsl = vlo ? psd[0][ii][wrel + g4] : 0.f;
-                const float dsh = vhi ? psd[0][ii][wrel + g4 + 8] : 0.f;
+                const float dsl = vlo ? psd[0][ii][wrel + g4] * cs_lo : 0.f;
+                const float dsh = vhi ? psd[0][ii][wrel + g4 + 8] * cs_hi : 0.f;
                 afr2[u][0] = pack_f16(c0 * dsl, c1 * dsl);
                 afr2[u][1] = 0u;
                 afr2[u][2] = pack_f16(c7 * dsl, 0.f);
@@ -643,9 +694,11 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             }
         }
 
-        // dShat_k as fp16 A fragment: the interpolation weights times dS of the row
-        const unsigned afr[4] = {pack_f16(c0 * ds_lo, c1 * ds_lo), 0u, pack_f16(c7 * ds_lo, 0.f),
-                                 pack_f16(c0 * ds_hi, c1 * ds_hi)};
+        // dShat_k as fp16 A fragment: the interpolation weights times the row's
+        // scaled dS
+        const float dsl = ds_lo * cs_lo, dsh = ds_hi * cs_hi;
+        const unsigned afr[4] = {pack_f16(c0 * dsl, c1 * dsl), 0u, pack_f16(c7 * dsl, 0.f),
+                                 pack_f16(c0 * dsh, c1 * dsh)};
         const int krow = L.act_smem[i] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
@@ -658,7 +711,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 
     // ---- dq = R(-theta pos) scale dq~, rows 0..14 of the tile
     const bool ok = ok_k && ok_v;
-    const float sc = ok ? s.scale : __int_as_float(0x7fc00000);
+    if (!ok) raise_status(a.status, kStatusWaitTimeout);
+    // scale / c of each row (exact: c is a power of two)
+    const float sc_lo = ok ? s.scale * exp_to_f(254 - ce_lo) : __int_as_float(0x7fc00000);
+    const float sc_hi = ok ? s.scale * exp_to_f(254 - ce_hi) : __int_as_float(0x7fc00000);
     __nv_bfloat16* dQ = reinterpret_cast<__nv_bfloat16*>(a.dq) + rowbase * kHeadDim;
     // cos, sin of pair m = 8n + 2c4 + u (m + 32 sits in n-tile n + 4) at qlo,
     // then advanced by 8 positions for qhi with the host's cos, sin(8 theta_m)
@@ -683,6 +739,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         }
         if (!(half ? vhi : vlo)) continue;
         const int q = half ? qhi : qlo;
+        const float sc = half ? sc_hi : sc_lo;
         __nv_bfloat16* row = dQ + (size_t)q * kHeadDim;
 #pragma unroll
         for (int n = 0; n < 4; ++n) {
@@ -747,7 +804,7 @@ cudaError_t launch_bwd_query_mma(const BwdArgs& a, const MmaLayout& L, cudaStrea
         !encode_rows_map(&mt.q, a.q, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 64) ||
         !encode_rows_map(&mt.g, a.dout, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 64) ||
         !encode_rows_map(&mt.o, a.out, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 64) ||
-        !encode_rows_map(&mt.qt, a.qt, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, a.s.T, qheads, 40))
+        !encode_rows_map(&mt.qt, a.qt, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, a.s.T, qheads, 40))
         return cudaErrorInvalidValue;
     const size_t smem = fwd_mma_smem_bytes(L);
     switch (L.nt) {

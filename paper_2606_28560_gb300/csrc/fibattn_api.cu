@@ -14,10 +14,17 @@
 
 #include "../../include/fibattn.h"
 #include "fibattn_internal.cuh"
-#include "fwd_staged.cuh"
 #include "fwd_mma.cuh"
+#include "mma_common.cuh"
 
 using namespace fibattn;
+
+namespace {
+// The device status word that kernels OR kStatus* bits into (one per device:
+// every device that loads the library holds its own copy).  Host code looks
+// up its device address once per device, with that device current.
+__device__ unsigned g_status_word;
+}  // namespace
 
 namespace fibattn {
 bool pdl_enabled() {
@@ -50,7 +57,7 @@ size_t rot_size(int dtype) { return dtype == FIBATTN_BF16 ? 2 : 4; }
 
 struct Resolved {
     float rope_base, scale;
-    int Hkv, dedup, fwd_kernel, bwd_kernel;
+    int Hkv, dedup, round_offsets, fwd_kernel, bwd_kernel;
     void* rotated_k;
     void* residuals;
 };
@@ -60,6 +67,7 @@ int resolve_opts(const fibattn_opts* o, int H, int D, Resolved* r) {
     r->scale = (o && o->scale > 0.f) ? o->scale : (float)(1.0 / std::sqrt((double)D));
     r->Hkv = (o && o->Hkv > 0) ? o->Hkv : H;
     r->dedup = (o && o->no_dedup) ? 0 : 1;
+    r->round_offsets = (o && o->round_offsets) ? 1 : 0;
     r->fwd_kernel = o ? o->fwd_kernel : 0;
     if (r->fwd_kernel < 0 || r->fwd_kernel > 3) return fail(FIBATTN_ERR_INVALID_ARG, "fwd_kernel must be 0, 1, 2 or 3");
     r->bwd_kernel = o ? o->bwd_kernel : 0;
@@ -88,7 +96,10 @@ int check_shape(int B, int H, int T, int D, int W, int K, int dtype) {
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
 // Section 2: d_k = alpha f_k, rounded once to fp32; s0 = floor(d_k), w = d_k - s0.
-int prep_rungs(float alpha, const float* f, int K, int W, int dedup, int T, RungParams* r) {
+// round_offsets: the integer-offset variants of the paper's boolean-mask path
+// (Section 2, "Implementation note"): d_k is then rounded half to even to an
+// integer after the fp32 product, so every rung reads one row (w = 0).
+int prep_rungs(float alpha, const float* f, int K, int W, int dedup, int T, RungParams* r, int round_offsets = 0) {
     if (!(alpha >= 0.5f && alpha <= 1.5f)) return fail(FIBATTN_ERR_INVALID_ARG, "alpha must be in [0.5, 1.5] (got %g)", (double)alpha);
     if (K > 0 && !f) return fail(FIBATTN_ERR_INVALID_ARG, "offsets is NULL");
     std::memset(r, 0, sizeof(*r));
@@ -97,6 +108,7 @@ int prep_rungs(float alpha, const float* f, int K, int W, int dedup, int T, Rung
         if (!std::isfinite(f[k]) || f[k] < 0.f) return fail(FIBATTN_ERR_INVALID_ARG, "offsets[%d] must be finite and >= 0", k);
         volatile float d = alpha * f[k];        // one fp32 rounding
         if (!std::isfinite(d)) return fail(FIBATTN_ERR_INVALID_ARG, "alpha*offsets[%d] overflows", k);
+        if (round_offsets) d = std::nearbyint((float)d);   // to nearest, ties to even (default mode)
         r->f[k] = f[k];
         r->d[k] = d;
         bool reach = d <= (float)(T - 1);       // otherwise masked for every query
@@ -131,7 +143,7 @@ Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
     return s;
 }
 
-// Forward residuals (fibattn_opts.residuals): rotated q (fp16), unnormalised
+// Forward residuals (fibattn_opts.residuals): rotated q (bf16), unnormalised
 // p per slot (slot-major), far-minus-floor rung scores (rung-major), 1 / (row
 // sum) per query.
 struct ResLayout {
@@ -175,6 +187,45 @@ BwdLayout bwd_layout(int B, int H, int Hkv, int T, int W, int K, int dtype, bool
 
 int cuda_fail(cudaError_t e, const char* what) {
     return fail(FIBATTN_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+// Device address of the current device's status word (looked up once per
+// device; no allocation).
+constexpr int kMaxDevices = 256;
+std::mutex g_status_mu;
+unsigned* g_status_addr[kMaxDevices];
+
+int status_word(unsigned** out) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(FIBATTN_ERR_CUDA, "device ordinal %d out of range", dev);
+    std::lock_guard<std::mutex> g(g_status_mu);
+    if (!g_status_addr[dev]) {
+        void* p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_status_word);
+        if (e != cudaSuccess || !p) return cuda_fail(e, "cudaGetSymbolAddress of the status word");
+        g_status_addr[dev] = static_cast<unsigned*>(p);
+    }
+    *out = g_status_addr[dev];
+    return FIBATTN_OK;
+}
+
+// Test hook: one warp arms an mbarrier for 128 bytes that no copy will
+// deliver and waits on it with the library's bounded wait, so the wait runs
+// out after limit_ns and raises kStatusWaitTimeout (nothing is ever written
+// into the barrier's transaction count, so nothing is left in flight).
+__global__ void wait_timeout_probe_kernel(unsigned* status, unsigned long long limit_ns) {
+    __shared__ unsigned long long bar;
+    if (threadIdx.x == 0) {
+        mma::mbar_init(&bar, 1);
+        asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
+    }
+    __syncwarp();
+    if (threadIdx.x == 0) mma::mbar_expect_tx(&bar, 128u);
+    __syncwarp();
+    const bool ok = mma::mbar_wait(&bar, 0, limit_ns);
+    if (!ok && threadIdx.x == 0) raise_status(status, kStatusWaitTimeout);
 }
 
 // Tensor maps are encoded through the driver, which needs a current context,
@@ -285,12 +336,12 @@ size_t fibattn_residual_bytes(int B, int H, int T, int D, int W, int K, int dtyp
     return res_layout(B, H, T, W, K).total;
 }
 
-int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup,
+int fibattn_rung_params(float alpha, const float* offsets, int K, int W, int no_dedup, int round_offsets,
                         float* d, int* s0, float* w, int* active) {
     if (K < 0 || K > kMaxRungs) return fail(FIBATTN_ERR_INVALID_ARG, "K must be in [0, %d]", kMaxRungs);
     if (W < 0) return fail(FIBATTN_ERR_INVALID_ARG, "W must be >= 0");
     RungParams r;
-    int rc = prep_rungs(alpha, offsets, K, W, no_dedup ? 0 : 1, 1 << 30, &r);
+    int rc = prep_rungs(alpha, offsets, K, W, no_dedup ? 0 : 1, 1 << 30, &r, round_offsets);
     if (rc) return rc;
     for (int k = 0; k < K; ++k) {
         if (d) d[k] = r.d[k];
@@ -339,6 +390,18 @@ int fibattn_alpha_schedule(int kind, int L, const float* theta, int stride, floa
     return FIBATTN_OK;
 }
 
+int fibattn_theta_of_alpha(int L, const float* alpha, float* theta) {
+    if (!alpha || !theta || L < 1) return fail(FIBATTN_ERR_INVALID_ARG, "bad arguments to fibattn_theta_of_alpha");
+    for (int l = 0; l < L; ++l) {
+        const double a = alpha[l];
+        if (!(a >= 0.5 && a <= 1.5)) return fail(FIBATTN_ERR_INVALID_ARG, "alpha[%d] = %g is outside [0.5, 1.5]", l, a);
+        // theta = logit(alpha - 0.5); the ends (theta = -/+ infinity) clamp to -/+ 30
+        const double t = (a <= 0.5) ? -30.0 : (a >= 1.5) ? 30.0 : std::log((a - 0.5) / (1.5 - a));
+        theta[l] = (float)std::min(30.0, std::max(-30.0, t));
+    }
+    return FIBATTN_OK;
+}
+
 size_t fibattn_fwd_workspace_bytes(int B, int H, int T, int D, int W, int K, int dtype, const fibattn_opts* opts) {
     Resolved o;
     if (check_shape(B, H, T, D, W, K, dtype) || resolve_opts(opts, H, D, &o)) return 0;
@@ -355,7 +418,7 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     if ((rc = resolve_opts(opts, H, D, &o))) return rc;
     FwdArgs a;
     std::memset(&a, 0, sizeof(a));
-    if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
+    if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r, o.round_offsets))) return rc;
     if (B == 0) return FIBATTN_OK;
     if (!q || !k || !v || !out || !lse || (!workspace && !o.rotated_k))
         return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor or workspace pointer");
@@ -370,16 +433,14 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
     const bool bf16 = dtype == FIBATTN_BF16;
     // bf16 I/O: the tensor-core kernel when its layout applies (W <= 16,
-    // K <= 16, shared memory fits), else the staged CUDA-core kernel, else the
-    // row-gather kernel (also the fp32 I/O path).
+    // K <= 16, shared memory fits), else the row-gather kernel (also the fp32
+    // I/O path).
     const size_t smem_limit = 227 * 1024;
     MmaLayout ML;
-    StageLayout L;
     const bool mma_ok = bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 3) &&
                         build_mma_layout(a.s, a.r, o.rope_base, smem_limit - fwd_mma_static_smem(), &ML);
-    const bool staged_ok = !mma_ok && bf16 && (o.fwd_kernel == 0 || o.fwd_kernel == 2) &&
-                           build_stage_layout(a.s, a.r, o.rope_base, smem_limit, &L);
-    if ((o.fwd_kernel == 3 && !mma_ok) || (o.fwd_kernel == 2 && !staged_ok))
+    if (o.fwd_kernel == 2) return fail(FIBATTN_ERR_UNSUPPORTED, "fwd_kernel 2 is not built");
+    if (o.fwd_kernel == 3 && !mma_ok)
         return fail(FIBATTN_ERR_UNSUPPORTED, "requested forward kernel does not apply to these arguments "
                                              "(bf16 I/O, W <= 16, K <= 16, shared-memory layout)");
     if (o.residuals) {
@@ -395,18 +456,16 @@ int fibattn_fwd(const void* q, const void* k, const void* v, void* out, float* l
     }
     a.S = W + 1 + K;
     if ((rc = bind_context())) return rc;
+    if ((rc = status_word(&a.status))) return rc;
     cudaError_t e;
     {
         ProfScope p("rope_k", st);
-        e = launch_rope_rows(k, kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+        e = launch_rope_rows(k, kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st, a.status);
     }
     if (e != cudaSuccess) return cuda_fail(e, "rope prologue launch");
     if (mma_ok) {
         ProfScope p("fwd", st);
         e = launch_fwd_mma(a, ML, st);
-    } else if (staged_ok) {
-        ProfScope p("fwd", st);
-        e = launch_fwd_staged(a, L, bf16, st);
     } else {
         ProfScope p("fwd", st);
         e = launch_fwd_simple(a, bf16, st);
@@ -431,7 +490,9 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     if ((rc = resolve_opts(opts, H, D, &o))) return rc;
     BwdArgs a;
     std::memset(&a, 0, sizeof(a));
-    if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r))) return rc;
+    if ((rc = prep_rungs(alpha, offsets, K, W, o.dedup, T, &a.r, o.round_offsets))) return rc;
+    if (o.round_offsets && (dtheta || dd))
+        return fail(FIBATTN_ERR_INVALID_ARG, "rounded rung distances do not vary with alpha: pass dtheta = dd = NULL");
     if (!workspace) return fail(FIBATTN_ERR_INVALID_ARG, "workspace is NULL");
     if (B > 0 && (!q || (!k && !o.rotated_k) || !v || !lse || !dout || !dq || !dk || !dv))
         return fail(FIBATTN_ERR_INVALID_ARG, "NULL tensor pointer");
@@ -479,15 +540,16 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
     }
     cudaError_t e;
     if ((rc = bind_context())) return rc;
+    if ((rc = status_word(&a.status))) return rc;
     if (B > 0) {
         if (!mma_ok) {
             ProfScope p("rope_q", st);
-            e = launch_rope_rows(q, a.qt, (long long)B * H * T, T, a.rope, bf16, st);
+            e = launch_rope_rows(q, a.qt, (long long)B * H * T, T, a.rope, bf16, st, a.status);
             if (e != cudaSuccess) return cuda_fail(e, "rope prologue (q) launch");
         }
         if (!o.rotated_k) {                      // else the rotated keys come from the forward
             ProfScope p("rope_k", st);
-            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st);
+            e = launch_rope_rows(k, a.kt, (long long)B * o.Hkv * T, T, a.rope, bf16, st, a.status);
             if (e != cudaSuccess) return cuda_fail(e, "rope prologue (k) launch");
         }
         if (mma_ok) {
@@ -514,6 +576,43 @@ int fibattn_bwd(const void* q, const void* k, const void* v, const void* out, co
         return FIBATTN_OK;
     }
     return FIBATTN_OK;                           // dtheta and dd: written by block 0 of the key pass
+}
+
+int fibattn_check_status(void* stream, unsigned* flags) {
+    if (flags) *flags = 0u;
+    int rc = bind_context();
+    if (rc) return rc;
+    unsigned* word = nullptr;
+    if ((rc = status_word(&word))) return rc;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    unsigned h = 0u;
+    cudaError_t e = cudaMemcpyAsync(&h, word, sizeof(h), cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e == cudaSuccess && h) e = cudaMemsetAsync(word, 0, sizeof(unsigned), st);
+    if (e == cudaSuccess && h) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the device status word");
+    if (flags) *flags = h;
+    if (h & kStatusWaitTimeout)
+        return fail(FIBATTN_ERR_INTERNAL, "a kernel gave up waiting for a staging copy (outputs of the affected "
+                                          "tiles are NaN)%s", (h & kStatusRange) ? "; a rotated q or k row also "
+                                          "overflowed fp16" : "");
+    if (h & kStatusRange)
+        return fail(FIBATTN_ERR_RANGE, "a RoPE-rotated q or k entry reached 65520 in magnitude, beyond the fp16 "
+                                       "rows of the bf16 path (scores with such operands are not meaningful)");
+    return FIBATTN_OK;
+}
+
+int fibattn_test_wait_timeout(unsigned timeout_us, void* stream) {
+    if (timeout_us == 0u || timeout_us > 10000000u)
+        return fail(FIBATTN_ERR_INVALID_ARG, "timeout_us must be in [1, 1e7]");
+    int rc = bind_context();
+    if (rc) return rc;
+    unsigned* word = nullptr;
+    if ((rc = status_word(&word))) return rc;
+    cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    wait_timeout_probe_kernel<<<1, 32, 0, st>>>(word, (unsigned long long)timeout_us * 1000ull);
+    cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? FIBATTN_OK : cuda_fail(e, "wait-timeout probe launch");
 }
 
 int fibattn_staging_layout(int kind, int T, int W, float alpha, const float* offsets, int K, int no_dedup,

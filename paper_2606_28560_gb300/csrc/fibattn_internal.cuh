@@ -39,6 +39,14 @@ struct Shape {
     float scale;              // score scale (1/sqrt(D) by default)
 };
 
+// Device status word (one per device, read and cleared by
+// fibattn_check_status): kernels OR these bits into it.
+constexpr unsigned kStatusWaitTimeout = 1u;   // a bounded wait on a staging copy ran out
+constexpr unsigned kStatusRange = 2u;         // a rotated row overflowed its fp16 storage
+__device__ __forceinline__ void raise_status(unsigned* st, unsigned bits) {
+    if (st) atomicOr(st, bits);
+}
+
 struct FwdArgs {
     const void* q;            // [B,H,T,D]
     const void* kt;           // rotated keys [B,Hkv,T,D] (workspace)
@@ -50,10 +58,11 @@ struct FwdArgs {
     // nullptr when not asked for): the rotated queries, the unnormalised
     // probability exp(s - max) of every slot (0 where not attended), the
     // far-minus-floor raw score of every rung row and 1 / (row sum) per query.
-    void* res_qt;             // fp16 [B,H,T,D]
+    void* res_qt;             // bf16 [B,H,T,D]
     float* res_P;             // slot-major [B,H,S,T], S = W + 1 + K
     float* res_sd;            // rung-major [B,H,K,T]
     float* res_il;            // [B,H,T]
+    unsigned* status;         // device status word
     int S;
     Shape s;
     RungParams r;
@@ -74,7 +83,7 @@ struct BwdArgs {
     int want_dd;              // compute dL/dd_k (dtheta or dd requested)
     float* dd;                // device [K] or nullptr
     // workspace views
-    void* qt;                 // rotated q [B,H,T,D]
+    void* qt;                 // rotated q [B,H,T,D] (bf16 from the tensor-core query pass, fp16 from the prologue)
     void* kt;                 // rotated k [B,Hkv,T,D]
     float* P;                 // softmax probabilities [B,H,T,S]
     float* DP;                // dL/dp = dO . val per slot [B,H,T,S]
@@ -86,6 +95,7 @@ struct BwdArgs {
     const float* res_sd;      // forward residual far-minus-floor rung scores [B,H,K,T], or nullptr;
                               // when the forward residuals are used, Ps and qt point into them
     int saved;                // tensor-core passes read p (Ps, unnormalised), sd and q~ (qt) from the forward residuals
+    unsigned* status;         // device status word
     int nblk_q;               // query-pass blocks
     int S;                    // slots per query = W + 1 + K
     float alpha;
@@ -288,7 +298,7 @@ cudaError_t launch_kernel(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t 
 // ----------------------------------------------------------- launchers ----
 
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
-                             bool bf16, cudaStream_t st);
+                             bool bf16, cudaStream_t st, unsigned* status);
 cudaError_t launch_fwd_simple(const FwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_query(const BwdArgs& a, bool bf16, cudaStream_t st);
 cudaError_t launch_bwd_key(const BwdArgs& a, bool bf16, cudaStream_t st);

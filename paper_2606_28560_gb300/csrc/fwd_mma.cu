@@ -126,7 +126,9 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 
     // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32)
     // Thread dims: 16kc + 2c4 + {0,1} and 16kc + 8 + 2c4 + {0,1} for kc = 0..3.
-    unsigned qa[4][4];
+    // SAVE: also as bf16 (qs), the residual the key pass reads.
+    unsigned qa[4][4], qs[SAVE ? 4 : 1][4];
+    float qmax = 0.f;                             // largest |q~| of the thread: fp16 holds < 65520
     {
         if (TEAMS == 2) load_q(bh);
         // cos/sin of the 8 pairs at position bw+g4, then advanced by 8 positions
@@ -169,15 +171,21 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
                     const float xa = x[kc][j], xb = x[kc + 2][j];
                     x[kc][j] = xa * cs[kc][j] - xb * sn[kc][j];
                     x[kc + 2][j] = xb * cs[kc][j] + xa * sn[kc][j];
+                    qmax = fmaxf(qmax, fmaxf(fabsf(x[kc][j]), fabsf(x[kc + 2][j])));
                 }
             }
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
                 qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);       // a0 / a1: k = 2c4, 2c4+1
                 qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);   // a2 / a3: k = 2c4+8, 2c4+9
+                if constexpr (SAVE) {
+                    qs[kc][half] = pack_bf16(x[kc][0], x[kc][1]);
+                    qs[kc][2 + half] = pack_bf16(x[kc][2], x[kc][3]);
+                }
             }
         }
     }
+    if (qmax >= 65520.f) raise_status(a.status, kStatusRange);
     const float sc2 = s.scale * kLog2e;           // scores in log2 units
     const int qlo = bw + g4, qhi = bw + g4 + 8;   // absolute queries of this thread's rows
     const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
@@ -188,13 +196,13 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         // (16-byte chunk c of row r at chunk c ^ r) and out as runs of rows
         static_assert(TEAMS == 1, "the residuals are written by the one-head form");
         unsigned* stage = ostage[warp];
-        __half* QT = reinterpret_cast<__half*>(a.res_qt) + rowbase * kHeadDim;
+        __nv_bfloat16* QT = reinterpret_cast<__nv_bfloat16*>(a.res_qt) + rowbase * kHeadDim;
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
-                stage[g4 * 32 + (((2 * kc) ^ g4) << 2) + c4] = qa[kc][half];
-                stage[g4 * 32 + (((2 * kc + 1) ^ g4) << 2) + c4] = qa[kc][2 + half];
+                stage[g4 * 32 + (((2 * kc) ^ g4) << 2) + c4] = qs[kc][half];
+                stage[g4 * 32 + (((2 * kc + 1) ^ g4) << 2) + c4] = qs[kc][2 + half];
             }
             __syncwarp();
             const int nrow = min(half ? kRowsPerWarp - 8 : 8, s.T - (bw + 8 * half));
@@ -420,6 +428,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 
     // ---- normalise and store rows 0..14 of the tile
     const bool ok = ok_k && ok_v;
+    if (!ok) raise_status(a.status, kStatusWaitTimeout);
     const float inv_lo = ok ? 1.f / llo : __int_as_float(0x7fc00000);
     const float inv_hi = ok ? 1.f / lhi : __int_as_float(0x7fc00000);
     // Rows g4 (half 0) and g4 + 8 (half 1) leave through this warp's stage, 8
@@ -460,13 +469,14 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
                     pack_bf16(o[n][2 * half] * inv, o[n][2 * half + 1] * inv);
         }
     }
+    // (a timed-out wait leaves NaN in lse and 1 / row sum too)
     if (c4 == 0 && vlo) {
-        a.lse[(size_t)bh * s.T + qlo] = (mlo + __log2f(llo)) * kLn2;
-        if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qlo] = 1.f / llo;
+        a.lse[(size_t)bh * s.T + qlo] = ok ? (mlo + __log2f(llo)) * kLn2 : inv_lo;
+        if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qlo] = inv_lo;
     }
     if (c4 == 0 && vhi) {
-        a.lse[(size_t)bh * s.T + qhi] = (mhi + __log2f(lhi)) * kLn2;
-        if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qhi] = 1.f / lhi;
+        a.lse[(size_t)bh * s.T + qhi] = ok ? (mhi + __log2f(lhi)) * kLn2 : inv_hi;
+        if constexpr (SAVE) a.res_il[(size_t)bh * s.T + qhi] = inv_hi;
     }
     }                                             // query heads of the group
 }

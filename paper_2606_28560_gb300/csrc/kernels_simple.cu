@@ -76,8 +76,9 @@ __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ sr
 constexpr int kRopeHeads = 4;
 __global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16* __restrict__ src,
                                                              __half* __restrict__ dst, int heads, int T_,
-                                                             RopeParams rp) {
+                                                             RopeParams rp, unsigned* status) {
     grid_dependency_sync();
+    float rmax = 0.f;                             // largest |rotated entry|: fp16 holds < 65520
     const int groups = (heads + kRopeHeads - 1) / kRopeHeads;
     const long long n = (long long)groups * T_ * 4;
     for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
@@ -108,8 +109,11 @@ __global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16
                 const float a0 = __uint_as_float(wa[e] << 16), a1 = __uint_as_float(wa[e] & 0xffff0000u);
                 const float b0 = __uint_as_float(wb[e] << 16), b1 = __uint_as_float(wb[e] & 0xffff0000u);
                 const int m0 = 2 * e, m1 = 2 * e + 1;        // pairs (8c + m, 32 + 8c + m)
-                __half2 ra = __floats2half2_rn(a0 * cs[m0] - b0 * sn[m0], a1 * cs[m1] - b1 * sn[m1]);
-                __half2 rb = __floats2half2_rn(b0 * cs[m0] + a0 * sn[m0], b1 * cs[m1] + a1 * sn[m1]);
+                const float xa0 = a0 * cs[m0] - b0 * sn[m0], xa1 = a1 * cs[m1] - b1 * sn[m1];
+                const float xb0 = b0 * cs[m0] + a0 * sn[m0], xb1 = b1 * cs[m1] + a1 * sn[m1];
+                rmax = fmaxf(rmax, fmaxf(fmaxf(fabsf(xa0), fabsf(xa1)), fmaxf(fabsf(xb0), fabsf(xb1))));
+                __half2 ra = __floats2half2_rn(xa0, xa1);
+                __half2 rb = __floats2half2_rn(xb0, xb1);
                 oa[e] = *reinterpret_cast<unsigned*>(&ra);
                 ob[e] = *reinterpret_cast<unsigned*>(&rb);
             }
@@ -118,6 +122,7 @@ __global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16
             *reinterpret_cast<uint4*>(row + kHalf + 8 * c) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
         }
     }
+    if (rmax >= 65520.f) raise_status(status, kStatusRange);
 }
 
 // ------------------------------------------------------------- forward ----
@@ -446,7 +451,7 @@ __global__ void __launch_bounds__(kThreads) bwd_key_kernel(BwdArgs a) {
 }  // namespace
 
 cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, const RopeParams& rp,
-                             bool bf16, cudaStream_t st) {
+                             bool bf16, cudaStream_t st, unsigned* status) {
     if (rows <= 0) return cudaSuccess;
     const long long items = rows * 4;
     long long grid = (items + 255) / 256;
@@ -472,7 +477,7 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
         if (g2 > wave) g2 = wave;
         return launch_kernel(rope_rows_bf16_kernel, dim3((unsigned)g2), dim3(256), 0, st,
                              reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), heads, T,
-                             rp);
+                             rp, status);
     }
     return launch_kernel(rope_rows_kernel<float, float>, dim3((unsigned)grid), dim3(256), 0, st,
                          reinterpret_cast<const float*>(src), reinterpret_cast<float*>(dst), rows, T, rp);

@@ -12,7 +12,9 @@
 namespace fibattn {
 namespace mma {
 
-constexpr unsigned kWaitLimit = 1u << 26;        // mbarrier polls before giving up
+// A wait on a staging copy gives up after this long (the copies are of at
+// most a few hundred KB from L2 or HBM and land within microseconds).
+constexpr unsigned long long kWaitLimitNs = 1000000000ull;   // 1 s
 
 __device__ __forceinline__ unsigned smem_u32(const void* p) { return (unsigned)__cvta_generic_to_shared(p); }
 
@@ -28,16 +30,31 @@ __device__ __forceinline__ void mbar_init(unsigned long long* bar, unsigned coun
 __device__ __forceinline__ void mbar_expect_tx(unsigned long long* bar, unsigned bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;\n" :: "r"(smem_u32(bar)), "r"(bytes));
 }
-// Bounded wait on phase `parity`; returns false after kWaitLimit polls.
-__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity) {
+__device__ __forceinline__ unsigned long long global_ns() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;\n" : "=l"(t));
+    return t;
+}
+
+// Bounded wait on phase `parity`: false once limit_ns of the global timer
+// have passed since the first poll that did not find the phase complete (the
+// timer is read every 64 polls).  The caller poisons its outputs and raises
+// kStatusWaitTimeout; nothing hangs.
+__device__ __forceinline__ bool mbar_wait(unsigned long long* bar, unsigned parity,
+                                          unsigned long long limit_ns = kWaitLimitNs) {
     const unsigned a = smem_u32(bar);
-    for (unsigned it = 0; it < kWaitLimit; ++it) {
+    unsigned long long t0 = 0;
+    for (unsigned it = 0;; ++it) {
         unsigned done;
         asm volatile("{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
                      " selp.u32 %0, 1, 0, p;\n}\n" : "=r"(done) : "r"(a), "r"(parity) : "memory");
         if (done) return true;
+        if ((it & 63u) == 0u) {
+            const unsigned long long now = global_ns();
+            if (it == 0) t0 = now;
+            else if (now - t0 > limit_ns) return false;
+        }
     }
-    return false;
 }
 __device__ __forceinline__ void tma_load_3d(void* dst, const CUtensorMap* map, int x, int y, int z,
                                             unsigned long long* bar) {

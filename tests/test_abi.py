@@ -4,6 +4,7 @@ definitions, and bad arguments are rejected before anything is launched."""
 from __future__ import annotations
 
 import ctypes
+import math
 import os
 import re
 
@@ -63,6 +64,36 @@ def test_rung_params_match_oracle(alpha, W):
     np.testing.assert_array_equal(p["active"], d > W)
     p2 = fa.rung_params(np.float32(alpha), f, W, dedup=False)
     assert p2["active"].all()
+    # the integer-offset variants: rounded to the nearest integer, ties to even
+    p3 = fa.rung_params(np.float32(alpha), f, W, round_offsets=True)
+    dr = O.offsets_rounded(float(np.float32(alpha)), f)
+    np.testing.assert_array_equal(p3["d"].astype(np.float64), dr)
+    np.testing.assert_array_equal(p3["s0"], dr.astype(np.int32))
+    assert not p3["w"].any()
+    np.testing.assert_array_equal(p3["active"], dr > W)
+
+
+def test_rounded_offsets_reject_rung_gradients():
+    """Rounded distances do not vary with alpha: the backward refuses dtheta/dd."""
+    lib = B.lib()
+    o = B._opts(round_offsets=True)
+    f = np.array([1, 2, 3], dtype=np.float32)
+    rc = lib.fibattn_bwd(16, 16, 16, None, 16, 16, 16, 16, 16, 16, None, 1, 2, 8, 64, 2, 1.0, B._fptr(f), 3, 0,
+                         ctypes.byref(o), 16, 1 << 30, None)
+    assert rc == 1 and "dtheta" in lib.fibattn_last_error().decode()
+
+
+def test_theta_alpha_maps_are_stable_and_inverse():
+    """alpha = 0.5 + sigmoid(theta) stays finite at extreme theta; the inverse
+    map clamps the ends and inverts the interior."""
+    a = fa.alpha_schedule("learned", 4, theta=[-1000.0, 1000.0, 0.0, 2.0])
+    assert a[0] == 0.5 and a[1] == 1.5 and a[2] == 1.0
+    assert abs(a[3] - (0.5 + 1 / (1 + math.exp(-2.0)))) < 1e-6
+    assert fa.alpha_of_theta(-1000.0) == 0.5 and fa.alpha_of_theta(1000.0) == 1.5
+    t = fa.theta_of_alpha_array([0.5, 1.5, 1.0, 0.8, 1.3])
+    assert t[0] == -30.0 and t[1] == 30.0 and t[2] == 0.0
+    back = fa.alpha_schedule("learned", 2, theta=t[3:])
+    np.testing.assert_allclose(back, [0.8, 1.3], rtol=0, atol=2e-7)
 
 
 def _call_fwd(**kw):
@@ -71,7 +102,7 @@ def _call_fwd(**kw):
                 K=3, dtype=0, ws=16, wsb=1 << 30, Hkv=0, rope_base=0.0, rk=None, res=None, fk=0)
     args.update(kw)
     f = np.array([1, 2, 3] + [5] * 40, dtype=np.float32)
-    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, args["fk"], 0, args["rk"], args["res"])
+    o = B.Opts(args["rope_base"], 0.0, args["Hkv"], 0, args["fk"], 0, args["rk"], args["res"], 0)
     rc = lib.fibattn_fwd(args["q"], args["k"], args["v"], args["out"], args["lse"], args["B"], args["H"],
                          args["T"], args["D"], args["W"], args["alpha"], B._fptr(f), args["K"], args["dtype"],
                          ctypes.byref(o), args["ws"], args["wsb"], None)

@@ -17,10 +17,13 @@ from paper_2606_28560_gb300 import inputs
 
 
 def test_alpha_theta_maps():
+    # both maps run in the library on fp32 host values: the round trip is
+    # exact to fp32 rounding of alpha over the sigmoid's slope (at most ~5e-6
+    # in theta at |theta| = 3)
     for th in (-3.0, -0.4, 0.0, 0.7, 2.5):
         a = fa.alpha_of_theta(th)
         assert 0.5 < a < 1.5
-        assert abs(fa.theta_of_alpha(a) - th) < 1e-9
+        assert abs(fa.theta_of_alpha(a) - th) < 3e-5
     assert fa.alpha_of_theta(0.0) == 1.0
     # the schedule of the library's learned kind is the same map
     th = [0.3, -1.2, 0.0]

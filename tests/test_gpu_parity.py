@@ -144,11 +144,10 @@ def _random_cases(n=16, seed=2606):
     return cases
 
 
-FWD_KERNELS = [(torch.float32, "auto"), (torch.bfloat16, "gather"), (torch.bfloat16, "staged"),
-               (torch.bfloat16, "mma")]
+FWD_KERNELS = [(torch.float32, "auto"), (torch.bfloat16, "gather"), (torch.bfloat16, "mma")]
 
 
-@pytest.mark.parametrize("dtype,kernel", FWD_KERNELS, ids=["f32", "bf16-gather", "bf16-staged", "bf16-mma"])
+@pytest.mark.parametrize("dtype,kernel", FWD_KERNELS, ids=["f32", "bf16-gather", "bf16-mma"])
 @pytest.mark.parametrize("case", SMALL, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]}{c[6]}{c[7]}d{int(c[8])}"
                                               for c in SMALL])
 def test_forward_small(case, dtype, kernel):
@@ -259,8 +258,6 @@ def test_config2_bf16_linear_stagger(W):
     for layer in (0, 7, 15):
         q, k, v = inputs.qkv(16, 8, 1024, seed=inputs.layer_seed(1, layer), dtype=torch.bfloat16)
         check_fwd(q, k, v, float(alphas[layer]), f, W)
-        if layer == 7:
-            check_fwd(q, k, v, float(alphas[layer]), f, W, kernel="staged")
 
 
 def test_config3_bf16_extrapolation_coprime():
@@ -304,10 +301,10 @@ def test_gqa_paper_shape_fwd_bwd():
 @pytest.mark.parametrize("base,K", [("fib", 15), ("pow2", 10)])
 def test_config5_bf16_long_stress(base, K):
     """B=2 H=8 T=16384 W=12, linear stagger, Fibonacci vs power-of-2 base:
-    fwd+bwd of layers 0 and 15 in full."""
+    fwd+bwd of layers 0, 7 (mid-ramp, alpha 0.9667) and 15 in full."""
     alphas = fa.alpha_schedule("linear", 16)
     f = _offsets(base, K)
-    for layer in (0, 15):
+    for layer in (0, 7, 15):
         s = inputs.layer_seed(4, layer)
         q, k, v = inputs.qkv(2, 8, 16384, seed=s, dtype=torch.bfloat16)
         g = inputs.dout(2, 8, 16384, seed=s, dtype=torch.bfloat16)
@@ -318,7 +315,7 @@ def test_config5_bf16_long_stress(base, K):
 RANDOM = _random_cases(n=8, seed=1404)
 
 
-@pytest.mark.parametrize("dtype,kernel", FWD_KERNELS, ids=["f32", "bf16-gather", "bf16-staged", "bf16-mma"])
+@pytest.mark.parametrize("dtype,kernel", FWD_KERNELS, ids=["f32", "bf16-gather", "bf16-mma"])
 @pytest.mark.parametrize("case", RANDOM, ids=[f"B{c[0]}H{c[1]}kv{c[2]}T{c[3]}W{c[4]}a{c[5]:.4f}{c[6]}{c[7]}d{int(c[8])}"
                                               for c in RANDOM])
 def test_forward_random_shapes(case, dtype, kernel):
@@ -347,3 +344,56 @@ def test_backward_random_shapes(case, dtype, kernel):
         if e.status == 2:
             pytest.skip(str(e))
         raise
+
+
+# ------------------------------------------ rounded (integer) rung offsets --
+
+def check_rounded(q, k, v, dout, alpha, f, W, kernel="auto", residuals=False):
+    """The integer-offset variant (round_offsets): forward and backward (no
+    rung gradient: the rounded distances do not vary with alpha) against the
+    oracle on the rounded distances."""
+    qc, kc, vc, gc = q.cuda(), k.cuda(), v.cuda(), dout.cuda()
+    kw = dict(round_offsets=True)
+    if residuals:
+        kw.update(rotated_k=fa.rotated_k_like(kc), residuals=fa.residuals_like(qc, W, len(f)))
+    out, lse = fa.fwd(qc, kc, vc, alpha, f, W, kernel="auto" if kernel != "gather" else "gather", **kw)
+    dq, dk, dv, dth, dd = fa.bwd(qc, kc, vc, lse, gc, alpha, f, W, out=None if kernel == "gather" else out,
+                                 kernel=kernel, rung_grads=False, **kw)
+    torch.cuda.synchronize()
+    d = O.offsets_rounded(float(np.float32(alpha)), f.astype(np.float64))
+    ro, rl = O.forward(_f64(q), _f64(k), _f64(v), W, d, nthreads=NTHREADS)
+    rq, rk, rv, _ = O.backward(_f64(q), _f64(k), _f64(v), _f64(dout), W, d, nthreads=NTHREADS)
+    tol = TOL[q.dtype]
+    diff = np.abs(_f64(out) - ro)
+    if q.dtype == torch.bfloat16:
+        assert not (diff > bf16_out_tol(ro)).any(), f"out err {diff.max()}"
+    else:
+        assert diff.max() <= tol["out"]
+    assert float(np.max(np.abs(_f64(lse) - rl))) <= tol["lse"]
+    for name, g, r in (("dq", dq, rq), ("dk", dk, rk), ("dv", dv, rv)):
+        e = _rel(_f64(g), r)
+        assert e <= tol["grad"], f"{name} rel err {e}"
+    assert dth is None and dd is None
+
+
+@pytest.mark.parametrize("kernel,dtype,residuals", [("mma", torch.bfloat16, False), ("mma", torch.bfloat16, True),
+                                                    ("gather", torch.bfloat16, False),
+                                                    ("gather", torch.float32, False)],
+                         ids=["bf16-mma", "bf16-residuals", "bf16-gather", "f32"])
+@pytest.mark.parametrize("kind,layer", [("linear", 5), ("linear", 12), ("coprime", 3)])
+def test_rounded_stagger_small(kind, layer, kernel, dtype, residuals):
+    alpha = float(fa.alpha_schedule(kind, 16)[layer])
+    q, k, v = inputs.qkv(2, 4, 533, seed=layer + 90, dtype=dtype, Hkv=2)
+    g = inputs.dout(2, 4, 533, seed=layer + 91, dtype=dtype)
+    check_rounded(q, k, v, g, alpha, _offsets("fib", 15), 8, kernel, residuals)
+
+
+def test_config2_rounded_linear_layer():
+    """Config 2's shape (B=16 H=8 T=1024 W=8) at layer 7 of the linear stagger
+    (alpha 0.9667) with the rung distances rounded: every output, and the
+    training path's gradients."""
+    alpha = float(fa.alpha_schedule("linear", 16)[7])
+    s = inputs.layer_seed(1, 7)
+    q, k, v = inputs.qkv(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+    g = inputs.dout(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+    check_rounded(q, k, v, g, alpha, _offsets("fib", 15), 8, "mma", residuals=True)

@@ -6,8 +6,9 @@ scores.
 Bars:
 - out, lse of a forward that writes residuals: bit-identical to the forward
   without them (the same arithmetic; the residuals are extra stores).
-- rotated q (fp16): |q~ - ref| <= 2^-11 |ref| + 1e-5 -- fp16 round-to-nearest
-  of a value whose fp32 rotation is accurate to ~1e-6 relative.
+- rotated q (bf16): |q~ - ref| <= 2^-8 |ref| + 1e-5 -- bf16 round-to-nearest
+  (8 significant bits) of a value whose fp32 rotation is accurate to ~1e-6
+  relative.
 - p per slot, the stored weight times the stored 1 / (weight sum):
   |p - ref| <= 1e-2, the bf16 output bar (p is in [0, 1]; the scores come
   from fp16 operands); the row's p sum to 1 within 1e-2 (the forward's sum
@@ -68,7 +69,7 @@ def test_residuals_of_the_forward(case):
             qr = rope_complex_np(qf[b, h])
             kr = rope_complex_np(kf[b, hk])
             got = qt[b, h].to(torch.float64).numpy()
-            assert np.all(np.abs(got - qr) <= 2.0 ** -11 * np.abs(qr) + 1e-5)
+            assert np.all(np.abs(got - qr) <= 2.0 ** -8 * np.abs(qr) + 1e-5)
             # every query up to 64 of them, the tail included
             idx = np.unique(np.concatenate([np.arange(min(T, 24)), np.arange(max(0, T - 24), T),
                                             rng.integers(0, T, size=16)]))
@@ -242,3 +243,31 @@ def test_random_shapes_forward_and_backward_from_residuals(case):
     ro, _ = O.forward(_f64(q), _f64(k), _f64(v), W, d, dedup=dedup, nthreads=NTHREADS)
     assert not (np.abs(_f64(out) - ro) > bf16_out_tol(ro)).any()
     _check_bwd_residuals(q, k, v, g, alpha, f, W, dedup)
+
+
+@pytest.mark.parametrize("layer", [0, 7, 12, 15])
+def test_config4_training_path_full(layer):
+    """Config 4 (B=16 H=8 T=1024 W=8, learned theta seed 3) through the path the
+    benchmark times: the forward keeps its rotated keys and residuals, the
+    backward reads them.  Every output and gradient of the layer against the
+    oracle; layer 12 (alpha 0.8801671) is the layer whose staged slab once sat
+    in the rounding padding of the interval before it."""
+    theta = inputs.theta_learned(16, seed=3)
+    alpha = float(fa.alpha_schedule("learned", 16, theta=theta)[layer])
+    s = inputs.layer_seed(3, layer)
+    q, k, v = inputs.qkv(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+    g = inputs.dout(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+    f = fa.base("fib", 15)
+    qc, kc, vc = q.cuda(), k.cuda(), v.cuda()
+    res = fa.residuals_like(qc, 8, 15)
+    rk = fa.rotated_k_like(kc)
+    out, lse = fa.fwd(qc, kc, vc, alpha, f, 8, residuals=res, rotated_k=rk)
+    torch.cuda.synchronize()
+    a32 = float(np.float32(alpha))
+    d = O.offsets_fp32(a32, f.astype(np.float64))
+    ro, rl = O.forward(_f64(q), _f64(k), _f64(v), 8, d, nthreads=NTHREADS)
+    diff = np.abs(_f64(out) - ro)
+    from tests.test_gpu_parity import bf16_out_tol
+    assert not (diff > bf16_out_tol(ro)).any(), f"out err {diff.max()}"
+    assert float(np.max(np.abs(_f64(lse) - rl))) <= 1e-2
+    _check_bwd_residuals(q, k, v, g, alpha, f, 8)

@@ -369,3 +369,40 @@ def test_oracle_threads_agree():
     gb = O.backward(q, k, v, g, W, d, nthreads=4)
     for x, y in zip(ga, gb):
         np.testing.assert_array_equal(x, y)
+
+
+# ---------------------------------- rounded offsets: the boolean-mask path --
+
+def _rounded_independently(alpha, f):
+    """Integer distances by another route than the oracle's: Python's round()
+    (ties to even) of the fp32 product."""
+    return [round(float(np.float32(np.float32(alpha) * np.float32(x)))) for x in f]
+
+
+def test_rounded_offsets_ties_to_even():
+    f = O.fib_base(15)
+    # alpha 0.5: 0.5 -> 0, 1.5 -> 2, 2.5 -> 2, 6.5 -> 6, 10.5 -> 10, 27.5 -> 28, 44.5 -> 44
+    d = O.offsets_rounded(0.5, f)
+    assert list(d[:11]) == [0, 1, 2, 2, 4, 6, 10, 17, 28, 44, 72]
+    for alpha in (0.5, 0.7333333, 1.0, 1.1, 1.5):
+        assert list(O.offsets_rounded(alpha, f)) == _rounded_independently(alpha, f)
+
+
+@pytest.mark.parametrize("kind,layers", [("linear", (1, 5, 11, 14)), ("coprime", (1, 3, 9))])
+@pytest.mark.parametrize("T,W", [(64, 8), (200, 6), (300, 12)])
+def test_rounded_stagger_equals_boolean_mask_attention(kind, layers, T, W):
+    """The rounded linear and coprime staggers are integer gathers: the oracle
+    on the rounded distances equals dense attention with the boolean mask of
+    those integer distances (Section 2, "Implementation note": numerically
+    identical), in dedup mode (the attended set is a union)."""
+    D = 16
+    f = O.fib_base(15)
+    alphas = O.alpha_schedule(kind, 16)
+    for l in layers:
+        q, k, v = _rand((1, 2, T, D), 100 + l), _rand((1, 2, T, D), 200 + l), _rand((1, 2, T, D), 300 + l)
+        d = O.offsets_rounded(float(alphas[l]), f)
+        o, lse = O.forward(q, k, v, W, d)
+        o2, lse2 = masked_attention_np(q, k, v, bool_mask(T, W, _rounded_independently(float(alphas[l]), f)),
+                                       1 / math.sqrt(D))
+        np.testing.assert_allclose(o, o2, rtol=0, atol=1e-12)
+        np.testing.assert_allclose(lse, lse2, rtol=0, atol=1e-12)
