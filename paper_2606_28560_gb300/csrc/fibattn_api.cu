@@ -140,6 +140,10 @@ void prep_rope(float base, RopeParams* rp) {
 Shape make_shape(int B, int H, int T, int W, const Resolved& o) {
     Shape s;
     s.B = B; s.H = H; s.Hkv = o.Hkv; s.T = T; s.W = W; s.G = H / o.Hkv; s.scale = o.scale;
+    s.dH = FastDiv::make((unsigned)H);
+    s.dHkv = FastDiv::make((unsigned)o.Hkv);
+    s.dG = FastDiv::make((unsigned)s.G);
+    s.dTiles = FastDiv::make((unsigned)((T + kMmaTile - 1) / kMmaTile));
     return s;
 }
 

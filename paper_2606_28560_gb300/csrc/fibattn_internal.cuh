@@ -34,9 +34,33 @@ struct RopeParams {
     unsigned long long F[kHalf];
 };
 
+// Division by a divisor fixed at launch, for numerators below 2^31: the
+// quotient is (umulhi(n, mul) + n) >> shift with shift = ceil(log2 d) and
+// mul = floor(2^32 (2^shift - d) / d) + 1 (the round-up multiplier method).
+struct FastDiv {
+    unsigned d, mul, shift;
+#ifdef __CUDACC__
+    __host__ __device__
+#endif
+    static FastDiv make(unsigned d) {
+        FastDiv f;
+        f.d = d;
+        f.shift = 0;
+        while ((1ull << f.shift) < d) ++f.shift;
+        f.mul = (unsigned)(((1ull << 32) * ((1ull << f.shift) - d)) / d + 1);
+        return f;
+    }
+};
+#ifdef __CUDACC__
+__device__ __forceinline__ unsigned fdiv(unsigned n, const FastDiv& f) {
+    return (__umulhi(n, f.mul) + n) >> f.shift;
+}
+#endif
+
 struct Shape {
     int B, H, Hkv, T, W, G;   // G = H / Hkv
     float scale;              // score scale (1/sqrt(D) by default)
+    FastDiv dH, dHkv, dG, dTiles;   // by H, Hkv, G and the tensor-core tiles per head
 };
 
 // Device status word (one per device, read and cleared by

@@ -76,12 +76,12 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     unsigned char* vbuf = TEAMS == 1 ? buf : buf + (size_t)L.rows * 128;
     const unsigned sbase = smem_u32(buf), vbase = smem_u32(vbuf);
 
-    const Shape s = a.s;
-    const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
-    const int unit = blockIdx.x / tiles;          // query head (b H + h), or kv head (b Hkv + hk) for TEAMS = 2
-    const int i0 = (blockIdx.x % tiles) * kMmaTile;
-    const int b = TEAMS == 1 ? unit / s.H : unit / s.Hkv;
-    const int hk = TEAMS == 1 ? (unit % s.H) / s.G : unit % s.Hkv;
+    const Shape& s = a.s;
+    // block = unit * tiles + tile; unit = query head (b H + h), or kv head (b Hkv + hk) for TEAMS = 2
+    const int unit = (int)fdiv(blockIdx.x, s.dTiles);
+    const int i0 = ((int)blockIdx.x - unit * (int)s.dTiles.d) * kMmaTile;
+    const int b = (int)fdiv((unsigned)unit, TEAMS == 1 ? s.dH : s.dHkv);
+    const int hk = TEAMS == 1 ? (int)fdiv((unsigned)(unit - b * s.H), s.dG) : unit - b * s.Hkv;
     const int head = b * s.Hkv + hk;
     const int tid = threadIdx.x, lane = tid & 31, warp = (tid >> 5) % kWarps, team = (tid >> 5) / kWarps;
     const int g4 = lane >> 2, c4 = lane & 3;
@@ -107,40 +107,87 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         pdl_wait();
     }
 
-    // ---- issue the key copies (and for TEAMS = 2 the value copies) (warp 0)
+    // ---- issue the key copies (and for TEAMS = 2 the value copies) (warp 0,
+    // once the barriers are initialised; the other warps go on to their q~)
+    __shared__ unsigned keys_done;                // warps done with the staged keys (TEAMS = 1)
     if (tid == 0) {
         mbar_init(&bars[0], 1);
         mbar_init(&bars[1], 1);
+        keys_done = 0;
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
     }
+    __syncthreads();                              // barrier init visible
     if (tid < 32) {
-        __syncwarp();
         issue_rows(buf, &tmK.m64, &tmK.m8, L, i0, head, &bars[0], lane);
         if (TEAMS == 2) issue_rows(vbuf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
     }
-    __syncthreads();                              // barrier init visible
+
+    // ---- per-lane constants of the fragment layouts
+    // ldmatrix (keys, non-transposed): lane supplies row lr of matrix lh; the
+    // swizzled chunk of a row r is chunk ^ (r & 7), so for the 8-row groups of
+    // one load the address is base(r) with (lh ^ r) & 7, and the loads of the
+    // next 8 rows (+1024 bytes) and of chunks 4..7 (address bit 6) follow.
+    const int lr = lane & 7, lh = lane >> 3;
+    // ldmatrix .trans (values): lane supplies row lv of the 16-row k-chunk and
+    // chunk n + lq of it (n even, so chunk n + lq = n ^ lq).
+    const int lv = (lane & 7) + (lane & 8), lq = lane >> 4;
+    // Rung columns: slab rows x = 0..15 at absolute bw - s0 - 1 + x.  Row r's
+    // far score is column x = r (weight w), its floor score column x = r + 1
+    // (weight 1-w).  Of this thread's entries (rows g4, g4+8; columns 2c4,
+    // 2c4+1 and 2c4+8, 2c4+9) only those with x - r in {-1, 0, 1} can be
+    // either, a pattern fixed by delta = 2c4 - g4: entries (g4, 2c4 + u) and
+    // (g4+8, 2c4+8 + u) take  u=0: w if delta = 0, 1-w if delta = 1;
+    //                         u=1: w if delta = -1, 1-w if delta = 0,
+    // each of the form A + B w; row g4 = 7 also has its floor at column 8.
+    // The same weights place p in the A fragment of the value product, and B
+    // alone (the derivative in w) gives the far-minus-floor score.
+    const int dl = 2 * c4 - g4;
+    const float ia0 = dl == 1 ? 1.f : 0.f, ib0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f);
+    const float ia1 = dl == 0 ? 1.f : 0.f, ib1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
+    const float m7 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
+    // A row's rung score lives in at most two lanes of its quad: for even g4
+    // lane g4/2 holds both columns; for odd g4 lanes (g4-1)/2 and (g4+1)/2
+    // (lanes 3 and 0 for g4 = 7) hold one each.  One shuffle from the partner
+    // lane completes the sum in both; a lane with no column of the row adds a
+    // partial of zero and takes no part in the softmax of that row.
+    const bool contrib = (dl >= -1 && dl <= 1) || m7 != 0.f;
+    const bool writer = dl == 0 || dl == -1;      // one lane per row stores its residuals
+    int partner;
+    if (g4 & 1) {
+        const int x = (g4 - 1) >> 1, y = ((g4 + 1) >> 1) & 3;
+        partner = c4 == x ? y : (c4 == y ? x : c4);
+    } else {
+        partner = ((g4 >> 1) + 1) & 3;
+    }
+    const int src = (lane & ~3) | partner;
 
 #pragma unroll 1
     for (int hq = TEAMS == 1 ? 0 : team; hq < (TEAMS == 1 ? 1 : s.G); hq += TEAMS) {
     const int bh = TEAMS == 1 ? unit : b * s.H + hk * s.G + hq;
 
-    // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32)
+    // ---- q~ as fp16 A fragments (rows g4, g4+8 of the tile; RoPE pairs m, m+32),
+    // pre-scaled by scale * log2(e) so that the scores come out in log2 units.
     // Thread dims: 16kc + 2c4 + {0,1} and 16kc + 8 + 2c4 + {0,1} for kc = 0..3.
-    // SAVE: also as bf16 (qs), the residual the key pass reads.
+    // SAVE: also q~ itself as bf16 (qs), the residual the key pass reads.
+    const float sc2 = s.scale * kLog2e;
     unsigned qa[4][4], qs[SAVE ? 4 : 1][4];
-    float qmax = 0.f;                             // largest |q~| of the thread: fp16 holds < 65520
+    float qmax = 0.f;                             // largest |fp16 operand| of the thread: fp16 holds < 65520
     {
         if (TEAMS == 2) load_q(bh);
         // cos/sin of the 8 pairs at position bw+g4, then advanced by 8 positions
-        // for row g4+8 with the host's fp64 cos/sin(8 theta_m)
+        // for row g4+8 with the host's fp64 cos/sin(8 theta_m); they carry the
+        // score scale (the SAVE residual divides it out again)
         float cs[2][4], sn[2][4];
         const int pos0 = bw + g4;
+        const float cscale = sc2;
 #pragma unroll
         for (int kc = 0; kc < 2; ++kc)
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
                 rope_cs(a.rope, m, pos0, cs[kc][j], sn[kc][j]);
+                cs[kc][j] *= cscale;
+                sn[kc][j] *= cscale;
             }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -176,20 +223,24 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             }
 #pragma unroll
             for (int kc = 0; kc < 4; ++kc) {
-                qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);       // a0 / a1: k = 2c4, 2c4+1
-                qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);   // a2 / a3: k = 2c4+8, 2c4+9
+                qa[kc][half] = pack_f16(x[kc][0], x[kc][1]);          // a0 / a1: k = 2c4, 2c4+1
+                qa[kc][2 + half] = pack_f16(x[kc][2], x[kc][3]);      // a2 / a3: k = 2c4+8, 2c4+9
                 if constexpr (SAVE) {
-                    qs[kc][half] = pack_bf16(x[kc][0], x[kc][1]);
-                    qs[kc][2 + half] = pack_bf16(x[kc][2], x[kc][3]);
+                    const float u = 1.f / sc2;
+                    qs[kc][half] = pack_bf16(x[kc][0] * u, x[kc][1] * u);
+                    qs[kc][2 + half] = pack_bf16(x[kc][2] * u, x[kc][3] * u);
                 }
             }
         }
     }
     if (qmax >= 65520.f) raise_status(a.status, kStatusRange);
-    const float sc2 = s.scale * kLog2e;           // scores in log2 units
     const int qlo = bw + g4, qhi = bw + g4 + 8;   // absolute queries of this thread's rows
     const bool vlo = qlo < s.T && g4 < kRowsPerWarp;
     const bool vhi = qhi < s.T && g4 + 8 < kRowsPerWarp;
+    // a rung slot of a row is attended when d_k <= query; this lane takes part
+    // in a row's rung softmax only where it holds part of the row's score
+    const float qlo_eff = (contrib && vlo) ? (float)qlo : -1.f;
+    const float qhi_eff = (contrib && vhi) ? (float)qhi : -1.f;
     const size_t rowbase = (size_t)bh * s.T;
     if constexpr (SAVE) {
         // rotated query rows 0..14 of the warp's tile, through the warp's stage
@@ -218,116 +269,131 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         }
     }
 
+    // The active rungs in increasing d: those with d_k > bw + 14 are masked
+    // for every row of the warp and form the tail of the list.
+    int n_use = L.n_act;
+    while (n_use > 0 && L.act_d[n_use - 1] > (float)(bw + kRowsPerWarp - 1)) --n_use;
+
     const bool ok_k = mbar_wait(&bars[0], 0);
 
     // ---- window band scores: keys [bw - Wp, bw + 16), n-tile j covers 8 keys
     float sw[NT][4];
+    {
+        const int rb = L.win_smem + wrel - Wp + lr;
+        const unsigned ab = sbase + ((unsigned)rb << 7) + ((unsigned)((rb ^ lh) & 7) << 4);
 #pragma unroll
-    for (int j = 0; j < NT; ++j) {
-        sw[j][0] = sw[j][1] = sw[j][2] = sw[j][3] = 0.f;
-        const int krow = L.win_smem + wrel - Wp + 8 * j + (lane & 7);
-#pragma unroll
-        for (int kc = 0; kc < 4; kc += 2) {
+        for (int j = 0; j < NT; ++j) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
-            mma_f16_16816(sw[j], qa[kc], b0, b1);
-            mma_f16_16816(sw[j], qa[kc + 1], b2, b3);
+            ldsm_x4(ab + 1024u * j, b0, b1, b2, b3);
+            mma_f16_16816_z(sw[j], qa[0], b0, b1);
+            mma_f16_16816(sw[j], qa[1], b2, b3);
+            ldsm_x4((ab ^ 64u) + 1024u * j, b0, b1, b2, b3);
+            mma_f16_16816(sw[j], qa[2], b0, b1);
+            mma_f16_16816(sw[j], qa[3], b2, b3);
         }
     }
-    float mlo = -INFINITY, mhi = -INFINITY;
+    float mlo = -INFINITY, mhi = -INFINITY;       // per-lane partial maxima until every slot is in
+    {
+        const int tb = g4 + Wp - 2 * c4;          // distance query - key of entry (row g4, column 2c4) in n-tile 0
 #pragma unroll
-    for (int j = 0; j < NT; ++j) {
+        for (int j = 0; j < NT; ++j)
 #pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            const int r = (e < 2) ? g4 : g4 + 8;
-            const int n = 8 * j + 2 * c4 + (e & 1);
-            const int t = r + Wp - n;                     // distance query - key
-            const int key = bw - Wp + n;
-            const bool ok = (e < 2 ? vlo : vhi) && t >= 0 && t <= s.W && key >= 0;
-            sw[j][e] = ok ? sw[j][e] * sc2 : -INFINITY;
-            if (e < 2) mlo = fmaxf(mlo, sw[j][e]); else mhi = fmaxf(mhi, sw[j][e]);
+            for (int e = 0; e < 4; ++e) {
+                const int t = tb + (e >= 2 ? 8 : 0) - 8 * j - (e & 1);
+                if ((unsigned)t > (unsigned)s.W) sw[j][e] = -INFINITY;
+            }
+        if (bw < Wp) {                            // the first tile: columns before position 0
+#pragma unroll
+            for (int j = 0; j < NT; ++j)
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (8 * j + 2 * c4 + (e & 1) < Wp - bw) sw[j][e] = -INFINITY;
+        }
+#pragma unroll
+        for (int j = 0; j < NT; ++j) {
+            mlo = fmaxf(mlo, fmaxf(sw[j][0], sw[j][1]));
+            mhi = fmaxf(mhi, fmaxf(sw[j][2], sw[j][3]));
         }
     }
-    mlo = quad_max(mlo);
-    mhi = quad_max(mhi);
 
-    // ---- rung scores: slab rows x = 0..15 at absolute bw - s0 - 1 + x.
-    // Row r's far score is column x = r (weight w), its floor score column
-    // x = r + 1 (weight 1-w).  Of this thread's entries (rows g4, g4+8; columns
-    // 2c4, 2c4+1 and 2c4+8, 2c4+9) only those with x - r in {-1, 0, 1} can be
-    // either, a pattern fixed by delta = 2c4 - g4: entries (g4, 2c4 + u) and
-    // (g4+8, 2c4+8 + u) take  u=0: w if delta = 0, 1-w if delta = 1;
-    //                         u=1: w if delta = -1, 1-w if delta = 0,
-    // each of the form A + B w; row g4 = 7 also has its floor at column 8.
-    // The same weights place p in the A fragment of the value product.
-    const int dl = 2 * c4 - g4;
-    const float ia0 = dl == 1 ? 1.f : 0.f, ib0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f);
-    const float ia1 = dl == 0 ? 1.f : 0.f, ib1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
-    const float m7 = (g4 == 7 && c4 == 0) ? 1.f : 0.f;
-    // far-minus-floor pattern (residual sd): +1 at the far entry, -1 at the floor entry
-    const float df0 = dl == 0 ? 1.f : (dl == 1 ? -1.f : 0.f), df1 = dl == -1 ? 1.f : (dl == 0 ? -1.f : 0.f);
+    // ---- rung scores (log2 units) of the rows this lane takes part in
+    const float inv_sc2 = 1.f / sc2;
     float rs[kMmaMaxRungs][2];
-#pragma unroll
-    for (int k = 0; k < kMmaMaxRungs; ++k) { rs[k][0] = -INFINITY; rs[k][1] = -INFINITY; }
-#pragma unroll
-    for (int k = 0; k < kMmaMaxRungs; ++k) {
-        if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
-        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;        // masked for the whole warp
-        const float w = a.r.w[k], w1 = 1.f - w;
-        float st[2][4];
-#pragma unroll
-        for (int t = 0; t < 2; ++t) {
-            st[t][0] = st[t][1] = st[t][2] = st[t][3] = 0.f;
-            const int krow = L.rung_smem[k] + wrel + 8 * t + (lane & 7);
-#pragma unroll
-            for (int kc = 0; kc < 4; kc += 2) {
-                unsigned b0, b1, b2, b3;
-                ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
-                mma_f16_16816(st[t], qa[kc], b0, b1);
-                mma_f16_16816(st[t], qa[kc + 1], b2, b3);
-            }
-        }
-        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-        const float plo = quad_sum(fmaf(c0, st[0][0], fmaf(c1, st[0][1], c7 * st[1][0]))) * sc2;
-        const float phi = quad_sum(fmaf(c0, st[1][2], c1 * st[1][3])) * sc2;
-        const float dk = a.r.d[k];
-        rs[k][0] = (vlo && dk <= (float)qlo) ? plo : -INFINITY;
-        rs[k][1] = (vhi && dk <= (float)qhi) ? phi : -INFINITY;
-        mlo = fmaxf(mlo, rs[k][0]);
-        mhi = fmaxf(mhi, rs[k][1]);
+    // rung i of the list sorted by d (i < n_use)
+    auto score_rung = [&](int i) {
+        const int r = L.act_smem[i] + wrel + lr;
+        const unsigned ak = sbase + ((unsigned)r << 7) + ((unsigned)((r ^ lh) & 7) << 4);
+        float s0[4], s1[4];
+        unsigned b0, b1, b2, b3;
+        ldsm_x4(ak, b0, b1, b2, b3);
+        mma_f16_16816_z(s0, qa[0], b0, b1);
+        mma_f16_16816(s0, qa[1], b2, b3);
+        ldsm_x4(ak + 1024u, b0, b1, b2, b3);
+        mma_f16_16816_z(s1, qa[0], b0, b1);
+        mma_f16_16816(s1, qa[1], b2, b3);
+        ldsm_x4(ak ^ 64u, b0, b1, b2, b3);
+        mma_f16_16816(s0, qa[2], b0, b1);
+        mma_f16_16816(s0, qa[3], b2, b3);
+        ldsm_x4((ak ^ 64u) + 1024u, b0, b1, b2, b3);
+        mma_f16_16816(s1, qa[2], b0, b1);
+        mma_f16_16816(s1, qa[3], b2, b3);
+        const float w = L.act_w[i];
+        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = fmaf(-m7, w, m7);
+        float plo = fmaf(c0, s0[0], fmaf(c1, s0[1], c7 * s1[0]));
+        float phi = fmaf(c0, s1[2], c1 * s1[3]);
+        plo += __shfl_sync(0xffffffffu, plo, src);
+        phi += __shfl_sync(0xffffffffu, phi, src);
+        const float d = L.act_d[i];
+        rs[i][0] = d <= qlo_eff ? plo : -INFINITY;
+        rs[i][1] = d <= qhi_eff ? phi : -INFINITY;
+        mlo = fmaxf(mlo, rs[i][0]);
+        mhi = fmaxf(mhi, rs[i][1]);
         if constexpr (SAVE) {
-            const float sdl = quad_sum(fmaf(df0, st[0][0], fmaf(df1, st[0][1], -m7 * st[1][0])));
-            const float sdh = quad_sum(fmaf(df0, st[1][2], df1 * st[1][3]));
-            if (c4 == 0) {
-                float* sd = a.res_sd + ((size_t)bh * a.r.K + k) * s.T;
-                if (vlo) sd[qlo] = sdl;
-                if (vhi) sd[qhi] = sdh;
+            float sdl = fmaf(ib0, s0[0], fmaf(ib1, s0[1], -m7 * s1[0]));
+            float sdh = fmaf(ib0, s1[2], ib1 * s1[3]);
+            sdl += __shfl_sync(0xffffffffu, sdl, src);
+            sdh += __shfl_sync(0xffffffffu, sdh, src);
+            if (writer) {
+                float* sd = a.res_sd + ((size_t)bh * a.r.K + L.act_k[i]) * s.T;
+                if (vlo) sd[qlo] = sdl * inv_sc2;
+                if (vhi) sd[qhi] = sdh * inv_sc2;
             }
         }
+    };
+#pragma unroll
+    for (int i = 0; i < kMmaMaxRungs; ++i) {
+        if (i >= n_use) break;
+        score_rung(i);
     }
 
     if (TEAMS == 1) {
-        // ---- all warps are done with the keys: stage the values into the same buffer
+        // ---- the last warp done with the keys stages the values into the same
+        // buffer (acquire-release counter: every warp's key reads come before
+        // the copies; the others go on without waiting)
         asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
-        __syncthreads();
-        if (warp == 0) issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
+        __syncwarp();
+        unsigned before = 0;
+        if (lane == 0) before = atom_add_acq_rel(&keys_done, 1u);
+        before = __shfl_sync(0xffffffffu, before, 0);
+        if (before == kWarps - 1) {
+            asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+            issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
+        }
     }
 
     // ---- probabilities (unnormalised, row max -> exactly 1) while values arrive
+    mlo = quad_max(mlo);
+    mhi = quad_max(mhi);
     if (mlo == -INFINITY) mlo = 0.f;              // rows beyond T: keep arithmetic finite
     if (mhi == -INFINITY) mhi = 0.f;
-    float llo = 0.f, lhi = 0.f;
     unsigned pa[NT][2];                           // window band P as bf16 A fragments
     float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;   // residual exp(s - max) per slot
 #pragma unroll
     for (int j = 0; j < NT; ++j) {
-        const float e0 = exp2f(sw[j][0] - mlo), e1 = exp2f(sw[j][1] - mlo);
-        const float e2 = exp2f(sw[j][2] - mhi), e3 = exp2f(sw[j][3] - mhi);
-        const float p0 = bf16_round(e0), p1 = bf16_round(e1), p2 = bf16_round(e2), p3 = bf16_round(e3);
-        llo += p0 + p1;
-        lhi += p2 + p3;
-        pa[j][0] = pack_bf16(p0, p1);
-        pa[j][1] = pack_bf16(p2, p3);
+        const float e0 = ex2(sw[j][0] - mlo), e1 = ex2(sw[j][1] - mlo);
+        const float e2 = ex2(sw[j][2] - mhi), e3 = ex2(sw[j][3] - mhi);
+        pa[j][0] = pack_bf16(e0, e1);
+        pa[j][1] = pack_bf16(e2, e3);
         if constexpr (SAVE) {                     // window slot t of rows 0..14 (0 before position 0)
             const float ev[4] = {e0, e1, e2, e3};
 #pragma unroll
@@ -339,17 +405,12 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             }
         }
     }
-    // (the row sums stay per-lane partials until every slot is in; one quad
-    // sum per row then completes them)
-
 
     if constexpr (SAVE) {
         // ---- residual p of the active rungs no row of the warp attends (the
         // tail of the list sorted by d): 0
         if (c4 == 0) {
-            int i = L.n_act;
-            while (i > 0 && L.act_d[i - 1] > (float)(bw + kRowsPerWarp - 1)) --i;
-            for (; i < L.n_act; ++i) {
+            for (int i = n_use; i < L.n_act; ++i) {
                 float* row = Pg + (size_t)(s.W + 1 + L.act_k[i]) * s.T;
                 if (vlo) row[qlo] = 0.f;
                 if (vhi) row[qhi] = 0.f;
@@ -359,74 +420,80 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 
     const bool ok_v = mbar_wait(&bars[1], 0);
 
-    float o[8][4];
+    // o: the value product; osum: the row sums of the same rounded weights
+    float o[8][4], osum[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
     for (int n = 0; n < 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
 
     // ---- window band values: k-chunks of 16 keys (+ one of 8 when NT is odd)
+    {
+        const int rv = L.win_smem + wrel - Wp + lv;
+        const unsigned av = vbase + ((unsigned)rv << 7) + ((unsigned)((rv ^ lq) & 7) << 4);
 #pragma unroll
-    for (int kk = 0; kk + 1 < NT; kk += 2) {
-        const unsigned afr[4] = {pa[kk][0], pa[kk][1], pa[kk + 1][0], pa[kk + 1][1]};
-        const int vrow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7) + 8 * ((lane >> 3) & 1);
+        for (int kk = 0; kk + 1 < NT; kk += 2) {
+            const unsigned afr[4] = {pa[kk][0], pa[kk][1], pa[kk + 1][0], pa[kk + 1][1]};
 #pragma unroll
-        for (int n = 0; n < 8; n += 2) {
-            unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(vbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
-            mma_bf16_16816(o[n], afr, b0, b1);
-            mma_bf16_16816(o[n + 1], afr, b2, b3);
+            for (int n = 0; n < 8; n += 2) {
+                unsigned b0, b1, b2, b3;
+                ldsm_x4_t((av ^ (unsigned)(n << 4)) + 1024u * kk, b0, b1, b2, b3);
+                mma_bf16_16816(o[n], afr, b0, b1);
+                mma_bf16_16816(o[n + 1], afr, b2, b3);
+            }
+            mma_bf16_16816(osum, afr, kOnesBf16x2, kOnesBf16x2);
         }
     }
     if constexpr (NT & 1) {
         const int kk = NT - 1;
-        const int vrow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7);
+        const int rt = L.win_smem + wrel - Wp + 8 * kk + lr;
+        const unsigned at = vbase + ((unsigned)rt << 7) + ((unsigned)((rt ^ lh) & 7) << 4);
 #pragma unroll
         for (int n = 0; n < 8; n += 4) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(vbase, vrow, n + (lane >> 3)), b0, b1, b2, b3);
+            ldsm_x4_t(at ^ (unsigned)(n << 4), b0, b1, b2, b3);
             mma_bf16_1688(o[n], pa[kk][0], pa[kk][1], b0);
             mma_bf16_1688(o[n + 1], pa[kk][0], pa[kk][1], b1);
             mma_bf16_1688(o[n + 2], pa[kk][0], pa[kk][1], b2);
             mma_bf16_1688(o[n + 3], pa[kk][0], pa[kk][1], b3);
         }
+        mma_bf16_1688(osum, pa[kk][0], pa[kk][1], kOnesBf16x2);
     }
 
     // ---- rung values: Phat[r][x] = p_r w at x = r, p_r (1-w) at x = r + 1
     // A-fragment columns of this thread: 2c4 + {0,1} (a0, a1) and 2c4 + 8 + {0,1} (a2, a3).
-#pragma unroll
-    for (int k = 0; k < kMmaMaxRungs; ++k) {
-        if (k >= a.r.K || !((a.r.active >> k) & 1u)) continue;
-        if (a.r.d[k] > (float)(bw + kRowsPerWarp - 1)) continue;
-        const float w = a.r.w[k], w1 = 1.f - w;
-        const float plo = exp2f(rs[k][0] - mlo), phi = exp2f(rs[k][1] - mhi);   // 0 when masked
-        // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
-        // take the same rounded entries, as for the window band
-        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
-        const float h00 = bf16_round(c0 * plo), h01 = bf16_round(c1 * plo), h20 = bf16_round(c7 * plo);
-        const float h30 = bf16_round(c0 * phi), h31 = bf16_round(c1 * phi);
-        llo += h00 + h01 + h20;
-        lhi += h30 + h31;
+    auto value_rung = [&](int i) {
+        const float w = L.act_w[i];
+        const float plo = ex2(rs[i][0] - mlo), phi = ex2(rs[i][1] - mhi);   // 0 when masked
         if constexpr (SAVE) {
-            if (c4 == 0) {                        // residual p of rung k
-                float* row = Pg + (size_t)(s.W + 1 + k) * s.T;
+            if (writer) {                         // residual p of the rung
+                float* row = Pg + (size_t)(s.W + 1 + L.act_k[i]) * s.T;
                 if (vlo) row[qlo] = plo;
                 if (vhi) row[qhi] = phi;
             }
         }
-        const unsigned ahi[4] = {pack_bf16(h00, h01), 0u, pack_bf16(h20, 0.f), pack_bf16(h30, h31)};
-        const int vrow = L.rung_smem[k] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+        // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
+        // come from the same rounded entries (the ones product below)
+        const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = fmaf(-m7, w, m7);
+        const unsigned ahi[4] = {pack_bf16(c0 * plo, c1 * plo), 0u, pack_bf16(c7 * plo, 0.f),
+                                 pack_bf16(c0 * phi, c1 * phi)};
+        const int rv = L.act_smem[i] + wrel + lv;
+        const unsigned av = vbase + ((unsigned)rv << 7) + ((unsigned)((rv ^ lq) & 7) << 4);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(vbase, vrow, n + (lane >> 4)), b0, b1, b2, b3);
+            ldsm_x4_t(av ^ (unsigned)(n << 4), b0, b1, b2, b3);
             mma_bf16_16816(o[n], ahi, b0, b1);
             mma_bf16_16816(o[n + 1], ahi, b2, b3);
         }
+        mma_bf16_16816(osum, ahi, kOnesBf16x2, kOnesBf16x2);
+    };
+#pragma unroll
+    for (int i = 0; i < kMmaMaxRungs; ++i) {
+        if (i >= n_use) break;
+        value_rung(i);
     }
 
-    llo = quad_sum(llo);
-    lhi = quad_sum(lhi);
-
     // ---- normalise and store rows 0..14 of the tile
+    const float llo = osum[0], lhi = osum[2];     // every column of the ones product is the row sum
     const bool ok = ok_k && ok_v;
     if (!ok) raise_status(a.status, kStatusWaitTimeout);
     const float inv_lo = ok ? 1.f / llo : __int_as_float(0x7fc00000);
