@@ -112,25 +112,26 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
     }
     ok = mbar_wait(bar, parity) && ok;
 
+    const int lv = (lane & 7) + (lane & 8);       // .trans loads: row of the 16-row k-chunk, chunk lane >> 4
+    const unsigned avb = row_chunk(sbase, L.win_smem + wrel + lv, lane >> 4);
 #pragma unroll
     for (int kk = 0; kk + 1 < NT; kk += 2) {
         const unsigned afr[4] = {band[kk][0], band[kk][1], band[kk + 1][0], band[kk + 1][1]};
-        const int xrow = L.win_smem + wrel + 8 * kk + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
+            ldsm_x4_t((avb ^ (unsigned)(n << 4)) + 1024u * kk, b0, b1, b2, b3);
             mma_bf16_16816(acc[n], afr, b0, b1);
             mma_bf16_16816(acc[n + 1], afr, b2, b3);
         }
     }
     if constexpr (NT & 1) {
         const int kk = NT - 1;
-        const int xrow = L.win_smem + wrel + 8 * kk + (lane & 7);
+        const unsigned at = row_chunk(sbase, L.win_smem + wrel + 8 * kk + (lane & 7), lane >> 3);
 #pragma unroll
         for (int n = 0; n < 8; n += 4) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 3)), b0, b1, b2, b3);
+            ldsm_x4_t(at ^ (unsigned)(n << 4), b0, b1, b2, b3);
             mma_bf16_1688(acc[n], band[kk][0], band[kk][1], b0);
             mma_bf16_1688(acc[n + 1], band[kk][0], band[kk][1], b1);
             mma_bf16_1688(acc[n + 2], band[kk][0], band[kk][1], b2);
@@ -167,11 +168,11 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
             const float2 v8 = *reinterpret_cast<const float2*>(&rv[ii][2 * c4 + 8]);
             const unsigned afr[4] = {pack_bf16(clo * v0.x, chi * v0.y), 0u,
                                      pack_bf16(m2 * w * v8.x, 0.f), pack_bf16(clo * v8.x, chi * v8.y)};
-            const int xrow = L.act_smem[ii] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+            const unsigned av = row_chunk(sbase, L.act_smem[ii] + wrel + lv, lane >> 4);
 #pragma unroll
             for (int n = 0; n < 8; n += 2) {
                 unsigned b0, b1, b2, b3;
-                ldsm_x4_t(row_chunk(sbase, xrow, n + (lane >> 4)), b0, b1, b2, b3);
+                ldsm_x4_t(av ^ (unsigned)(n << 4), b0, b1, b2, b3);
                 mma_bf16_16816(acc[n], afr, b0, b1);
                 mma_bf16_16816(acc[n + 1], afr, b2, b3);
             }
@@ -192,8 +193,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     // so the wait for it comes before pass 1 (dS), whose first block then sums
     // the query pass's rung partials.
     pdl_trigger();
-    const int tiles = (a.s.T + kMmaTile - 1) / kMmaTile;
-    const int units = tiles * a.s.B * a.s.Hkv;
+    const int units = (int)a.s.dTiles.d * a.s.B * a.s.Hkv;
     const int pass_first = SPLIT && (int)blockIdx.x >= units ? 1 : 0;
     const int pass_end = SPLIT ? pass_first + 1 : 2;
     const int blk = (int)blockIdx.x - pass_first * units;
@@ -209,10 +209,10 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const unsigned sbase = smem_u32(buf);
 
-    const Shape s = a.s;
-    const int bhk = blk / tiles;                          // b * Hkv + hk
-    const int j0 = (blk % tiles) * kMmaTile;
-    const int b = bhk / s.Hkv, hk = bhk % s.Hkv;
+    const Shape& s = a.s;
+    const int bhk = (int)fdiv((unsigned)blk, s.dTiles);   // b * Hkv + hk; blk = bhk * tiles + tile
+    const int j0 = (blk - bhk * (int)s.dTiles.d) * kMmaTile;
+    const int b = (int)fdiv((unsigned)bhk, s.dHkv), hk = bhk - b * s.Hkv;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int g4 = lane >> 2, c4 = lane & 3;
     const int wrel = warp * kRowsPerWarp;

@@ -86,11 +86,10 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     unsigned char* buf = reinterpret_cast<unsigned char*>(((uintptr_t)smem_raw + 1023) & ~(uintptr_t)1023);
     const unsigned sbase = smem_u32(buf);
 
-    const Shape s = a.s;
-    const int tiles = (s.T + kMmaTile - 1) / kMmaTile;
-    const int bh = blockIdx.x / tiles;
-    const int i0 = (blockIdx.x % tiles) * kMmaTile;
-    const int b = bh / s.H, h = bh % s.H, hk = h / s.G;
+    const Shape& s = a.s;
+    const int bh = (int)fdiv(blockIdx.x, s.dTiles);              // block = bh * tiles + tile
+    const int i0 = ((int)blockIdx.x - bh * (int)s.dTiles.d) * kMmaTile;
+    const int b = (int)fdiv((unsigned)bh, s.dH), hk = (int)fdiv((unsigned)(bh - b * s.H), s.dG);
     const int head = b * s.Hkv + hk;
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int g4 = lane >> 2, c4 = lane & 3;
@@ -315,15 +314,17 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     // ---- window band dp = dO . v
     float dpw[NT][4];
 #pragma unroll
-    for (int j = 0; j < NT; ++j) {
-        dpw[j][0] = dpw[j][1] = dpw[j][2] = dpw[j][3] = 0.f;
-        const int krow = L.win_smem + wrel - Wp + 8 * j + (lane & 7);
+    {
+        const unsigned ab = row_chunk(sbase, L.win_smem + wrel - Wp + (lane & 7), lane >> 3);
 #pragma unroll
-        for (int kc = 0; kc < 4; kc += 2) {
+        for (int j = 0; j < NT; ++j) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
-            mma_bf16_16816(dpw[j], da[kc], b0, b1);
-            mma_bf16_16816(dpw[j], da[kc + 1], b2, b3);
+            ldsm_x4(ab + 1024u * j, b0, b1, b2, b3);
+            mma_bf16_16816_z(dpw[j], da[0], b0, b1);
+            mma_bf16_16816(dpw[j], da[1], b2, b3);
+            ldsm_x4((ab ^ 64u) + 1024u * j, b0, b1, b2, b3);
+            mma_bf16_16816(dpw[j], da[2], b0, b1);
+            mma_bf16_16816(dpw[j], da[3], b2, b3);
         }
     }
     // the rows' largest |dp - Delta| over the band (rung terms join below):
@@ -391,19 +392,19 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             need_rows(L.act_smem[ib[1]] + wrel);
             float dt[2][2][4];
 #pragma unroll
-            for (int u = 0; u < 2; ++u)
+            for (int u = 0; u < 2; ++u) {
+                const unsigned ak = row_chunk(sbase, L.act_smem[ib[u]] + wrel + (lane & 7), lane >> 3);
 #pragma unroll
                 for (int t = 0; t < 2; ++t) {
-                    dt[u][t][0] = dt[u][t][1] = dt[u][t][2] = dt[u][t][3] = 0.f;
-                    const int krow = L.act_smem[ib[u]] + wrel + 8 * t + (lane & 7);
-#pragma unroll
-                    for (int kc = 0; kc < 4; kc += 2) {
-                        unsigned b0, b1, b2, b3;
-                        ldsm_x4(row_chunk(sbase, krow, 2 * kc + (lane >> 3)), b0, b1, b2, b3);
-                        mma_bf16_16816(dt[u][t], da[kc], b0, b1);
-                        mma_bf16_16816(dt[u][t], da[kc + 1], b2, b3);
-                    }
+                    unsigned b0, b1, b2, b3;
+                    ldsm_x4(ak + 1024u * t, b0, b1, b2, b3);
+                    mma_bf16_16816_z(dt[u][t], da[0], b0, b1);
+                    mma_bf16_16816(dt[u][t], da[1], b2, b3);
+                    ldsm_x4((ak ^ 64u) + 1024u * t, b0, b1, b2, b3);
+                    mma_bf16_16816(dt[u][t], da[2], b0, b1);
+                    mma_bf16_16816(dt[u][t], da[3], b2, b3);
                 }
+            }
             // per rung: this lane's shares of dp and ddp for rows g4 and g4+8,
             // reduce-scattered over the quad (lanes c4 = 0, 1 end with row g4,
             // lanes 2, 3 with row g4+8); lanes 0 and 2 then form their row's dS
@@ -565,25 +566,25 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         }
     }
     {
+        const unsigned avb = row_chunk(sbase, L.win_smem + wrel - Wp + (lane & 7) + (lane & 8), lane >> 4);
 #pragma unroll
         for (int kk = 0; kk + 1 < NT; kk += 2) {
             const unsigned afr[4] = {dsa[kk][0], dsa[kk][1], dsa[kk + 1][0], dsa[kk + 1][1]};
-            const int krow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7) + 8 * ((lane >> 3) & 1);
 #pragma unroll
             for (int n = 0; n < 8; n += 2) {
                 unsigned b0, b1, b2, b3;
-                ldsm_x4_t(row_chunk(sbase, krow, n + (lane >> 4)), b0, b1, b2, b3);
+                ldsm_x4_t((avb ^ (unsigned)(n << 4)) + 1024u * kk, b0, b1, b2, b3);
                 mma_f16_16816(dq[n], afr, b0, b1);
                 mma_f16_16816(dq[n + 1], afr, b2, b3);
             }
         }
         if constexpr (NT & 1) {
             const int kk = NT - 1;
-            const int krow = L.win_smem + wrel - Wp + 8 * kk + (lane & 7);
+            const unsigned at = row_chunk(sbase, L.win_smem + wrel - Wp + 8 * kk + (lane & 7), lane >> 3);
 #pragma unroll
             for (int n = 0; n < 8; n += 4) {
                 unsigned b0, b1, b2, b3;
-                ldsm_x4_t(row_chunk(sbase, krow, n + (lane >> 3)), b0, b1, b2, b3);
+                ldsm_x4_t(at ^ (unsigned)(n << 4), b0, b1, b2, b3);
                 mma_f16_1688(dq[n], dsa[kk][0], dsa[kk][1], b0);
                 mma_f16_1688(dq[n + 1], dsa[kk][0], dsa[kk][1], b1);
                 mma_f16_1688(dq[n + 2], dsa[kk][0], dsa[kk][1], b2);
@@ -624,13 +625,14 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 afr2[u][2] = pack_f16(c7 * dsl, 0.f);
                 afr2[u][3] = pack_f16(c0 * dsh, c1 * dsh);
             }
-            const int krow0 = L.act_smem[i_first] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
-            const int krow1 = L.act_smem[i_first + 1] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+            const int lv = (lane & 7) + (lane & 8);
+            const unsigned av0 = row_chunk(sbase, L.act_smem[i_first] + wrel + lv, lane >> 4);
+            const unsigned av1 = row_chunk(sbase, L.act_smem[i_first + 1] + wrel + lv, lane >> 4);
 #pragma unroll
             for (int n = 0; n < 8; n += 2) {
                 unsigned b0, b1, b2, b3, e0, e1, e2, e3;
-                ldsm_x4_t(row_chunk(sbase, krow0, n + (lane >> 4)), b0, b1, b2, b3);
-                ldsm_x4_t(row_chunk(sbase, krow1, n + (lane >> 4)), e0, e1, e2, e3);
+                ldsm_x4_t(av0 ^ (unsigned)(n << 4), b0, b1, b2, b3);
+                ldsm_x4_t(av1 ^ (unsigned)(n << 4), e0, e1, e2, e3);
                 mma_f16_16816(dq[n], afr2[0], b0, b1);
                 mma_f16_16816(dq[n + 1], afr2[0], b2, b3);
                 mma_f16_16816(dq[n], afr2[1], e0, e1);
@@ -699,11 +701,11 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
         const float dsl = ds_lo * cs_lo, dsh = ds_hi * cs_hi;
         const unsigned afr[4] = {pack_f16(c0 * dsl, c1 * dsl), 0u, pack_f16(c7 * dsl, 0.f),
                                  pack_f16(c0 * dsh, c1 * dsh)};
-        const int krow = L.act_smem[i] + wrel + (lane & 7) + 8 * ((lane >> 3) & 1);
+        const unsigned av = row_chunk(sbase, L.act_smem[i] + wrel + (lane & 7) + (lane & 8), lane >> 4);
 #pragma unroll
         for (int n = 0; n < 8; n += 2) {
             unsigned b0, b1, b2, b3;
-            ldsm_x4_t(row_chunk(sbase, krow, n + (lane >> 4)), b0, b1, b2, b3);
+            ldsm_x4_t(av ^ (unsigned)(n << 4), b0, b1, b2, b3);
             mma_f16_16816(dq[n], afr, b0, b1);
             mma_f16_16816(dq[n + 1], afr, b2, b3);
         }

@@ -121,6 +121,22 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         issue_rows(buf, &tmK.m64, &tmK.m8, L, i0, head, &bars[0], lane);
         if (TEAMS == 2) issue_rows(vbuf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
     }
+    // A warp whose tile starts past the end of the sequence (the last tile of
+    // a head) has no query to compute; in the one-head form it still counts
+    // as done with the keys, and issues the value copies if it is the last.
+    if (bw >= s.T) {
+        if (TEAMS == 1) {
+            __syncwarp();
+            unsigned before = 0;
+            if (lane == 0) before = atom_add_acq_rel(&keys_done, 1u);
+            before = __shfl_sync(0xffffffffu, before, 0);
+            if (before == kWarps - 1) {
+                asm volatile("fence.proxy.async.shared::cta;\n" ::: "memory");
+                issue_rows(buf, &tmV.m64, &tmV.m8, L, i0, head, &bars[1], lane);
+            }
+        }
+        return;
+    }
 
     // ---- per-lane constants of the fragment layouts
     // ldmatrix (keys, non-transposed): lane supplies row lr of matrix lh; the

@@ -91,6 +91,12 @@ __device__ __forceinline__ void mma_bf16_16816(float* d, const unsigned* a, unsi
                  : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
                  : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
+__device__ __forceinline__ void mma_bf16_16816_z(float* d, const unsigned* a, unsigned b0, unsigned b1) {
+    asm volatile("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+                 "{%10,%10,%10,%10};\n"
+                 : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+                 : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1), "f"(0.f));
+}
 __device__ __forceinline__ void mma_bf16_1688(float* d, unsigned a0, unsigned a1, unsigned b0) {
     asm volatile("mma.sync.aligned.m16n8k8.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5}, {%6}, "
                  "{%0,%1,%2,%3};\n"
@@ -129,10 +135,12 @@ __device__ __forceinline__ float quad_max(float x) {
     return x;
 }
 
-// Shared-memory byte address of 16-byte chunk `ch` of staged row `row` under the
-// 128-byte swizzle (chunk index XOR row % 8), buffer base 1024-byte aligned.
+// Shared-memory byte address of 16-byte chunk `ch` (< 8) of staged row `row`
+// under the 128-byte swizzle (chunk index XOR row % 8), buffer base 1024-byte
+// aligned.  XOR being linear, chunk ch ^ m of the same row is at the address
+// XOR (m << 4), and the row 8 further on 1024 bytes on.
 __device__ __forceinline__ unsigned row_chunk(unsigned base, int row, int ch) {
-    return base + (unsigned)row * 128u + (unsigned)((ch ^ (row & 7)) << 4);
+    return base + ((unsigned)row << 7) + ((unsigned)((row ^ ch) & 7) << 4);
 }
 
 // Warp 0 issues the copies of one staged tensor.  Lane n copies merged
