@@ -221,6 +221,8 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
     const bool vlo = klo < s.T && g4 < kRowsPerWarp;
     const bool vhi = khi < s.T && g4 + 8 < kRowsPerWarp;
 
+    __shared__ RopeSmem rsm;
+    rope_to_smem(rsm, a.rope, L, tid);
     if (tid == 0) {
         mbar_init(&bar, 1);
         asm volatile("fence.mbarrier_init.release.cluster;\n" ::: "memory");
@@ -269,7 +271,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
 #pragma unroll
             for (int n = 0; n < 4; ++n)
 #pragma unroll
-                for (int u = 0; u < 2; ++u) rope_cs(a.rope, 8 * n + 2 * c4 + u, klo, ec[n][u], es[n][u]);
+                for (int u = 0; u < 2; ++u) rope_cs_s(rsm, 8 * n + 2 * c4 + u, klo, ec[n][u], es[n][u]);
         }
         // Rows g4 (half 0) and g4 + 8 (half 1) leave through this warp's table,
         // 8 rows of 128 bytes at a time (16-byte chunk c of row r at chunk
@@ -285,7 +287,7 @@ bwd_key_mma_kernel(const __grid_constant__ RowMaps tmQ, const __grid_constant__ 
 #pragma unroll
                     for (int u = 0; u < 2; ++u) {
                         const int m = 8 * n + 2 * c4 + u;
-                        const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                        const float c8 = rsm.c8[m], s8 = rsm.s8[m];
                         const float cn = ec[n][u] * c8 - es[n][u] * s8;
                         es[n][u] = es[n][u] * c8 + ec[n][u] * s8;
                         ec[n][u] = cn;
@@ -350,7 +352,7 @@ cudaError_t launch_nt(const RowMaps& mq, const RowMaps& mg, const BwdArgs& a, co
 
 size_t bwd_key_mma_static_smem() {
     return sizeof(float) * (kWarps * kMmaMaxRungs * 16 + kWarps * 32 + kMmaMaxRungs) +
-           sizeof(long long) * kWarps * kMmaMaxRungs + 64;
+           sizeof(long long) * kWarps * kMmaMaxRungs + sizeof(RopeSmem) + 64;
 }
 
 size_t bwd_key_mma_smem_bytes(const MmaLayout& L, bool) { return fwd_mma_smem_bytes(L); }

@@ -98,6 +98,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 
     // ---- the tile's q, dO, o rows (two 64-row boxes each) to buffer rows
     // [0, 384), and the value rows that do not overlap them
+    __shared__ RopeSmem rsm;
+    rope_to_smem(rsm, a.rope, L, tid);
     if (tid == 0) {
         for (int i = 0; i < 4; ++i) mbar_init(&bars[i], 1);
         for (int j = 0; j < L.n_iv; ++j) {
@@ -201,7 +203,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
-                rope_cs(a.rope, m, qlo, cs[kc][j], sn[kc][j]);
+                rope_cs_s(rsm, m, qlo, cs[kc][j], sn[kc][j]);
             }
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
@@ -218,7 +220,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
-                        const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                        const float c8 = rsm.c8[m], s8 = rsm.s8[m];
                         const float cn = cs[kc][j] * c8 - sn[kc][j] * s8;
                         sn[kc][j] = sn[kc][j] * c8 + cs[kc][j] * s8;
                         cs[kc][j] = cn;
@@ -724,7 +726,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 #pragma unroll
     for (int n = 0; n < 4; ++n)
 #pragma unroll
-        for (int u = 0; u < 2; ++u) rope_cs(a.rope, 8 * n + 2 * c4 + u, qlo, ec[n][u], es[n][u]);
+        for (int u = 0; u < 2; ++u) rope_cs_s(rsm, 8 * n + 2 * c4 + u, qlo, ec[n][u], es[n][u]);
 #pragma unroll
     for (int half = 0; half < 2; ++half) {
         if (half == 1) {
@@ -733,7 +735,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 #pragma unroll
                 for (int u = 0; u < 2; ++u) {
                     const int m = 8 * n + 2 * c4 + u;
-                    const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                    const float c8 = rsm.c8[m], s8 = rsm.s8[m];
                     const float cn = ec[n][u] * c8 - es[n][u] * s8;
                     es[n][u] = es[n][u] * c8 + ec[n][u] * s8;
                     ec[n][u] = cn;
@@ -785,9 +787,10 @@ cudaError_t launch_nt(const RowMaps& mk, const RowMaps& mv, const QTileMaps& mt,
 }  // namespace
 
 size_t bwd_mma_static_smem() {
-    // dps, gsm, the interval barriers and counters, the four phase barriers
+    // dps, gsm, the interval barriers and counters, the four phase barriers, the RoPE steps
     return sizeof(float) * kWarps * kMmaMaxRungs * 16 * 2 + sizeof(float) * kWarps * kMmaMaxRungs +
-           (sizeof(unsigned long long) + sizeof(unsigned)) * (kMmaMaxRungs + 1) + 4 * sizeof(unsigned long long) + 64;
+           (sizeof(unsigned long long) + sizeof(unsigned)) * (kMmaMaxRungs + 1) + 4 * sizeof(unsigned long long) +
+           sizeof(RopeSmem) + 64;
 }
 
 int bwd_mma_blocks(const Shape& s) {

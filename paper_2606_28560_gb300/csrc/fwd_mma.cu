@@ -110,6 +110,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     // ---- issue the key copies (and for TEAMS = 2 the value copies) (warp 0,
     // once the barriers are initialised; the other warps go on to their q~)
     __shared__ unsigned keys_done;                // warps done with the staged keys (TEAMS = 1)
+    __shared__ RopeSmem rsm;
+    rope_to_smem(rsm, a.rope, L, tid);
     if (tid == 0) {
         mbar_init(&bars[0], 1);
         mbar_init(&bars[1], 1);
@@ -201,7 +203,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
                 const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
-                rope_cs(a.rope, m, pos0, cs[kc][j], sn[kc][j]);
+                rope_cs_s(rsm, m, pos0, cs[kc][j], sn[kc][j]);
                 cs[kc][j] *= cscale;
                 sn[kc][j] *= cscale;
             }
@@ -221,7 +223,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
                     for (int j = 0; j < 4; ++j) {
                         const int m = 16 * kc + 2 * c4 + (j & 1) + 8 * (j >> 1);
-                        const float c8 = L.rope_c8[m], s8 = L.rope_s8[m];
+                        const float c8 = rsm.c8[m], s8 = rsm.s8[m];
                         const float cn = cs[kc][j] * c8 - sn[kc][j] * s8;
                         sn[kc][j] = sn[kc][j] * c8 + cs[kc][j] * s8;
                         cs[kc][j] = cn;
@@ -605,8 +607,9 @@ bool encode_rows_map(CUtensorMap* map, const void* base, CUtensorMapDataType dt,
 
 size_t fwd_mma_smem_bytes(const MmaLayout& L) { return (size_t)L.buf_rows * 128 + 1024; }
 
-// the two barriers of a CTA (rounded up) and its warps' output stages
-size_t fwd_mma_static_smem() { return 64 + kWarps * 1024; }
+// the barriers and counter of a CTA (rounded up), its warps' output stages
+// and the RoPE steps
+size_t fwd_mma_static_smem() { return 64 + kWarps * 1024 + sizeof(RopeSmem); }
 
 size_t fwd_mma_gqa_smem_limit() { return 227 * 1024 - 64 - 1024; }
 

@@ -189,6 +189,29 @@ __device__ __forceinline__ void issue_interval(unsigned char* dst, const CUtenso
     for (; r < len; r += 8) tma_load_3d(dst + (size_t)(srow + r) * 128, map8, 0, grow + r, head, bar);
 }
 
+// The RoPE phase steps of the 32 pairs (see RopeParams) and the cos, sin of 8
+// position steps, copied into shared memory once per CTA: a thread reads the
+// pairs of its fragment columns, which differ between the lanes of a warp, and
+// lane-dependent reads of kernel parameters are serialised.
+struct RopeSmem {
+    unsigned long long F[kHalf];
+    float c8[kHalf], s8[kHalf];
+};
+// Called by threads 0..31 (or all: others do nothing) before a CTA barrier.
+__device__ __forceinline__ void rope_to_smem(RopeSmem& r, const RopeParams& rp, const MmaLayout& L, int tid) {
+    if (tid < kHalf) {
+        r.F[tid] = rp.F[tid];
+        r.c8[tid] = L.rope_c8[tid];
+        r.s8[tid] = L.rope_s8[tid];
+    }
+}
+// cos/sin of the angle of pair m at position pos (as rope_cs).
+__device__ __forceinline__ void rope_cs_s(const RopeSmem& r, int m, int pos, float& c, float& s) {
+    const unsigned long long ph = (unsigned long long)(unsigned)pos * r.F[m];
+    const int hi = (int)(unsigned)(ph >> 32);        // signed turn fraction in [-1/2, 1/2)
+    __sincosf((float)hi * 1.4629180792671596e-09f, &s, &c);   // 2*pi / 2^32
+}
+
 // Shared-memory counter increment with acquire-release order (CTA scope);
 // returns the old value.
 __device__ __forceinline__ unsigned atom_add_acq_rel(unsigned* p, unsigned v) {
