@@ -172,9 +172,10 @@ const char* fibattn_last_error(void);
  *   bit 0 -- a kernel gave up waiting for one of its own shared-memory staging
  *            copies (each wait is bounded to 1 s of the GPU's global timer);
  *            the affected tiles' outputs (out, lse, gradients) are NaN.
- *   bit 1 -- a RoPE-rotated q or k entry reached 65520 in magnitude: the bf16
- *            path keeps rotated rows in fp16 (for score precision), which
- *            cannot hold it.
+ *   bit 1 -- an entry of a 16-bit rotated row reached 65520 in magnitude:
+ *            the bf16 path keeps the RoPE-rotated keys, and the rotated
+ *            queries times the score scale, in fp16 (for score precision),
+ *            which cannot hold it.
  * fibattn_check_status synchronises `stream`, reads the calling thread's
  * current device's word into *flags (may be NULL) and clears it.  Returns
  * FIBATTN_ERR_INTERNAL if bit 0 was set, else FIBATTN_ERR_RANGE if bit 1 was
