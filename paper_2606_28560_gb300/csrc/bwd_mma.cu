@@ -75,7 +75,8 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     extern __shared__ unsigned char smem_raw[];
     __shared__ unsigned long long bars[4];        // V (first batch), K~, V (second batch), tile rows
     // !SV: rung dp, ddp of each warp's tile rows.  SV: p (replaced by dS once
-    // known) and sd of each active rung (list order) and tile row.
+    // known) and sd (replaced by the row's dL/dd_k term once known) of each
+    // active rung (list order) and tile row.
     constexpr int kXs = SV ? 2 * kMmaMaxRungs * kMmaTile : kWarps * kMmaMaxRungs * 16 * 2;
     __shared__ __align__(16) float xs[kXs];
     auto dps = reinterpret_cast<float (*)[kMmaMaxRungs][16][2]>(xs);
@@ -416,7 +417,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             const bool up = c4 >= 2;
             const int row = wrel + g4 + (up ? 8 : 0);
             const bool rv = up ? vhi : vlo;
-            float ds[2];
+            float ds[2], gr[2];
 #pragma unroll
             for (int u = 0; u < 2; ++u) {
                 const float w = L.act_w[ib[u]], w1 = 1.f - w;
@@ -437,21 +438,17 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 const float e = dp - (up ? dlt_hi : dlt_lo);
                 emax_row = fmaxf(emax_row, fabsf(e));
                 ds[u] = p * e;
-                if constexpr (DD) {
+                if constexpr (DD) {               // the row's dL/dd_k term, summed over the tile at the end
                     const float sd = rv ? psd[1][ib[u]][row] : 0.f;
-                    float g = (c4 & 1) == 0 ? p * fmaf(s.scale * sd, e, ddp) : 0.f;
-                    g += __shfl_xor_sync(0xffffffffu, g, 2);
-                    g += __shfl_xor_sync(0xffffffffu, g, 4);
-                    g += __shfl_xor_sync(0xffffffffu, g, 8);
-                    g += __shfl_xor_sync(0xffffffffu, g, 16);
-                    if (lane == 0) gsm[warp][L.act_k[ib[u]]] = g;
+                    gr[u] = p * fmaf(s.scale * sd, e, ddp);
                 }
             }
-            __syncwarp();                         // the quad has read p before it is replaced
+            __syncwarp();                         // the quad has read p (and sd) before they are replaced
             if ((c4 & 1) == 0 && rv) {
 #pragma unroll
                 for (int u = 0; u < 2; ++u) {
                     psd[0][ib[u]][row] = ds[u];
+                    if constexpr (DD) psd[1][ib[u]][row] = gr[u];
                     DSg[(size_t)(s.W + 1 + L.act_k[ib[u]]) * s.T + bw + g4 + (up ? 8 : 0)] = ds[u];
                 }
             }
@@ -602,7 +599,11 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             if (vlo) { if (!SV) Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
             if (vhi) { if (!SV) Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
         }
-        if (lane == 0) gsm[warp][L.act_k[i]] = 0.f;
+        if constexpr (SV) {
+            if (DD && lane < kRowsPerWarp) psd[1][i][wrel + lane] = 0.f;   // no dL/dd_k term
+        } else {
+            if (lane == 0) gsm[warp][L.act_k[i]] = 0.f;
+        }
     }
     // ---- rungs: scores, p, dS, dL/dd_k (SV: dS from the value phase);
     // dq~ += dShat_k K~_slab.  SV: two rungs per iteration (the second's dS
@@ -759,8 +760,26 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
             *reinterpret_cast<unsigned*>(row + 8 * n + 2 * c4) = pack_bf16(dq[n][2 * half], dq[n][2 * half + 1]);
     }
 
-    // ---- per-CTA rung partials, warps summed in a fixed order
-    if constexpr (DD) {
+    // ---- per-CTA rung partials, summed in a fixed order
+    if constexpr (DD && SV) {
+        // the tile rows' terms of active rung i are in psd[1][i][0..119] (0
+        // for rows past T and rungs a warp does not attend): warp w sums list
+        // entries 2w and 2w+1 (lane l: rows l, l+32, l+64, l+96, then a
+        // butterfly over the lanes); inactive rungs get a zero partial
+        __syncthreads();
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int i = 2 * warp + u;
+            if (i >= L.n_act) break;
+            float x = 0.f;
+#pragma unroll
+            for (int r = lane; r < kMmaTile; r += 32) x += psd[1][i][r];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+            if (lane == 0) a.rpart[(size_t)L.act_k[i] * a.nblk_q + blockIdx.x] = __float2ll_rn(x * 4294967296.0f);
+        }
+        if (tid < a.r.K && !((a.r.active >> tid) & 1u)) a.rpart[(size_t)tid * a.nblk_q + blockIdx.x] = 0;
+    } else if constexpr (DD) {                    // warps summed in a fixed order
         __syncthreads();
         float x = 0.f;
         if (tid < a.r.K && ((a.r.active >> tid) & 1u))
