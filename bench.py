@@ -268,9 +268,15 @@ def step_method_bytes():
 # file of the kernel changes, the figure is reported as null until the next
 # capture.
 NCU_TRAFFIC = {
-    "bwd_query_mma": {"bytes_at_b32": 165859328 + 35686912,
+    "bwd_query_mma": {"bytes_at_b32": 165825792 + 34679552,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "c6aaa7b76693a7c57d07d9a1f5b35a29b60580b7b86101a0f829cf0d6ddda1af"},
+                      "sha256": "8c87f25753a0bf1af367fd7d43247404126f93efb5e403373766b7fbb0a98248"},
+    "bwd_key_mma": {"bytes_at_b32": 104573952 + 36702976,
+                    "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
+                    "sha256": "21a88a9dc0afab090cf199306b01f512490be9075bbb179fbc11a9f01fbbe04f"},
+    "fwd": {"bytes_at_b32": 100815360 + 57420288,
+            "sources": ("fwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
+            "sha256": "bc880c4077ef7aa6a99fd1523b6e3d6c2b97569bece22f7d4165c8275a1c26c2"},
 }
 
 
@@ -811,7 +817,8 @@ def ncu_case(which: str):
     than L2), one forward (and backward) per layer after one warm-up pass, the
     path the bench times: the forward keeps its rotated keys and residuals,
     the backward reads them (per layer and pass: RoPE of k, forward, query
-    pass, key pass)."""
+    pass, key pass).  `fwd_plain`: the forward alone without residuals (the
+    forward-only workload, alpha 0.9 in both layers)."""
     import __graft_entry__
     __graft_entry__.build()
     import paper_2606_28560_gb300 as fa
@@ -827,6 +834,9 @@ def ncu_case(which: str):
         bufs.append(ts + [fa.residuals_like(ts[0], W, K), fa.rotated_k_like(ts[1])])
     for rep in range(2):
         for l, (q, k, v, g, res, rk) in enumerate(bufs):
+            if which == "fwd_plain":
+                fa.fwd(q, k, v, 0.9, f, W, rotated_k=rk)
+                continue
             out, lse = fa.fwd(q, k, v, 0.8 + 0.1 * l, f, W, residuals=res, rotated_k=rk)
             if which == "bwd":
                 fa.bwd(q, k, v, lse, g, 0.8 + 0.1 * l, f, W, out=out, residuals=res, rotated_k=rk)
@@ -843,7 +853,7 @@ def main():
     ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--ncu-case", choices=["fwd", "bwd"], default=None,
+    ap.add_argument("--ncu-case", choices=["fwd", "fwd_plain", "bwd"], default=None,
                     help="run a small fixed case for an ncu capture and exit")
     args = ap.parse_args()
     if args.ncu_case:
