@@ -480,11 +480,12 @@ def run_gpu(args, rank, world, device):
     recompute["residuals_speedup"] = round(recompute["ms_per_step"] / recompute["residuals_ms_per_step"], 3)
 
     gqa = run_gqa_forward(wl, device, args, stream)
+    configs = run_configs(device, args, stream)
     e2e = run_e2e(args, wl, device, dist)
     stack = run_autograd_stack(device)
     return dict(value=value, ms=ms_max, clk=clk, dom=dom, achieved=achieved, hbm=hbm, peak_kind=peak_kind,
                 algo=algo, over=over, kernels=kernels, fwd_sweep=fwd_sweep, e2e=e2e, launches=launches_per_step * args.steps,
-                stack=stack, integer=integer, gqa=gqa, recompute=recompute,
+                stack=stack, integer=integer, gqa=gqa, configs=configs, recompute=recompute,
                 median_ms=step_ms[len(step_ms) // 2], min_ms=step_ms[0], max_ms=step_ms[-1])
 
 
@@ -547,6 +548,81 @@ def run_gqa_forward(wl, device, args, stream):
             out["fwd_bwd_ms_per_step"] = round(ms, 4)
             out["fwd_bwd_query_heads_per_s"] = round(B * H * T * L / (ms * 1e-3), 1)
     del kv
+    return out
+
+
+def run_configs(device, args, stream):
+    """The long-sequence workloads, 16 layers of distinct buffers, graphed
+    (RoPE of k included): T = 4096 extrapolation (B4 H8 W10, coprime
+    stagger), forward alone; T = 16384 stress (B2 H8 W12, linear stagger),
+    forward alone and forward + backward with residuals, for the Fibonacci
+    (K = 15) and the power-of-2 (K = 10) base."""
+    import paper_2606_28560_gb300 as fa
+    from paper_2606_28560_gb300 import inputs
+    hbm = peaks()[0]
+    out = {}
+    cases = (("T4096_B4_W10_coprime_fib", 4, 4096, 10, "coprime", "fib", 15, False),
+             ("T16384_B2_W12_linear_fib", 2, 16384, 12, "linear", "fib", 15, True),
+             ("T16384_B2_W12_linear_pow2", 2, 16384, 12, "linear", "pow2", 10, True))
+    for name, Bc, Tc, Wc, sched, base, Kc, bwd in cases:
+        alphas = [float(a) for a in fa.alpha_schedule(sched, L)]
+        f = fa.base(base, Kc)
+        shp = (Bc, H, Tc, D)
+        bf = torch.bfloat16
+        lay = []
+        for l in range(L):
+            ts = [torch.empty(shp, dtype=bf, device=device) for _ in range(4)]
+            for j, t in enumerate(ts):
+                inputs.device_normal_(t, 7000 + 10 * l + j)
+            lay.append({"q": ts[0], "k": ts[1], "v": ts[2], "g": ts[3], "o": torch.empty_like(ts[0]),
+                        "lse": torch.empty((Bc, H, Tc), dtype=torch.float32, device=device),
+                        "rk": torch.empty(shp, dtype=torch.float16, device=device),
+                        "res": fa.residuals_like(ts[0], Wc, Kc) if bwd else None,
+                        "dq": torch.empty_like(ts[0]), "dk": torch.empty_like(ts[0]), "dv": torch.empty_like(ts[0])})
+        ws_f = torch.empty(fa.fwd_workspace_bytes(Bc, H, Tc, Wc, Kc, bf), dtype=torch.uint8, device=device)
+        ws_b = torch.empty(fa.bwd_workspace_bytes(Bc, H, Tc, Wc, Kc, bf), dtype=torch.uint8, device=device)
+        dth = torch.zeros((L, 4), dtype=torch.float32, device=device)
+
+        def fwd_all(res=False):
+            for l, c in enumerate(lay):
+                fa.fwd(c["q"], c["k"], c["v"], alphas[l], f, Wc, out=c["o"], lse=c["lse"], workspace=ws_f,
+                       rotated_k=c["rk"], residuals=c["res"] if res else None)
+
+        def step():
+            fwd_all(True)
+            for l in reversed(range(L)):
+                c = lay[l]
+                fa.bwd(c["q"], c["k"], c["v"], c["lse"], c["g"], alphas[l], f, Wc, out=c["o"], dq=c["dq"],
+                       dk=c["dk"], dv=c["dv"], dtheta=dth[l], workspace=ws_b, rotated_k=c["rk"],
+                       residuals=c["res"])
+
+        r = {"B": Bc, "H": H, "T": Tc, "W": Wc, "K": Kc, "schedule": sched, "base": base}
+        for what, fn in (("fwd", fwd_all), ("fwd_bwd", step)) if bwd else (("fwd", fwd_all),):
+            fn()
+            torch.cuda.synchronize(device)
+            g = capture(fn, device, profile=False)
+            g.replay()
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            reps = 3
+            a0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            a1.record(stream)
+            torch.cuda.synchronize(device)
+            ms = a0.elapsed_time(a1) / reps
+            del g
+            qh = Bc * H * Tc * L
+            if what == "fwd":
+                r["fwd_layer_us_incl_rope"] = round(ms / L * 1e3, 2)
+                r["fwd_query_heads_per_s"] = round(qh / (ms * 1e-3), 1)
+                r["fwd_frac_of_hbm"] = round(qh * 4 * ROW_BYTES / (ms * 1e-3) / 1e9 / hbm, 4)
+            else:
+                r["fwd_bwd_ms_per_step"] = round(ms, 4)
+                r["fwd_bwd_query_heads_per_s"] = round(qh / (ms * 1e-3), 1)
+                r["step_frac_of_hbm"] = round(qh * 12 * ROW_BYTES / (ms * 1e-3) / 1e9 / hbm, 4)
+        out[name] = r
+        del lay, ws_f, ws_b
+        torch.cuda.empty_cache()
     return out
 
 
@@ -908,6 +984,7 @@ def main():
             "integer_vs_interpolated_16_layers": r["integer"],
             "backward_recomputing_scores_16_layers": r["recompute"],
             "forward_gqa_16_layers": r["gqa"],
+            "long_sequence_16_layers": r["configs"],
             "cpu_baseline": cpu,
             "cpu_oracle_per_config": cpu_configs,
             "e2e": r["e2e"],
