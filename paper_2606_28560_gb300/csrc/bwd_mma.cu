@@ -316,7 +316,6 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
 
     // ---- window band dp = dO . v
     float dpw[NT][4];
-#pragma unroll
     {
         const unsigned ab = row_chunk(sbase, L.win_smem + wrel - Wp + (lane & 7), lane >> 3);
 #pragma unroll
