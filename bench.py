@@ -270,7 +270,7 @@ def step_method_bytes():
 NCU_TRAFFIC = {
     "bwd_query_mma": {"bytes_at_b32": 165825792 + 34679552,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "8c87f25753a0bf1af367fd7d43247404126f93efb5e403373766b7fbb0a98248"},
+                      "sha256": "51f0558f106fb85115ab0551659fef3350ac120753bdc736fc6dcba9a89d5386"},
     "bwd_key_mma": {"bytes_at_b32": 104573952 + 36702976,
                     "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
                     "sha256": "21a88a9dc0afab090cf199306b01f512490be9075bbb179fbc11a9f01fbbe04f"},
