@@ -9,25 +9,29 @@
 //   window band  S = Q~ K~[b-Wp, b+16)^T   (16 x (16+Wp), the causal band t=0..W)
 //   rung k       S = Q~ K~[b-s0-1, +16)^T (16 x 16; the diagonal and the first
 //                superdiagonal are the far and floor scores)
-// The interpolated rung score (1-w) S[u][u+1] + w S[u][u] is summed inside the
-// quad of lanes that share a row.  Softmax is two-pass in registers (row max,
-// then P); the probability-weighted values are again 16x8 MMAs:
+// The interpolated rung score (1-w) S[u][u+1] + w S[u][u] is held by at most
+// two lanes of the quad that shares a row (one shuffle between them).  The q~
+// fragments carry scale * log2(e), so scores are in log2 units.  Softmax is
+// two-pass in registers (row max, then P = 2^(s - max)); the
+// probability-weighted values are again 16x8 MMAs:
 //   window band  O += P_band V[b-Wp, b+16)
 //   rung k       O += Phat_k V[b-s0-1, +16),  Phat_k[u][u] = p w, Phat_k[u][u+1] = p (1-w)
+// and one more MMA per k-step against a B fragment of ones gives the row sums.
 //
 // Precision (bf16 I/O): q~ and k~ enter the score MMAs as fp16 (11-bit
 // significands); P of the window band is the unnormalised exp(s - max) in
 // bf16, so the largest entry of each row is exactly 1; the entries p w and
-// p (1-w) of a rung's Phat are rounded to bf16 the same way.  Row sums use the
-// same rounded values, so each output is a normalised average of the values.
-// Accumulation is fp32.
+// p (1-w) of a rung's Phat are rounded to bf16 the same way.  Row sums add
+// the same rounded values, so each output is a normalised average of the
+// values.  Accumulation is fp32.
 //
 // Staging: the CTA's union of key rows (rotated keys, fp16) and then of value
 // rows (bf16, same buffer) is copied by TMA (3-D tensor maps [heads][T][64],
 // 64-row boxes with 8-row tails, 128-byte swizzle, rows outside [0, T)
-// zero-filled) under an mbarrier with a bounded wait.  The one-head form
-// writes its output rows (and the rotated query rows it keeps) through a
-// 1 KB stage per warp, as 16-byte pieces of runs of consecutive rows.
+// zero-filled) under mbarriers with bounded waits; the value copies are
+// issued by the last warp done with the keys.  The one-head form writes its
+// output rows (and the rotated query rows it keeps) through a 1 KB stage per
+// warp, as 16-byte pieces of runs of consecutive rows.
 #include <cmath>
 
 #include <cuda.h>
