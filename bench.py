@@ -264,28 +264,36 @@ def step_method_bytes():
 # DRAM traffic (dram__bytes_read.sum + dram__bytes_write.sum) of one launch,
 # from an `ncu --set full` capture of `bench.py --ncu-case bwd` (B=32, the same
 # H, T, D, W); every launch reads and writes each of its tensors once, so the
-# bytes scale with B.  The counters belong to the sources hashed here: once a
-# file of the kernel changes, the figure is reported as null until the next
-# capture.
+# bytes scale with B.  The counters belong to the sources hashed here (code
+# lines only: comments and blank lines are left out): once the code of a file
+# of the kernel changes, the figure is reported as null until the next capture.
 NCU_TRAFFIC = {
     "bwd_query_mma": {"bytes_at_b32": 165825792 + 34679552,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "51f0558f106fb85115ab0551659fef3350ac120753bdc736fc6dcba9a89d5386"},
+                      "sha256": "f3e380549fe08580763e30a83c4597006e04b021d73b1c542397d022ae41d76d"},
     "bwd_key_mma": {"bytes_at_b32": 104573952 + 36702976,
                     "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                    "sha256": "21a88a9dc0afab090cf199306b01f512490be9075bbb179fbc11a9f01fbbe04f"},
+                    "sha256": "32dace1d003ef050369134c7d28b6fb8347d93f8f406c1724acda85747d9f8d2"},
     "fwd": {"bytes_at_b32": 100815360 + 57420288,
             "sources": ("fwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-            "sha256": "bc880c4077ef7aa6a99fd1523b6e3d6c2b97569bece22f7d4165c8275a1c26c2"},
+            "sha256": "89c6cf5cfae09e48d5d393d2941e24d5eb772188af3f4eb283e5994bfb45cc54"},
 }
 
 
 def sources_sha256(names) -> str:
+    """sha256 over the code lines of the named kernel sources (// and /* */
+    comments, trailing blanks and empty lines removed; the sources hold no
+    string literal with a comment marker)."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for n in names:
-        with open(os.path.join(ROOT, "paper_2606_28560_gb300", "csrc", n), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, "paper_2606_28560_gb300", "csrc", n), encoding="utf-8") as fh:
+            text = re.sub(r"/\*.*?\*/", "", fh.read(), flags=re.S)
+        for line in text.splitlines():
+            line = line.split("//", 1)[0].rstrip()
+            if line:
+                h.update(line.encode() + b"\n")
     return h.hexdigest()
 
 
