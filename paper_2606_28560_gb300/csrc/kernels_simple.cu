@@ -68,42 +68,59 @@ __global__ void __launch_bounds__(256) rope_rows_kernel(const T* __restrict__ sr
     }
 }
 
-// bf16 rows in, fp16 rotated rows out.  Thread item = (group of kRopeHeads
-// heads, position, chunk): the 8 angles of the chunk's pairs are evaluated
-// once and applied to that position's row in each head of the group; the
-// rows' loads are all issued before any arithmetic.  A warp covers 8
-// consecutive positions x 4 chunks of one head per access: 1 KB contiguous.
-// One head per item measured fastest in the 16-layer training step (2.361 ms
-// with 4 heads, 2.331 with 2, 2.318 with 1): fewer registers per thread, more
-// resident warps and more loads in flight outweigh the repeated angles.
-constexpr int kRopeHeads = 1;
+// bf16 rows in, fp16 rotated rows out.  A block tile is kRopePos consecutive
+// positions of kRopeTileHeads heads: the tile's cos/sin (one pair and
+// position per thread, evaluated before the wait for the previous kernel)
+// go to shared memory, and every row of the tile reads them from there, so
+// an angle is evaluated once per tile instead of once per head.  Thread item
+// = (head, position, chunk c): dims 8c..8c+7 and their RoPE partners
+// 32+8c..32+8c+7; a warp covers the tile's 8 positions x 4 chunks of one
+// head (1 KB contiguous), and a thread issues the loads of all its items
+// before any arithmetic.
+constexpr int kRopePos = 8, kRopeTileHeads = 16;
+constexpr int kRopeItems = kRopePos * kRopeTileHeads * 4 / 256;   // per thread (256 threads)
+constexpr int kRopeTabStride = 34;            // floats per position (32 + pad: conflict-free float2 reads)
 __global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16* __restrict__ src,
                                                              __half* __restrict__ dst, int heads, int T_,
                                                              RopeParams rp, unsigned* status) {
-    grid_dependency_sync();
+    __shared__ __align__(16) float ctab[kRopePos * kRopeTabStride], stab[kRopePos * kRopeTabStride];
+    const int tid = threadIdx.x;
+    const int c = tid & 3, pr = (tid >> 2) & 7, hr0 = tid >> 5;
+    const int tiles_p = (T_ + kRopePos - 1) / kRopePos;
+    const long long tiles = (long long)tiles_p * ((heads + kRopeTileHeads - 1) / kRopeTileHeads);
     float rmax = 0.f;                             // largest |rotated entry|: fp16 holds < 65520
-    const int groups = (heads + kRopeHeads - 1) / kRopeHeads;
-    const long long n = (long long)groups * T_ * 4;
-    for (long long g = blockIdx.x * (long long)blockDim.x + threadIdx.x; g < n;
-         g += (long long)gridDim.x * blockDim.x) {
-        const int c = (int)(g & 3);
-        const long long pg = g >> 2;
-        const int p = (int)(pg % T_), h0 = (int)(pg / T_) * kRopeHeads;
-        uint4 raw[kRopeHeads][2];
+    bool waited = false;
+    for (long long tile = blockIdx.x; tile < tiles; tile += gridDim.x) {
+        const int tp = (int)(tile % tiles_p), th = (int)(tile / tiles_p);
+        const int p0 = tp * kRopePos, h0 = th * kRopeTileHeads;
+        {                                         // pair m = tid & 31 at position p0 + (tid >> 5)
+            float cs, sn;
+            rope_cs(rp, tid & 31, p0 + (tid >> 5), cs, sn);
+            ctab[(tid >> 5) * kRopeTabStride + (tid & 31)] = cs;
+            stab[(tid >> 5) * kRopeTabStride + (tid & 31)] = sn;
+        }
+        if (!waited) {
+            grid_dependency_sync();
+            waited = true;
+        }
+        const int p = p0 + pr;
+        uint4 raw[kRopeItems][2];
 #pragma unroll
-        for (int u = 0; u < kRopeHeads; ++u) {
-            if (h0 + u < heads) {
-                const __nv_bfloat16* row = src + ((size_t)(h0 + u) * T_ + p) * kHeadDim;
+        for (int u = 0; u < kRopeItems; ++u) {
+            const int h = h0 + hr0 + 8 * u;
+            if (h < heads && p < T_) {
+                const __nv_bfloat16* row = src + ((size_t)h * T_ + p) * kHeadDim;
                 raw[u][0] = *reinterpret_cast<const uint4*>(row + 8 * c);
                 raw[u][1] = *reinterpret_cast<const uint4*>(row + kHalf + 8 * c);
             }
         }
-        float cs[8], sn[8];
+        __syncthreads();                          // the tile's cos/sin are in shared memory
+        const float2* cp = reinterpret_cast<const float2*>(ctab + pr * kRopeTabStride + 8 * c);
+        const float2* sp = reinterpret_cast<const float2*>(stab + pr * kRopeTabStride + 8 * c);
 #pragma unroll
-        for (int e = 0; e < 8; ++e) rope_cs(rp, 8 * c + e, p, cs[e], sn[e]);
-#pragma unroll
-        for (int u = 0; u < kRopeHeads; ++u) {
-            if (h0 + u >= heads) break;
+        for (int u = 0; u < kRopeItems; ++u) {
+            const int h = h0 + hr0 + 8 * u;
+            if (h >= heads || p >= T_) continue;
             const unsigned* wa = reinterpret_cast<const unsigned*>(&raw[u][0]);
             const unsigned* wb = reinterpret_cast<const unsigned*>(&raw[u][1]);
             unsigned oa[4], ob[4];
@@ -111,20 +128,22 @@ __global__ void __launch_bounds__(256) rope_rows_bf16_kernel(const __nv_bfloat16
             for (int e = 0; e < 4; ++e) {
                 const float a0 = __uint_as_float(wa[e] << 16), a1 = __uint_as_float(wa[e] & 0xffff0000u);
                 const float b0 = __uint_as_float(wb[e] << 16), b1 = __uint_as_float(wb[e] & 0xffff0000u);
-                const int m0 = 2 * e, m1 = 2 * e + 1;        // pairs (8c + m, 32 + 8c + m)
-                const float xa0 = a0 * cs[m0] - b0 * sn[m0], xa1 = a1 * cs[m1] - b1 * sn[m1];
-                const float xb0 = b0 * cs[m0] + a0 * sn[m0], xb1 = b1 * cs[m1] + a1 * sn[m1];
+                const float2 ce = cp[e], se = sp[e];         // pairs (8c + 2e, 32 + 8c + 2e) and the next
+                const float xa0 = a0 * ce.x - b0 * se.x, xa1 = a1 * ce.y - b1 * se.y;
+                const float xb0 = b0 * ce.x + a0 * se.x, xb1 = b1 * ce.y + a1 * se.y;
                 rmax = fmaxf(rmax, fmaxf(fmaxf(fabsf(xa0), fabsf(xa1)), fmaxf(fabsf(xb0), fabsf(xb1))));
                 __half2 ra = __floats2half2_rn(xa0, xa1);
                 __half2 rb = __floats2half2_rn(xb0, xb1);
                 oa[e] = *reinterpret_cast<unsigned*>(&ra);
                 ob[e] = *reinterpret_cast<unsigned*>(&rb);
             }
-            __half* row = dst + ((size_t)(h0 + u) * T_ + p) * kHeadDim;
+            __half* row = dst + ((size_t)h * T_ + p) * kHeadDim;
             *reinterpret_cast<uint4*>(row + 8 * c) = make_uint4(oa[0], oa[1], oa[2], oa[3]);
             *reinterpret_cast<uint4*>(row + kHalf + 8 * c) = make_uint4(ob[0], ob[1], ob[2], ob[3]);
         }
+        __syncthreads();                          // read before the next tile rewrites them
     }
+    if (!waited) grid_dependency_sync();
     if (rmax >= 65520.f) raise_status(status, kStatusRange);
 }
 
@@ -461,23 +480,11 @@ cudaError_t launch_rope_rows(const void* src, void* dst, long long rows, int T, 
     if (grid > 152 * 16) grid = 152 * 16;       // 16 resident 256-thread blocks on each of 152 SMs
     if (bf16) {
         const int heads = (int)(rows / T);
-        // one wave: as many blocks as are resident at once (a partial second
-        // wave would run on a nearly idle GPU); the grid-stride loop spreads
-        // the remainder over every SM
-        const long long gitems = (long long)((heads + kRopeHeads - 1) / kRopeHeads) * T * 4;
-        static int wave = 0;
-        if (wave == 0) {
-            int dev = 0, sms = 0, per_sm = 0;
-            if (cudaGetDevice(&dev) == cudaSuccess &&
-                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess &&
-                cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, rope_rows_bf16_kernel, 256, 0) == cudaSuccess &&
-                sms > 0 && per_sm > 0)
-                wave = sms * per_sm;
-            else
-                wave = 152 * 3;
-        }
-        long long g2 = (gitems + 255) / 256;
-        if (g2 > wave) g2 = wave;
+        // one tile per block: the hardware hands the blocks to the SMs as
+        // they free up, which balances the load better than a grid-stride loop
+        const long long tiles = (long long)((T + kRopePos - 1) / kRopePos) *
+                                ((heads + kRopeTileHeads - 1) / kRopeTileHeads);
+        const long long g2 = tiles < 0x7fffffffLL ? tiles : 0x7fffffffLL;
         return launch_kernel(rope_rows_bf16_kernel, dim3((unsigned)g2), dim3(256), 0, st,
                              reinterpret_cast<const __nv_bfloat16*>(src), reinterpret_cast<__half*>(dst), heads, T,
                              rp, status);
