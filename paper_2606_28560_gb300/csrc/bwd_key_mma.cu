@@ -73,7 +73,7 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
             const int t = x - r;                              // query - key
             const int q = bw + x;
             const bool use = (hi ? vhi : vlo) && t >= 0 && t <= s.W && q < s.T;
-            bv[j][e] = use ? X[(size_t)t * s.T + q] : 0.f;
+            bv[j][e] = use ? X[(unsigned)(t * s.T + q)] : 0.f;
         }
     float rvv[kMmaMaxRungs * 16 / 32];
 #pragma unroll
@@ -82,7 +82,7 @@ __device__ __forceinline__ void key_pass(float (&acc)[8][4], const float* X, con
         const int i = u >> 4, x = u & 15;
         const int q = bw + L.act_s0[i] + x;
         const bool use = i < L.n_act && q < s.T;
-        rvv[j] = use ? X[(size_t)(s.W + 1 + L.act_k[i]) * s.T + q] : 0.f;
+        rvv[j] = use ? X[(unsigned)((s.W + 1 + L.act_k[i]) * s.T + q)] : 0.f;
     }
     if (IL) {
         asm volatile("cp.async.wait_group 0;\n" ::: "memory");

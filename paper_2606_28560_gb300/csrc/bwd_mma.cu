@@ -146,7 +146,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 const bool hi = e >= 2;
                 const int r = hi ? g4 + 8 : g4;
                 const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
-                pb[j][e] = ((hi ? vhi : vlo) && t >= 0 && t <= s.W) ? Pg[(size_t)t * s.T + bw + r] : 0.f;
+                pb[j][e] = ((hi ? vhi : vlo) && t >= 0 && t <= s.W) ? Pg[(unsigned)(t * s.T + bw + r)] : 0.f;
             }
         const float* SDg = DD ? a.res_sd + (size_t)bh * a.r.K * s.T : nullptr;
         for (int u = tid; u < L.n_act * kMmaTile; u += kWarps * 32) {
@@ -353,7 +353,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 const int r = hi ? g4 + 8 : g4;
                 const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
                 dsb[j][e] = pb[j][e] * (hi ? il_hi : il_lo) * (dpw[j][e] - (hi ? dlt_hi : dlt_lo));
-                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) DSg[(size_t)t * s.T + bw + r] = dsb[j][e];
+                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) DSg[(unsigned)(t * s.T + bw + r)] = dsb[j][e];
             }
         }
     }
@@ -448,7 +448,7 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                 for (int u = 0; u < 2; ++u) {
                     psd[0][ib[u]][row] = ds[u];
                     if constexpr (DD) psd[1][ib[u]][row] = gr[u];
-                    DSg[(size_t)(s.W + 1 + L.act_k[ib[u]]) * s.T + bw + g4 + (up ? 8 : 0)] = ds[u];
+                    DSg[(unsigned)((s.W + 1 + L.act_k[ib[u]]) * s.T + bw + g4 + (up ? 8 : 0))] = ds[u];
                 }
             }
         }
@@ -595,8 +595,9 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     for (int i = n_use; i < L.n_act; ++i) {
         const int slot = s.W + 1 + L.act_k[i];
         if (c4 == 0) {                            // (SV: the forward wrote p = 0 there)
-            if (vlo) { if (!SV) Pg[(size_t)slot * s.T + qlo] = 0.f; DSg[(size_t)slot * s.T + qlo] = 0.f; }
-            if (vhi) { if (!SV) Pg[(size_t)slot * s.T + qhi] = 0.f; DSg[(size_t)slot * s.T + qhi] = 0.f; }
+            const unsigned o = (unsigned)(slot * s.T + qlo);
+            if (vlo) { if (!SV) Pg[o] = 0.f; DSg[o] = 0.f; }
+            if (vhi) { if (!SV) Pg[o + 8] = 0.f; DSg[o + 8] = 0.f; }
         }
         if constexpr (SV) {
             if (DD && lane < kRowsPerWarp) psd[1][i][wrel + lane] = 0.f;   // no dL/dd_k term

@@ -340,6 +340,10 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 
     // ---- rung scores (log2 units) of the rows this lane takes part in
     const float inv_sc2 = 1.f / sc2;
+    // SAVE: the residual arrays of this head, addressed by 32-bit offsets
+    // (S T and K T stay below 2^31); row qhi = qlo + 8 is 8 entries on
+    float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;   // residual exp(s - max) per slot
+    float* SDg = SAVE ? a.res_sd + (size_t)bh * a.r.K * s.T : nullptr;
     float rs[kMmaMaxRungs][2];
     // rung i of the list sorted by d (i < n_use)
     auto score_rung = [&](int i) {
@@ -376,9 +380,9 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
             sdl += __shfl_sync(0xffffffffu, sdl, src);
             sdh += __shfl_sync(0xffffffffu, sdh, src);
             if (writer) {
-                float* sd = a.res_sd + ((size_t)bh * a.r.K + L.act_k[i]) * s.T;
-                if (vlo) sd[qlo] = sdl * inv_sc2;
-                if (vhi) sd[qhi] = sdh * inv_sc2;
+                float* sd = SDg + (unsigned)(L.act_k[i] * s.T + qlo);
+                if (vlo) sd[0] = sdl * inv_sc2;
+                if (vhi) sd[8] = sdh * inv_sc2;
             }
         }
     };
@@ -409,7 +413,10 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     if (mlo == -INFINITY) mlo = 0.f;              // rows beyond T: keep arithmetic finite
     if (mhi == -INFINITY) mhi = 0.f;
     unsigned pa[NT][2];                           // window band P as bf16 A fragments
-    float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;   // residual exp(s - max) per slot
+    // SAVE: entry (j, e) of the band is row g4 + 8 (e >> 1), slot
+    // t = tb + 8 (e >> 1) - 8 j - (e & 1), at offset t T + bw + row
+    const int tb = g4 + Wp - 2 * c4;
+    const int pband = tb * s.T + bw + g4;
 #pragma unroll
     for (int j = 0; j < NT; ++j) {
         const float e0 = ex2(sw[j][0] - mlo), e1 = ex2(sw[j][1] - mlo);
@@ -421,9 +428,10 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
                 const bool hi = e >= 2;
-                const int r = hi ? g4 + 8 : g4;
-                const int t = r + Wp - (8 * j + 2 * c4 + (e & 1));
-                if ((hi ? vhi : vlo) && t >= 0 && t <= s.W) Pg[(size_t)t * s.T + bw + r] = ev[e];
+                const int dt = (hi ? 8 : 0) - 8 * j - (e & 1);
+                const int t = tb + dt;
+                if ((hi ? vhi : vlo) && (unsigned)t <= (unsigned)s.W)
+                    Pg[(unsigned)(pband + dt * s.T + (hi ? 8 : 0))] = ev[e];
             }
         }
     }
@@ -433,9 +441,9 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         // tail of the list sorted by d): 0
         if (c4 == 0) {
             for (int i = n_use; i < L.n_act; ++i) {
-                float* row = Pg + (size_t)(s.W + 1 + L.act_k[i]) * s.T;
-                if (vlo) row[qlo] = 0.f;
-                if (vhi) row[qhi] = 0.f;
+                float* row = Pg + (unsigned)((s.W + 1 + L.act_k[i]) * s.T + qlo);
+                if (vlo) row[0] = 0.f;
+                if (vhi) row[8] = 0.f;
             }
         }
     }
@@ -487,9 +495,9 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         const float plo = ex2(rs[i][0] - mlo), phi = ex2(rs[i][1] - mhi);   // 0 when masked
         if constexpr (SAVE) {
             if (writer) {                         // residual p of the rung
-                float* row = Pg + (size_t)(s.W + 1 + L.act_k[i]) * s.T;
-                if (vlo) row[qlo] = plo;
-                if (vhi) row[qhi] = phi;
+                float* row = Pg + (unsigned)((s.W + 1 + L.act_k[i]) * s.T + qlo);
+                if (vlo) row[0] = plo;
+                if (vhi) row[8] = phi;
             }
         }
         // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
