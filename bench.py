@@ -268,15 +268,15 @@ def step_method_bytes():
 # lines only: comments and blank lines are left out): once the code of a file
 # of the kernel changes, the figure is reported as null until the next capture.
 NCU_TRAFFIC = {
-    "bwd_query_mma": {"bytes_at_b32": 165825792 + 34679552,
+    "bwd_query_mma": {"bytes_at_b32": 165817600 + 34578944,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "f3e380549fe08580763e30a83c4597006e04b021d73b1c542397d022ae41d76d"},
-    "bwd_key_mma": {"bytes_at_b32": 104573952 + 36702976,
+                      "sha256": "f26ab4bf0a4909d64b35f8c4d74470c5c254896408b22636f16aabc43cf89a4c"},
+    "bwd_key_mma": {"bytes_at_b32": 104528640 + 36358400,
                     "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                    "sha256": "32dace1d003ef050369134c7d28b6fb8347d93f8f406c1724acda85747d9f8d2"},
-    "fwd": {"bytes_at_b32": 100815360 + 57420288,
+                    "sha256": "fa0f295cc49f2f2944012800d4c8fc99cdae1c71abb60604c1c90cbb78907148"},
+    "fwd": {"bytes_at_b32": 100784384 + 57288960,
             "sources": ("fwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-            "sha256": "89c6cf5cfae09e48d5d393d2941e24d5eb772188af3f4eb283e5994bfb45cc54"},
+            "sha256": "996f0724b47aa24f6cc37ec5f4f9d0d368dd99c76ee8367593b9bd1f118fc02a"},
 }
 
 
