@@ -448,6 +448,22 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
         }
     }
 
+    // rung probabilities (and their residuals) while the values arrive: the
+    // rung scores become p = 2^(s - max) in place
+#pragma unroll
+    for (int i = 0; i < kMmaMaxRungs; ++i) {
+        if (i >= n_use) break;
+        rs[i][0] = ex2(rs[i][0] - mlo);           // 0 when masked
+        rs[i][1] = ex2(rs[i][1] - mhi);
+        if constexpr (SAVE) {
+            if (writer) {                         // residual p of the rung
+                float* row = Pg + (unsigned)((s.W + 1 + L.act_k[i]) * s.T + qlo);
+                if (vlo) row[0] = rs[i][0];
+                if (vhi) row[8] = rs[i][1];
+            }
+        }
+    }
+
     const bool ok_v = mbar_wait(&bars[1], 0);
 
     // o: the value product; osum: the row sums of the same rounded weights
@@ -492,14 +508,7 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     // A-fragment columns of this thread: 2c4 + {0,1} (a0, a1) and 2c4 + 8 + {0,1} (a2, a3).
     auto value_rung = [&](int i) {
         const float w = L.act_w[i];
-        const float plo = ex2(rs[i][0] - mlo), phi = ex2(rs[i][1] - mhi);   // 0 when masked
-        if constexpr (SAVE) {
-            if (writer) {                         // residual p of the rung
-                float* row = Pg + (unsigned)((s.W + 1 + L.act_k[i]) * s.T + qlo);
-                if (vlo) row[0] = plo;
-                if (vhi) row[8] = phi;
-            }
-        }
+        const float plo = rs[i][0], phi = rs[i][1];
         // Phat in bf16 (a1, row g4+8 at columns 2c4.., is zero); the row sums
         // come from the same rounded entries (the ones product below)
         const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = fmaf(-m7, w, m7);
