@@ -274,9 +274,9 @@ NCU_TRAFFIC = {
     "bwd_key_mma": {"bytes_at_b32": 104528640 + 36358400,
                     "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
                     "sha256": "fa0f295cc49f2f2944012800d4c8fc99cdae1c71abb60604c1c90cbb78907148"},
-    "fwd": {"bytes_at_b32": 100784384 + 57288960,
+    "fwd": {"bytes_at_b32": 100805632 + 57507584,
             "sources": ("fwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-            "sha256": "996f0724b47aa24f6cc37ec5f4f9d0d368dd99c76ee8367593b9bd1f118fc02a"},
+            "sha256": "2f780130e04b0e375c268701fe84957643af88ee457a2fe6cf9a75df59879d68"},
 }
 
 
