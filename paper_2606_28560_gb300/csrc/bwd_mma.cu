@@ -33,6 +33,7 @@
 // bf16-autocast training step passes upstream gradients of 1e-5 .. 1e-8).
 // Accumulation is fp32.
 #include <cmath>
+#include <type_traits>
 
 #include "fibattn_internal.cuh"
 #include "fwd_mma.cuh"
@@ -382,20 +383,27 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
     // ---- rung dp (interpolated) and ddp = dp_far - dp_floor, to shared memory
     if constexpr (SV) {
         // Two rungs per iteration (their MMA and reduction chains are
-        // independent); with an odd count the last pair repeats its first rung,
-        // whose second copy reads and writes the same values.  Each lane tracks
-        // its row's largest |dp - Delta| (lanes c4 < 2: row g4, else g4 + 8).
+        // independent), the last of an odd count alone.  Each lane tracks its
+        // row's largest |dp - Delta| (lanes c4 < 2: row g4, else g4 + 8).
         float emax_row = 0.f;
-#pragma unroll 1
-        for (int i = 0; i < n_use; i += 2) {
-            const int ib[2] = {i, i + 1 < n_use ? i + 1 : i};
+        // per rung: this lane's shares of dp and ddp for rows g4 and g4+8,
+        // reduce-scattered over the quad (lanes c4 = 0, 1 end with row g4,
+        // lanes 2, 3 with row g4+8); lanes 0 and 2 then form their row's dS
+        // (from the residual p) and dL/dd_k term, the terms summed over the
+        // warp's rows in a fixed order; dS replaces p in shared memory for
+        // the key phase
+        const bool up = c4 >= 2;
+        const int row = wrel + g4 + (up ? 8 : 0);
+        const bool rv = up ? vhi : vlo;
+        auto value_block = [&](int i, auto nu) {  // NU rungs from list position i
+            constexpr int NU = decltype(nu)::value;
             release_above(L.act_iv[i]);
-            need_rows(L.act_smem[ib[0]] + wrel);
-            need_rows(L.act_smem[ib[1]] + wrel);
-            float dt[2][2][4];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const unsigned ak = row_chunk(sbase, L.act_smem[ib[u]] + wrel + (lane & 7), lane >> 3);
+            for (int u = 0; u < NU; ++u) need_rows(L.act_smem[i + u] + wrel);
+            float dt[NU][2][4];
+#pragma unroll
+            for (int u = 0; u < NU; ++u) {
+                const unsigned ak = row_chunk(sbase, L.act_smem[i + u] + wrel + (lane & 7), lane >> 3);
 #pragma unroll
                 for (int t = 0; t < 2; ++t) {
                     unsigned b0, b1, b2, b3;
@@ -407,19 +415,11 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                     mma_bf16_16816(dt[u][t], da[3], b2, b3);
                 }
             }
-            // per rung: this lane's shares of dp and ddp for rows g4 and g4+8,
-            // reduce-scattered over the quad (lanes c4 = 0, 1 end with row g4,
-            // lanes 2, 3 with row g4+8); lanes 0 and 2 then form their row's dS
-            // (from the residual p) and dL/dd_k term, the terms summed over the
-            // warp's rows in a fixed order; dS replaces p in shared memory for
-            // the key phase
-            const bool up = c4 >= 2;
-            const int row = wrel + g4 + (up ? 8 : 0);
-            const bool rv = up ? vhi : vlo;
-            float ds[2], gr[2];
+            float ds[NU];
+            [[maybe_unused]] float gr[NU];
 #pragma unroll
-            for (int u = 0; u < 2; ++u) {
-                const float w = L.act_w[ib[u]], w1 = 1.f - w;
+            for (int u = 0; u < NU; ++u) {
+                const float w = L.act_w[i + u], w1 = 1.f - w;
                 const float c0 = fmaf(ib0, w, ia0), c1 = fmaf(ib1, w, ia1), c7 = m7 * w1;
                 const float x0 = fmaf(c0, dt[u][0][0], fmaf(c1, dt[u][0][1], c7 * dt[u][1][0]));
                 const float x2 = fmaf(c0, dt[u][1][2], c1 * dt[u][1][3]);
@@ -428,30 +428,35 @@ bwd_query_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant_
                     x1 = fmaf(df0, dt[u][0][0], fmaf(df1, dt[u][0][1], -m7 * dt[u][1][0]));
                     x3 = fmaf(df0, dt[u][1][2], df1 * dt[u][1][3]);
                 }
-                float dp = up ? x2 : x0, ddp = up ? x3 : x1;
+                float dp = up ? x2 : x0;
+                [[maybe_unused]] float ddp = up ? x3 : x1;
                 dp += __shfl_xor_sync(0xffffffffu, up ? x0 : x2, 2);
                 if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, up ? x1 : x3, 2);
                 dp += __shfl_xor_sync(0xffffffffu, dp, 1);
                 if constexpr (DD) ddp += __shfl_xor_sync(0xffffffffu, ddp, 1);
-                const float p = rv ? psd[0][ib[u]][row] * (up ? il_hi : il_lo) : 0.f;
+                const float p = rv ? psd[0][i + u][row] * (up ? il_hi : il_lo) : 0.f;
                 const float e = dp - (up ? dlt_hi : dlt_lo);
                 emax_row = fmaxf(emax_row, fabsf(e));
                 ds[u] = p * e;
                 if constexpr (DD) {               // the row's dL/dd_k term, summed over the tile at the end
-                    const float sd = rv ? psd[1][ib[u]][row] : 0.f;
+                    const float sd = rv ? psd[1][i + u][row] : 0.f;
                     gr[u] = p * fmaf(s.scale * sd, e, ddp);
                 }
             }
             __syncwarp();                         // the quad has read p (and sd) before they are replaced
             if ((c4 & 1) == 0 && rv) {
 #pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    psd[0][ib[u]][row] = ds[u];
-                    if constexpr (DD) psd[1][ib[u]][row] = gr[u];
-                    DSg[(unsigned)((s.W + 1 + L.act_k[ib[u]]) * s.T + bw + g4 + (up ? 8 : 0))] = ds[u];
+                for (int u = 0; u < NU; ++u) {
+                    psd[0][i + u][row] = ds[u];
+                    if constexpr (DD) psd[1][i + u][row] = gr[u];
+                    DSg[(unsigned)((s.W + 1 + L.act_k[i + u]) * s.T + bw + g4 + (up ? 8 : 0))] = ds[u];
                 }
             }
-        }
+        };
+        int i = 0;
+#pragma unroll 1
+        for (; i + 1 < n_use; i += 2) value_block(i, std::integral_constant<int, 2>{});
+        if (i < n_use) value_block(i, std::integral_constant<int, 1>{});
         emax_lo = fmaxf(emax_lo, __shfl_sync(0xffffffffu, emax_row, lane & ~3));
         emax_hi = fmaxf(emax_hi, __shfl_sync(0xffffffffu, emax_row, (lane & ~3) | 2));
     } else {
