@@ -268,9 +268,9 @@ def step_method_bytes():
 # lines only: comments and blank lines are left out): once the code of a file
 # of the kernel changes, the figure is reported as null until the next capture.
 NCU_TRAFFIC = {
-    "bwd_query_mma": {"bytes_at_b32": 165817600 + 34578944,
+    "bwd_query_mma": {"bytes_at_b32": 165865728 + 34423040,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "f26ab4bf0a4909d64b35f8c4d74470c5c254896408b22636f16aabc43cf89a4c"},
+                      "sha256": "4d61b595507d055ae3581e4acfe993135787e966f3d97f3fb89476756504ee0e"},
     "bwd_key_mma": {"bytes_at_b32": 104528640 + 36358400,
                     "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
                     "sha256": "fa0f295cc49f2f2944012800d4c8fc99cdae1c71abb60604c1c90cbb78907148"},
