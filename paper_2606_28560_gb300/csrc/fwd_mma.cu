@@ -341,7 +341,8 @@ fwd_mma_kernel(const __grid_constant__ RowMaps tmK, const __grid_constant__ RowM
     // ---- rung scores (log2 units) of the rows this lane takes part in
     const float inv_sc2 = 1.f / sc2;
     // SAVE: the residual arrays of this head, addressed by 32-bit offsets
-    // (S T and K T stay below 2^31); row qhi = qlo + 8 is 8 entries on
+    // (S T <= 33 x 2^20 with W, K <= 16 and T <= 2^20); row qhi = qlo + 8 is 8
+    // entries on
     float* Pg = SAVE ? a.res_P + (size_t)bh * a.S * s.T : nullptr;   // residual exp(s - max) per slot
     float* SDg = SAVE ? a.res_sd + (size_t)bh * a.r.K * s.T : nullptr;
     float rs[kMmaMaxRungs][2];
