@@ -270,13 +270,13 @@ def step_method_bytes():
 NCU_TRAFFIC = {
     "bwd_query_mma": {"bytes_at_b32": 165865728 + 34423040,
                       "sources": ("bwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                      "sha256": "4d61b595507d055ae3581e4acfe993135787e966f3d97f3fb89476756504ee0e"},
+                      "sha256": "b200e61a7c2718d93368c317cf0bc8c056fae5f1aeb7699de3da502589b892ee"},
     "bwd_key_mma": {"bytes_at_b32": 104528640 + 36358400,
                     "sources": ("bwd_key_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-                    "sha256": "fa0f295cc49f2f2944012800d4c8fc99cdae1c71abb60604c1c90cbb78907148"},
+                    "sha256": "73f3bd8d30f5d7b450147f07b9118be3981338e5afd560b7cbc599c314caa730"},
     "fwd": {"bytes_at_b32": 100805632 + 57507584,
             "sources": ("fwd_mma.cu", "mma_common.cuh", "fwd_mma.cuh", "fibattn_internal.cuh"),
-            "sha256": "2f780130e04b0e375c268701fe84957643af88ee457a2fe6cf9a75df59879d68"},
+            "sha256": "69c9b864ca4eec6a2feb267f6b72a25de32b0681fa874692afc5e807f9d29d48"},
 }
 
 

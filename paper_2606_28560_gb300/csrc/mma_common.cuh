@@ -111,7 +111,6 @@ __device__ __forceinline__ unsigned pack_bf16(float lo, float hi) {
     __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<unsigned*>(&h);
 }
-__device__ __forceinline__ float bf16_round(float x) { return __bfloat162float(__float2bfloat16_rn(x)); }
 
 // Two bf16 ones: a B fragment of all ones makes an MMA return the row sums
 // of its A operand (exactly the rounded entries the value product uses).
