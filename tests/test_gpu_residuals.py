@@ -245,6 +245,19 @@ def test_random_shapes_forward_and_backward_from_residuals(case):
     _check_bwd_residuals(q, k, v, g, alpha, f, W, dedup)
 
 
+@pytest.mark.parametrize("base,K", [("fib", 15), ("pow2", 10)])
+def test_config5_training_path_mid_layer(base, K):
+    """Config 5 (B=2 H=8 T=16384 W=12, linear stagger) through the path the
+    long-sequence benchmark times -- the forward keeps its rotated keys and
+    residuals, the backward reads them -- at the mid-ramp layer 7 (alpha
+    0.9667), every gradient and dtheta against the oracle."""
+    alpha = float(fa.alpha_schedule("linear", 16)[7])
+    s = inputs.layer_seed(4, 7)
+    q, k, v = inputs.qkv(2, 8, 16384, seed=s, dtype=torch.bfloat16)
+    g = inputs.dout(2, 8, 16384, seed=s, dtype=torch.bfloat16)
+    _check_bwd_residuals(q, k, v, g, alpha, fa.base(base, K), 12)
+
+
 @pytest.mark.parametrize("layer", [0, 7, 12, 15])
 def test_config4_training_path_full(layer):
     """Config 4 (B=16 H=8 T=1024 W=8, learned theta seed 3) through the path the
