@@ -258,6 +258,19 @@ def test_config5_training_path_mid_layer(base, K):
     _check_bwd_residuals(q, k, v, g, alpha, fa.base(base, K), 12)
 
 
+def test_gqa_training_path_bench_shape():
+    """The grouped-query step the benchmark times (B=16 H=8 Hkv=2 T=1024 W=8,
+    learned theta seed 3; the key pass takes one block per pass there, its
+    grid being under two waves) through the residual path, layer 7, against
+    the oracle."""
+    theta = inputs.theta_learned(16, seed=3)
+    alpha = float(fa.alpha_schedule("learned", 16, theta=theta)[7])
+    s = inputs.layer_seed(3, 7)
+    q, k, v = inputs.qkv(16, 8, 1024, seed=s, dtype=torch.bfloat16, Hkv=2)
+    g = inputs.dout(16, 8, 1024, seed=s, dtype=torch.bfloat16)
+    _check_bwd_residuals(q, k, v, g, alpha, fa.base("fib", 15), 8)
+
+
 @pytest.mark.parametrize("layer", [0, 7, 12, 15])
 def test_config4_training_path_full(layer):
     """Config 4 (B=16 H=8 T=1024 W=8, learned theta seed 3) through the path the
